@@ -1,0 +1,215 @@
+/*
+ * isam_oracle.c -- plain, slow, fp64 CPU oracle for the matrix-multiplication
+ * hot path of "ISA Mapper: A Compute and Hardware Agnostic Deep Learning
+ * Compiler" (Sotoudeh et al., SysML 2019).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the library's product path may link,
+ * load or call this file; only the tests, the smoke check and the benchmark's
+ * CPU-baseline leg do.  It shares no code, header or constant with the CUDA
+ * path.
+ *
+ * Conventions
+ *   - bf16 operands arrive as their uint16 bit patterns and are widened
+ *     exactly to double (the pattern is the top half of an IEEE float32).
+ *   - fp32 operands are widened exactly to double.
+ *   - All arithmetic is double precision, each sum taken in increasing order of
+ *     its reduction index; the file is compiled with -ffp-contract=off so the
+ *     compiler fuses nothing.
+ *   - Matrices are row-major and packed.
+ *   - Parallelism (OpenMP) is only over independent output elements; it never
+ *     changes an output's arithmetic.
+ *
+ * Return value of every entry: 0 on success, 1 on an invalid argument.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+static double bf(uint16_t bits) {
+    uint32_t u = (uint32_t)bits << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+int oracle_num_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/*
+ * GEMM, Listing 1 (the matmul loop nest) and Listing 4 (its three-operand
+ * form: tmp := A[i][k]; tmp *= B[k][j]; C[i][j] += tmp):
+ *
+ *   C_out[i][j] = alpha * sum_{k=0..K-1} opA[i][k] * opB[k][j] + beta * C_in[i][j]
+ *
+ * opA[i][k] = A[i*K + k] (transA = 0, A stored M x K) or A[k*M + i] (transA = 1).
+ * opB[k][j] = B[k*N + j] (transB = 0, B stored K x N) or B[j*K + k] (transB = 1).
+ * With beta == 0 C_in is not read (BLAS convention) and may be NULL.
+ *
+ * rows / nrows select which rows i of C to compute (rows == NULL: all M rows,
+ * in order).  C_out has nrows x N entries (row r of C_out is row rows[r]).
+ */
+int oracle_gemm_rows(int M, int N, int K, int transA, int transB, double alpha,
+                     const uint16_t *A, const uint16_t *B, double beta,
+                     const float *C_in, int nrows, const int *rows, double *C_out) {
+    if (M < 1 || N < 1 || K < 1 || !A || !B || !C_out) return 1;
+    if (beta != 0.0 && !C_in) return 1;
+    if (!rows) nrows = M;
+    for (int r = 0; rows && r < nrows; ++r)
+        if (rows[r] < 0 || rows[r] >= M) return 1;
+
+#pragma omp parallel
+    {
+        double *acc = (double *)malloc(sizeof(double) * (size_t)N);
+#pragma omp for schedule(dynamic, 1)
+        for (int r = 0; r < nrows; ++r) {
+            const int i = rows ? rows[r] : r;
+            for (int j = 0; j < N; ++j) acc[j] = 0.0;
+            for (int k = 0; k < K; ++k) {
+                const double a = transA ? bf(A[(size_t)k * M + i]) : bf(A[(size_t)i * K + k]);
+                if (transB) {
+                    for (int j = 0; j < N; ++j) acc[j] += a * bf(B[(size_t)j * K + k]);
+                } else {
+                    const uint16_t *brow = B + (size_t)k * N;
+                    for (int j = 0; j < N; ++j) acc[j] += a * bf(brow[j]);
+                }
+            }
+            double *out = C_out + (size_t)r * N;
+            for (int j = 0; j < N; ++j) {
+                double v = alpha * acc[j];
+                if (beta != 0.0) v += beta * (double)C_in[(size_t)i * N + j];
+                out[j] = v;
+            }
+        }
+        free(acc);
+    }
+    return 0;
+}
+
+int oracle_gemm(int M, int N, int K, int transA, int transB, double alpha,
+                const uint16_t *A, const uint16_t *B, double beta,
+                const float *C_in, double *C_out) {
+    return oracle_gemm_rows(M, N, K, transA, transB, alpha, A, B, beta, C_in,
+                            M, NULL, C_out);
+}
+
+static double sigmoid(double v) { return 1.0 / (1.0 + exp(-v)); }
+
+/*
+ * GRU forward over T steps (Section 3.6, recurrent scheduling; Section 5.1.2,
+ * a GRU over 128 steps).  The paper names the cell but not its equations; this
+ * is the gate-order (r, z, n) form whose recurrent product is one fused
+ * 3H-wide matrix product per step, with the reset gate applied after that
+ * product:
+ *
+ *   gx = W x_t + b_ih                    (3H; rows r | z | n)
+ *   gh = U h_{t-1} + b_hh                (3H)
+ *   r  = sigmoid(gx_r + gh_r)
+ *   z  = sigmoid(gx_z + gh_z)
+ *   n  = tanh(gx_n + r * gh_n)
+ *   h_t = (1 - z) * n + z * h_{t-1}
+ *
+ * x [T][batch][H] bf16, W and U [3H][H] bf16 (row = output unit, col = input),
+ * b [6H] fp32 = b_ih then b_hh, h0 [batch][H] fp32 or NULL (zeros),
+ * h_out [T][batch][H] double (every step's hidden state).
+ * Sequences in a batch are independent; the loop over them is parallel.
+ */
+int oracle_gru_forward(int T, int batch, int H, const uint16_t *x, const uint16_t *W,
+                       const uint16_t *U, const float *b, const float *h0, double *h_out) {
+    if (T < 1 || batch < 1 || H < 1 || !x || !W || !U || !b || !h_out) return 1;
+    const int G = 3 * H;
+#pragma omp parallel
+    {
+        double *h = (double *)malloc(sizeof(double) * (size_t)H);
+        double *hn = (double *)malloc(sizeof(double) * (size_t)H);
+        double *gx = (double *)malloc(sizeof(double) * (size_t)G);
+        double *gh = (double *)malloc(sizeof(double) * (size_t)G);
+#pragma omp for schedule(dynamic, 1)
+        for (int s = 0; s < batch; ++s) {
+            for (int j = 0; j < H; ++j) h[j] = h0 ? (double)h0[(size_t)s * H + j] : 0.0;
+            for (int t = 0; t < T; ++t) {
+                const uint16_t *xt = x + ((size_t)t * batch + s) * H;
+                for (int g = 0; g < G; ++g) {
+                    double ax = 0.0, ah = 0.0;
+                    const uint16_t *wr = W + (size_t)g * H;
+                    const uint16_t *ur = U + (size_t)g * H;
+                    for (int k = 0; k < H; ++k) ax += bf(wr[k]) * bf(xt[k]);
+                    for (int k = 0; k < H; ++k) ah += bf(ur[k]) * h[k];
+                    gx[g] = ax + (double)b[g];
+                    gh[g] = ah + (double)b[G + g];
+                }
+                double *ho = h_out + ((size_t)t * batch + s) * H;
+                for (int j = 0; j < H; ++j) {
+                    const double r = sigmoid(gx[j] + gh[j]);
+                    const double z = sigmoid(gx[H + j] + gh[H + j]);
+                    const double n = tanh(gx[2 * H + j] + r * gh[2 * H + j]);
+                    hn[j] = (1.0 - z) * n + z * h[j];
+                    ho[j] = hn[j];
+                }
+                double *tmp = h; h = hn; hn = tmp;
+            }
+        }
+        free(h); free(hn); free(gx); free(gh);
+    }
+    return 0;
+}
+
+/*
+ * Separable depthwise convolution, Listing 3, with stride s = 1, channel
+ * multiplier c = 1 (so r = 0 and P is indexed P[q][k]) and a zero border of
+ * one pixel (input row i + di - 1, column j + dj - 1), taken in the factored
+ * form the paper's factorisation pass produces (Section 2.3): the
+ * D-weighted window sum over (di, dj) is formed first, then multiplied by P
+ * and summed over q:
+ *
+ *   Y[b][i][j][q] = sum_{di,dj in 0..2} X[b][i+di-1][j+dj-1][q] * D[di][dj][q]
+ *   C[b][i][j][k] = sum_{q} Y[b][i][j][q] * P[q][k]
+ *
+ * x NHWC [N][H][W][Cin] bf16, dw [3][3][Cin] bf16, pw [Cin][Cout] bf16,
+ * out NHWC [N][H][W][Cout] double.  No rounding between the two stages.
+ */
+int oracle_dwsep(int N, int H, int W, int Cin, int Cout, const uint16_t *x,
+                 const uint16_t *dw, const uint16_t *pw, double *out) {
+    if (N < 1 || H < 1 || W < 1 || Cin < 1 || Cout < 1 || !x || !dw || !pw || !out) return 1;
+    const long npix = (long)N * H * W;
+#pragma omp parallel
+    {
+        double *y = (double *)malloc(sizeof(double) * (size_t)Cin);
+#pragma omp for schedule(static)
+        for (long p = 0; p < npix; ++p) {
+            const int b = (int)(p / ((long)H * W));
+            const int i = (int)((p / W) % H);
+            const int j = (int)(p % W);
+            for (int q = 0; q < Cin; ++q) {
+                double s = 0.0;
+                for (int di = 0; di < 3; ++di) {
+                    const int ii = i + di - 1;
+                    if (ii < 0 || ii >= H) continue;
+                    for (int dj = 0; dj < 3; ++dj) {
+                        const int jj = j + dj - 1;
+                        if (jj < 0 || jj >= W) continue;
+                        s += bf(x[(((size_t)b * H + ii) * W + jj) * Cin + q]) *
+                             bf(dw[((size_t)di * 3 + dj) * Cin + q]);
+                    }
+                }
+                y[q] = s;
+            }
+            double *o = out + (size_t)p * Cout;
+            for (int k = 0; k < Cout; ++k) {
+                double s = 0.0;
+                for (int q = 0; q < Cin; ++q) s += y[q] * bf(pw[(size_t)q * Cout + k]);
+                o[k] = s;
+            }
+        }
+        free(y);
+    }
+    return 0;
+}

@@ -1,0 +1,291 @@
+"""Pins the fp64 oracle to facts that do not come from the oracle itself:
+brute force on tiny inputs, exact integer arithmetic, identity and permutation
+matrices, closed forms of the GRU recurrence, the boundary pattern of the 3x3
+window, and independent library routines (numpy / torch float64).
+
+Each pin is chosen so that a plausible slip in the oracle (a dropped term, a
+swapped index or operand, a wrong sign, a bias in the wrong place) fails it.
+"""
+import math
+
+import numpy as np
+import pytest
+
+from paper_1810_09958_gb300 import synth
+
+
+def f64(bits):
+    return synth.bf16_bits_to_f64(bits)
+
+
+def opA(A, M, K, transA):
+    a = f64(A)
+    return a.reshape(K, M).T if transA else a.reshape(M, K)
+
+
+def opB(B, K, N, transB):
+    b = f64(B)
+    return b.reshape(N, K).T if transB else b.reshape(K, N)
+
+
+# --------------------------------------------------------------------------
+# GEMM (Listing 1 / Listing 4)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("transA", [0, 1])
+@pytest.mark.parametrize("transB", [0, 1])
+def test_gemm_bruteforce_tiny(oracle_lib, transA, transB):
+    rng = np.random.default_rng(7)
+    for trial in range(6):
+        M, N, K = (int(v) for v in rng.integers(1, 34, size=3))
+        A, B, C = synth.gemm_operands(M, N, K, transA, transB, seed=100 + trial, beta_c=True)
+        alpha, beta = 1.5, -0.75
+        got = oracle_lib.gemm(M, N, K, transA, transB, alpha, A, B, beta, C)
+        a, b = opA(A, M, K, transA), opB(B, K, N, transB)
+        for i in range(M):
+            for j in range(N):
+                s = 0.0
+                for k in range(K):
+                    s += float(a[i, k]) * float(b[k, j])
+                want = alpha * s + beta * float(C[i, j])
+                assert got[i, j] == want, (M, N, K, i, j)
+
+
+def test_gemm_integer_exact(oracle_lib):
+    for transA in (0, 1):
+        M, N, K = 37, 19, 301
+        A, B, C = synth.gemm_operands(M, N, K, transA, 0, seed=11, dist="int4", beta_c=True)
+        ai = opA(A, M, K, transA).astype(np.int64)
+        bi = opB(B, K, N, 0).astype(np.int64)
+        got = oracle_lib.gemm(M, N, K, transA, 0, 1.0, A, B)
+        assert np.array_equal(got, (ai @ bi).astype(np.float64))
+        # alpha = 2, beta = -1 closed form on integers.
+        got2 = oracle_lib.gemm(M, N, K, transA, 0, 2.0, A, B, -1.0, C)
+        want2 = 2 * (ai @ bi) - C.astype(np.int64)
+        assert np.array_equal(got2, want2.astype(np.float64))
+
+
+def test_gemm_identity_and_permutation(oracle_lib):
+    M, K = 23, 40
+    A, _, _ = synth.gemm_operands(M, K, K, 0, 0, seed=5)
+    eye = synth.to_bf16_bits(np.eye(K))
+    got = oracle_lib.gemm(M, K, K, 0, 0, 1.0, A, eye)
+    assert np.array_equal(got, f64(A).reshape(M, K))
+    perm = np.random.default_rng(3).permutation(K)
+    P = np.zeros((K, K))
+    P[perm, np.arange(K)] = 1.0          # column j of A @ P is column perm[j] of A
+    got = oracle_lib.gemm(M, K, K, 0, 0, 1.0, A, synth.to_bf16_bits(P))
+    assert np.array_equal(got, f64(A).reshape(M, K)[:, perm])
+    # Same through the transposed-A path: I @ A^T stored K x M.
+    At = np.ascontiguousarray(A.reshape(M, K).T)
+    got = oracle_lib.gemm(M, K, K, 1, 0, 1.0, At, eye)
+    assert np.array_equal(got, f64(A).reshape(M, K))
+    # Left identity through transB: A = I_M @ A with A read as B^T.
+    eyeM = synth.to_bf16_bits(np.eye(M))
+    got = oracle_lib.gemm(M, K, M, 0, 1, 1.0, eyeM, At)
+    assert np.array_equal(got, f64(A).reshape(M, K))
+
+
+def test_gemm_beta_zero_ignores_c(oracle_lib):
+    M, N, K = 8, 9, 10
+    A, B, _ = synth.gemm_operands(M, N, K, 0, 0, seed=9)
+    Cnan = np.full((M, N), np.nan, dtype=np.float32)
+    got = oracle_lib.gemm(M, N, K, 0, 0, 1.0, A, B, 0.0, Cnan)
+    assert np.isfinite(got).all()
+
+
+def test_gemm_vs_numpy_float64(oracle_lib):
+    for transA, transB in ((0, 0), (1, 0), (0, 1)):
+        M, N, K = 130, 70, 257
+        A, B, C = synth.gemm_operands(M, N, K, transA, transB, seed=21, beta_c=True)
+        got = oracle_lib.gemm(M, N, K, transA, transB, 0.5, A, B, 2.0, C)
+        want = 0.5 * (opA(A, M, K, transA) @ opB(B, K, N, transB)) + 2.0 * C.astype(np.float64)
+        assert np.max(np.abs(got - want)) <= 1e-12 * np.max(np.abs(want))
+
+
+def test_gemm_rows_subset_matches_full(oracle_lib):
+    M, N, K = 50, 33, 64
+    A, B, C = synth.gemm_operands(M, N, K, 1, 0, seed=31, beta_c=True)
+    full = oracle_lib.gemm(M, N, K, 1, 0, 1.0, A, B, 1.0, C)
+    rows = np.array([49, 0, 17, 17, 3])
+    sub = oracle_lib.gemm(M, N, K, 1, 0, 1.0, A, B, 1.0, C, rows=rows)
+    assert np.array_equal(sub, full[rows])
+
+
+def test_gemm_rejects_bad_args(oracle_lib):
+    A = np.zeros(4, np.uint16)
+    with pytest.raises(ValueError):
+        oracle_lib.gemm(2, 2, 2, 0, 0, 1.0, A, A, 1.0, None)   # beta != 0 needs C
+
+
+# --------------------------------------------------------------------------
+# GRU (Section 3.6 recurrent scheduling; Section 5.1.2)
+# --------------------------------------------------------------------------
+def sig(v):
+    return 1.0 / (1.0 + np.exp(-v))
+
+
+def test_gru_zero_weights_closed_form(oracle_lib):
+    """W = U = 0: r, z, n are constants from the biases and
+    h_t = n + z**t * (h0 - n) (geometric decay towards n)."""
+    T, batch, H = 9, 3, 16
+    zero = np.zeros((3 * H, H), np.uint16)
+    x = synth.bf16_normal(1, (T, batch, H))
+    b = synth.f32_uniform(2, (6 * H,), -2.0, 2.0)
+    h0 = synth.f32_uniform(3, (batch, H))
+    got = oracle_lib.gru_forward(x, zero, zero, b, h0)
+    bd = b.astype(np.float64)
+    r = sig(bd[0:H] + bd[3 * H:4 * H])
+    z = sig(bd[H:2 * H] + bd[4 * H:5 * H])
+    n = np.tanh(bd[2 * H:3 * H] + r * bd[5 * H:6 * H])
+    for t in range(T):
+        want = n[None, :] + z[None, :] ** (t + 1) * (h0.astype(np.float64) - n[None, :])
+        np.testing.assert_allclose(got[t], want, rtol=0, atol=1e-14)
+
+
+def test_gru_saturated_update_gate_keeps_h0(oracle_lib):
+    """b_z = +30 drives z to 1 - 9.4e-14, so h_t stays at h0."""
+    T, batch, H = 12, 2, 32
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=4)
+    b = b.copy()
+    b[H:2 * H] = 30.0
+    h0 = synth.f32_uniform(5, (batch, H))
+    got = oracle_lib.gru_forward(x, W, U, b, h0)
+    for t in range(T):
+        np.testing.assert_allclose(got[t], h0.astype(np.float64), rtol=0, atol=1e-11)
+
+
+def test_gru_matches_torch_float64(oracle_lib):
+    """torch.nn.GRU uses the same (r, z, n) order with the reset gate applied
+    after the recurrent product, so it is an independent implementation."""
+    torch = pytest.importorskip("torch")
+    T, batch, H = 7, 4, 24
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=8)
+    h0 = synth.f32_uniform(9, (batch, H))
+    got = oracle_lib.gru_forward(x, W, U, b, h0)
+    gru = torch.nn.GRU(H, H, num_layers=1, bias=True).double()
+    with torch.no_grad():
+        gru.weight_ih_l0.copy_(torch.from_numpy(f64(W)))
+        gru.weight_hh_l0.copy_(torch.from_numpy(f64(U)))
+        gru.bias_ih_l0.copy_(torch.from_numpy(b[:3 * H].astype(np.float64)))
+        gru.bias_hh_l0.copy_(torch.from_numpy(b[3 * H:].astype(np.float64)))
+        out, hT = gru(torch.from_numpy(f64(x)), torch.from_numpy(h0.astype(np.float64))[None])
+    np.testing.assert_allclose(got, out.numpy(), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(got[-1], hT[0].numpy(), rtol=0, atol=1e-12)
+
+
+def test_gru_single_step_from_zero_state(oracle_lib):
+    """T = 1 and h0 = 0: the recurrent product vanishes, so h_1 = (1 - z) n with
+    every gate a function of W x + biases alone (one GEMM, numpy's)."""
+    T, batch, H = 1, 5, 16
+    x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=12)
+    got = oracle_lib.gru_forward(x, W, U, b, h0)
+    gx = f64(x[0]) @ f64(W).T + b[:3 * H].astype(np.float64)
+    bh = b[3 * H:].astype(np.float64)
+    r = sig(gx[:, :H] + bh[:H])
+    z = sig(gx[:, H:2 * H] + bh[H:2 * H])
+    n = np.tanh(gx[:, 2 * H:] + r * bh[2 * H:])
+    np.testing.assert_allclose(got[0], (1 - z) * n, rtol=0, atol=1e-14)
+
+
+def test_gru_batch_rows_independent(oracle_lib):
+    T, batch, H = 5, 6, 16
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=14)
+    h0 = synth.f32_uniform(15, (batch, H))
+    full = oracle_lib.gru_forward(x, W, U, b, h0)
+    sel = [4, 1]
+    sub = oracle_lib.gru_forward(np.ascontiguousarray(x[:, sel]), W, U, b, h0[sel])
+    assert np.array_equal(sub, full[:, sel])
+
+
+# --------------------------------------------------------------------------
+# Separable depthwise convolution (Listing 3, factorisation of Section 2.3)
+# --------------------------------------------------------------------------
+def test_dwsep_literal_listing_loop(oracle_lib):
+    """The unfactored 8-deep loop of Listing 3 (s = 1, c = 1, zero border of
+    one pixel), brute force on a tiny case, equals the factored oracle."""
+    N, H, W, Cin, Cout = 2, 4, 5, 3, 4
+    x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=17)
+    X, D, P = f64(x), f64(dw), f64(pw)
+    want = np.zeros((N, H, W, Cout))
+    for b in range(N):
+        for i in range(H):
+            for j in range(W):
+                for k in range(Cout):
+                    for di in range(3):
+                        for dj in range(3):
+                            for q in range(Cin):
+                                for r in range(1):
+                                    ii, jj = i + di - 1, j + dj - 1
+                                    if 0 <= ii < H and 0 <= jj < W:
+                                        want[b, i, j, k] += X[b, ii, jj, q] * D[di, dj, q] * P[q + r, k]
+    got = oracle_lib.dwsep(x, dw, pw)
+    np.testing.assert_allclose(got, want, rtol=1e-13, atol=1e-15)
+
+
+def test_dwsep_delta_kernel_is_pointwise_gemm(oracle_lib):
+    N, H, W, Cin, Cout = 2, 6, 7, 16, 24
+    x, _, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=19)
+    D = np.zeros((3, 3, Cin))
+    D[1, 1, :] = 1.0
+    got = oracle_lib.dwsep(x, synth.to_bf16_bits(D), pw)
+    want = f64(x).reshape(-1, Cin) @ f64(pw)
+    np.testing.assert_allclose(got.reshape(-1, Cout), want, rtol=1e-13, atol=1e-15)
+
+
+def test_dwsep_ones_window_boundary_pattern(oracle_lib):
+    """All-ones 3x3 window on a constant image, identity pointwise: 9c inside,
+    6c on edges, 4c in corners (exact)."""
+    N, H, W, C = 1, 5, 6, 8
+    c = 1.5
+    x = synth.to_bf16_bits(np.full((N, H, W, C), c))
+    D = synth.to_bf16_bits(np.ones((3, 3, C)))
+    P = synth.to_bf16_bits(np.eye(C))
+    got = oracle_lib.dwsep(x, D, P)[0, :, :, 0]
+    rows = np.array([2] + [3] * (H - 2) + [2])
+    cols = np.array([2] + [3] * (W - 2) + [2])
+    assert np.array_equal(got, c * np.outer(rows, cols))
+
+
+def test_dwsep_integer_exact(oracle_lib):
+    N, H, W, Cin, Cout = 1, 7, 9, 16, 8
+    x = synth.bf16_integers(31, (N, H, W, Cin), -3, 3)
+    dw = synth.bf16_integers(32, (3, 3, Cin), -2, 2)
+    pw = synth.bf16_integers(33, (Cin, Cout), -2, 2)
+    X = np.pad(f64(x).astype(np.int64), ((0, 0), (1, 1), (1, 1), (0, 0)))
+    D = f64(dw).astype(np.int64)
+    Y = np.zeros((N, H, W, Cin), np.int64)
+    for di in range(3):
+        for dj in range(3):
+            Y += X[:, di:di + H, dj:dj + W, :] * D[di, dj]
+    want = (Y.reshape(-1, Cin) @ f64(pw).astype(np.int64)).reshape(N, H, W, Cout)
+    assert np.array_equal(oracle_lib.dwsep(x, dw, pw), want.astype(np.float64))
+
+
+def test_dwsep_matches_torch_conv_float64(oracle_lib):
+    torch = pytest.importorskip("torch")
+    F = torch.nn.functional
+    N, H, W, Cin, Cout = 2, 9, 8, 16, 32
+    x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=41)
+    xt = torch.from_numpy(f64(x)).permute(0, 3, 1, 2)                  # NCHW
+    wd = torch.from_numpy(f64(dw)).permute(2, 0, 1).unsqueeze(1)       # [Cin,1,3,3]
+    wp = torch.from_numpy(f64(pw)).t().reshape(Cout, Cin, 1, 1)
+    y = F.conv2d(F.conv2d(xt, wd, padding=1, groups=Cin), wp)
+    want = y.permute(0, 2, 3, 1).numpy()
+    np.testing.assert_allclose(oracle_lib.dwsep(x, dw, pw), want, rtol=0, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# Input generator sanity (it feeds both sides)
+# --------------------------------------------------------------------------
+def test_splitmix64_reference_values():
+    """First outputs of SplitMix64 seeded with 0 (published reference values
+    of the generator as defined by Steele, Lea and Flood / Vigna)."""
+    z = synth.splitmix64(0, 0, 3)
+    assert [int(v) for v in z] == [0xE220A8397B1DCDAF, 0x6E789E6AA1B965F4, 0x06C45D188009454F]
+
+
+def test_bf16_rounding_is_nearest_even():
+    vals = np.array([1.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -2.5, 1.0 + 2 ** -9], dtype=np.float32)
+    bits = synth.to_bf16_bits(vals)
+    back = synth.bf16_bits_to_f32(bits)
+    assert back.tolist() == [1.0, 1.0, 1.0 + 2 ** -6, -2.5, 1.0]
