@@ -1,0 +1,160 @@
+/*
+ * isam.h -- C ABI of the GB300 (sm_103a) matrix-multiplication hot path
+ * extracted and scheduled by the ISA Mapper (Sotoudeh et al., "ISA Mapper: A
+ * Compute and Hardware Agnostic Deep Learning Compiler", SysML 2019).
+ *
+ * Library: libisam.so.  Plain C types only: sizes are int, scalars float,
+ * bf16 tensors are passed as pointers to their 16-bit patterns (isam_bf16,
+ * IEEE bfloat16, round-to-nearest-even where the caller rounds).
+ *
+ * Memory and ownership
+ *   - Every tensor pointer is a DEVICE pointer on the current CUDA device,
+ *     allocated and owned by the caller.  The library never frees or keeps
+ *     them past the call's completion on the stream.
+ *   - Tensors are packed row-major (no leading-dimension arguments).
+ *   - The library owns small internal workspaces (an error word per device,
+ *     the GRU's input-projection buffer, its hidden-state exchange buffer and
+ *     step counter).  They are allocated on first use, reused, and released
+ *     by isam_shutdown().
+ *
+ * Execution
+ *   - Every compute call is asynchronous on the stream set by
+ *     isam_set_stream() (default: the legacy default stream) and returns
+ *     after the launch.  Argument errors are reported at once and nothing is
+ *     launched.  Device-side failures (a bounded wait that ran out) are
+ *     reported by the next isam_sync().
+ *   - Every spin-wait inside the kernels is bounded in time (default 2 s,
+ *     ISAM_WAIT_TIMEOUT_MS in the environment overrides); a wait that runs out
+ *     sets the device error word and the kernel returns.
+ *
+ * Status codes: every entry returns one of the ISAM_* codes below;
+ * isam_last_error_string() describes the last failure on the calling thread.
+ */
+#ifndef ISAM_H
+#define ISAM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t isam_bf16;
+
+enum {
+    ISAM_OK = 0,
+    ISAM_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, bad flag     */
+    ISAM_ERR_UNSUPPORTED = 2, /* valid but outside the supported shapes/aligns */
+    ISAM_ERR_CUDA = 3,        /* a CUDA runtime or driver call failed          */
+    ISAM_ERR_TIMEOUT = 4      /* a bounded device wait ran out (see isam_sync) */
+};
+
+/* Version of this ABI (major * 100 + minor). */
+int isam_version(void);
+
+/* Stream for subsequent calls from any thread: a cudaStream_t passed as
+ * void*, or NULL for the legacy default stream.  Returns ISAM_OK. */
+int isam_set_stream(void *stream);
+
+/* Waits for the stream, then reads and clears the device error word.
+ * ISAM_OK, ISAM_ERR_TIMEOUT (a bounded wait ran out; outputs of the failed
+ * call are undefined) or ISAM_ERR_CUDA. */
+int isam_sync(void);
+
+/* Human-readable description of the last failure on this thread. */
+const char *isam_last_error_string(void);
+
+/* Releases every internal workspace on every device it was made on.  Waits
+ * for the device first.  Later calls allocate again. */
+int isam_shutdown(void);
+
+/*
+ * GEMM: C <- alpha * op(A) * op(B) + beta * C
+ *
+ * The computation of Listing 1 (C[i][j] += A[i][k] * B[k][j]) and its
+ * three-operand form in Listing 4, with BLAS scaling; the paper's GEMM
+ * benchmark (Section 5.1.1) runs it at DeepBench sizes.
+ *
+ *   op(A) is M x K: A stored M x K when transA == 0, K x M when transA == 1.
+ *   op(B) is K x N: B stored K x N when transB == 0, N x K when transB == 1.
+ *   A, B: bf16, C: fp32 (M x N), all row-major packed, device pointers.
+ *   Products are exact in fp32 and accumulated in fp32 (tensor cores).
+ *   beta == 0: C is write-only (never read, NaNs in it do not propagate).
+ *
+ * Supported: M, N, K >= 1; A and B 16-byte aligned; every stored row pitch a
+ * multiple of 16 bytes, i.e. K % 8 == 0 when transA == 0 or transB == 1,
+ * M % 8 == 0 when transA == 1, N % 8 == 0 when transB == 0; C 16-byte
+ * aligned.  Otherwise ISAM_ERR_UNSUPPORTED.
+ * ISAM_ERR_INVALID_ARG for null pointers, sizes < 1, trans flags not 0/1.
+ */
+int isam_gemm(int M, int N, int K, int transA, int transB, float alpha,
+              const isam_bf16 *A, const isam_bf16 *B, float beta, float *C);
+
+/*
+ * The tile plan isam_gemm would use for this problem, chosen by the
+ * library's analytic cost model (the paper's "Approach" interface for
+ * tiling and device-allocation choices, Sections 3.4 and 4).  Nothing is
+ * launched.  out (host, 6 ints): tile width BN (tile height is 128), split-K
+ * factor (CTAs of one cluster sharing a tile), shared-memory ring depth,
+ * rasterisation group height, persistent grid size, dynamic shared memory
+ * bytes.  Same argument checks as isam_gemm (pointers are not needed).
+ */
+int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta, int *out);
+
+/*
+ * GRU forward inference over T steps (input size == hidden).
+ *
+ * The recurrent model the paper schedules with a priming, a recursive and a
+ * finish iteration over persistent weights (Section 3.6) and benchmarks over
+ * 128 steps (Section 5.1.2).  The paper names the cell without equations;
+ * this library computes the (r, z, n) form with the reset gate applied after
+ * the recurrent product:
+ *
+ *   gx = W x_t + b_ih,  gh = U h_{t-1} + b_hh        (3H each, rows r|z|n)
+ *   r = sigmoid(gx_r + gh_r),  z = sigmoid(gx_z + gh_z)
+ *   n = tanh(gx_n + r * gh_n),  h_t = (1 - z) * n + z * h_{t-1}
+ *
+ *   x     [T][batch][hidden] bf16
+ *   W, U  [3*hidden][hidden] bf16 (row = output unit of gate r, z, then n)
+ *   b     [6*hidden] fp32: b_ih (3*hidden) then b_hh (3*hidden)
+ *   h0    [batch][hidden] fp32, or NULL for zeros
+ *   h_out [T][batch][hidden] fp32: every step's hidden state (h_T = h_out[T-1])
+ *
+ * The input projection for all T steps runs as one GEMM into a library
+ * workspace; the recurrence runs in one persistent kernel that keeps U
+ * resident in shared memory and multiplies bf16(h_{t-1}) on the tensor cores
+ * (h itself is carried in fp32).  Gates are evaluated in fp32.
+ *
+ * Supported: T >= 1, 1 <= batch <= 32, hidden a multiple of 128 with
+ * hidden <= 2048 (hidden / 16 cooperating CTAs must be co-resident); all
+ * pointers 16-byte aligned.  Otherwise ISAM_ERR_UNSUPPORTED.
+ */
+int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
+                     const isam_bf16 *W, const isam_bf16 *U, const float *b,
+                     const float *h0, float *h_out);
+
+/*
+ * Separable depthwise convolution, NHWC: a 3x3 depthwise stage (stride 1,
+ * zero border of one pixel, channel multiplier 1) followed by a pointwise
+ * 1x1 stage, i.e. Listing 3 with s = 1 and c = 1, executed in the factored
+ * form of Section 2.3: the depthwise sum feeds a GEMM with
+ * M = N*H*W, K = Cin, N = Cout.
+ *
+ *   x     [N][H][W][Cin] bf16
+ *   dw_w  [3][3][Cin] bf16   (D[di][dj][q])
+ *   pw_w  [Cin][Cout] bf16   (P[q][k])
+ *   out   [N][H][W][Cout] fp32
+ *
+ * The depthwise result is formed in fp32 and rounded to bf16 for the tensor
+ * cores; it never leaves the chip.
+ * Supported: Cin % 16 == 0, 16 <= Cin <= 256, Cout % 16 == 0,
+ * 16 <= Cout <= 256; pointers 16-byte aligned.  Otherwise
+ * ISAM_ERR_UNSUPPORTED.
+ */
+int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
+                    const isam_bf16 *dw_w, const isam_bf16 *pw_w, float *out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ISAM_H */

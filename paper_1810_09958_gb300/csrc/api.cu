@@ -1,0 +1,289 @@
+// api.cu -- the extern "C" boundary of libisam.so (declared in include/isam.h):
+// argument checking, per-device state and workspaces, the stream, the device
+// error word, and TMA descriptor encoding.
+#include <cudaTypedefs.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "internal.h"
+
+namespace isam {
+
+namespace {
+
+thread_local char t_err[512] = "no error";
+std::mutex g_mu;
+cudaStream_t g_stream = nullptr;
+constexpr int kMaxDevices = 64;
+DeviceState *g_dev[kMaxDevices] = {};
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+struct TmapEntry {
+    uint64_t key[12];
+    CUtensorMap map;
+    bool used;
+};
+constexpr int kTmapCache = 128;
+TmapEntry g_tmaps[kTmapCache];
+int g_tmap_next = 0;
+std::mutex g_tmap_mu;
+
+int get_encoder() {
+    if (g_encode) return ISAM_OK;
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                     cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn)
+        return set_error(ISAM_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    return ISAM_OK;
+}
+
+int encode(CUtensorMap *out, const uint64_t key[12], cuuint32_t rank, const void *base,
+           const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box) {
+    {
+        std::lock_guard<std::mutex> lk(g_tmap_mu);
+        for (int i = 0; i < kTmapCache; ++i)
+            if (g_tmaps[i].used && memcmp(g_tmaps[i].key, key, sizeof(uint64_t) * 12) == 0) {
+                *out = g_tmaps[i].map;
+                return ISAM_OK;
+            }
+    }
+    int rc = get_encoder();
+    if (rc) return rc;
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = g_encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), dims,
+                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return set_error(ISAM_ERR_UNSUPPORTED, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+    std::lock_guard<std::mutex> lk(g_tmap_mu);
+    TmapEntry &e = g_tmaps[g_tmap_next];
+    g_tmap_next = (g_tmap_next + 1) % kTmapCache;
+    memcpy(e.key, key, sizeof(uint64_t) * 12);
+    e.map = *out;
+    e.used = true;
+    return ISAM_OK;
+}
+
+}  // namespace
+
+int set_error(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(t_err, sizeof t_err, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_error(cudaError_t e, const char *what) {
+    return set_error(ISAM_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+cudaStream_t current_stream() {
+    std::lock_guard<std::mutex> lk(g_mu);
+    return g_stream;
+}
+
+unsigned long long wait_timeout_ns() {
+    static unsigned long long v = [] {
+        const char *s = getenv("ISAM_WAIT_TIMEOUT_MS");
+        long ms = s ? strtol(s, nullptr, 10) : 2000;
+        if (ms < 1) ms = 1;
+        if (ms > 60000) ms = 60000;
+        return static_cast<unsigned long long>(ms) * 1000000ull;
+    }();
+    return v;
+}
+
+DeviceState *device_state(int *status) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        *status = cuda_error(e, "cudaGetDevice");
+        return nullptr;
+    }
+    if (dev < 0 || dev >= kMaxDevices) {
+        *status = set_error(ISAM_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+        return nullptr;
+    }
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (g_dev[dev]) {
+        *status = ISAM_OK;
+        return g_dev[dev];
+    }
+    cudaDeviceProp prop;
+    if ((e = cudaGetDeviceProperties(&prop, dev)) != cudaSuccess) {
+        *status = cuda_error(e, "cudaGetDeviceProperties");
+        return nullptr;
+    }
+    if (prop.major != 10 || prop.minor != 3) {
+        *status = set_error(ISAM_ERR_UNSUPPORTED,
+                            "libisam is built for sm_103a (GB300); device %d is sm_%d%d", dev,
+                            prop.major, prop.minor);
+        return nullptr;
+    }
+    auto *ds = new DeviceState();
+    ds->device = dev;
+    ds->num_sms = prop.multiProcessorCount;
+    ds->max_smem_optin = static_cast<int>(prop.sharedMemPerBlockOptin);
+    if ((e = cudaMalloc(&ds->err_word, 16)) != cudaSuccess ||
+        (e = cudaMemset(ds->err_word, 0, 16)) != cudaSuccess) {
+        *status = cuda_error(e, "allocating the device error word");
+        delete ds;
+        return nullptr;
+    }
+    g_dev[dev] = ds;
+    *status = ISAM_OK;
+    return ds;
+}
+
+int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
+                      uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer) {
+    const uint64_t key[12] = {2, reinterpret_cast<uint64_t>(base), inner, outer, row_pitch_bytes,
+                              box_inner, box_outer, 0, 0, 0, 0, 0};
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_pitch_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    return encode(out, key, 2, base, dims, strides, box);
+}
+
+int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims_in[3],
+                      const uint64_t strides_bytes[2], const uint32_t box_in[3]) {
+    const uint64_t key[12] = {3,           reinterpret_cast<uint64_t>(base),
+                              dims_in[0],  dims_in[1],
+                              dims_in[2],  strides_bytes[0],
+                              strides_bytes[1], box_in[0],
+                              box_in[1],   box_in[2],
+                              0,           0};
+    cuuint64_t dims[3] = {dims_in[0], dims_in[1], dims_in[2]};
+    cuuint64_t strides[2] = {strides_bytes[0], strides_bytes[1]};
+    cuuint32_t box[3] = {box_in[0], box_in[1], box_in[2]};
+    return encode(out, key, 3, base, dims, strides, box);
+}
+
+}  // namespace isam
+
+using namespace isam;
+
+extern "C" {
+
+int isam_version(void) { return 100; }
+
+int isam_set_stream(void *stream) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    g_stream = static_cast<cudaStream_t>(stream);
+    return ISAM_OK;
+}
+
+const char *isam_last_error_string(void) { return t_err; }
+
+int isam_sync(void) {
+    int st;
+    DeviceState *ds = device_state(&st);
+    if (!ds) return st;
+    cudaError_t e = cudaStreamSynchronize(current_stream());
+    if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize");
+    uint32_t w[4] = {0, 0, 0, 0};
+    if ((e = cudaMemcpy(w, ds->err_word, sizeof w, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_error(e, "reading the device error word");
+    if (w[0] != 0) {
+        cudaMemset(ds->err_word, 0, 16);
+        return set_error(ISAM_ERR_TIMEOUT,
+                         "a bounded device wait ran out (site 0x%x, block %u); outputs of the "
+                         "failed call are undefined",
+                         w[1], w[2]);
+    }
+    return ISAM_OK;
+}
+
+int isam_shutdown(void) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    int cur = -1;
+    cudaGetDevice(&cur);
+    for (int d = 0; d < kMaxDevices; ++d) {
+        DeviceState *ds = g_dev[d];
+        if (!ds) continue;
+        cudaSetDevice(d);
+        cudaDeviceSynchronize();
+        cudaFree(ds->err_word);
+        cudaFree(ds->gru_gx);
+        cudaFree(ds->gru_hx);
+        cudaFree(ds->gru_counter);
+        delete ds;
+        g_dev[d] = nullptr;
+    }
+    if (cur >= 0) cudaSetDevice(cur);
+    {
+        std::lock_guard<std::mutex> lk2(g_tmap_mu);
+        for (auto &e : g_tmaps) e.used = false;
+    }
+    return ISAM_OK;
+}
+
+int isam_gemm(int M, int N, int K, int transA, int transB, float alpha, const isam_bf16 *A,
+              const isam_bf16 *B, float beta, float *C) {
+    GemmDesc g{M, N, K, transA, transB, alpha, beta, A, B, C, nullptr};
+    int rc = gemm_validate(g);
+    if (rc) return rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    GemmPlan plan;
+    if ((rc = gemm_plan(g, *ds, &plan))) return rc;
+    return gemm_launch(g, plan, *ds, current_stream());
+}
+
+// Reports the tile plan the cost model picks for a GEMM (for benchmarks and
+// tests; nothing is launched).  out[0..5] = BN, split, stages, group_m, grid,
+// shared-memory bytes.
+int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta, int *out) {
+    if (!out) return set_error(ISAM_ERR_INVALID_ARG, "null output");
+    GemmDesc g{M, N, K, transA, transB, 1.0f, beta, reinterpret_cast<const uint16_t *>(16),
+               reinterpret_cast<const uint16_t *>(16), reinterpret_cast<float *>(16), nullptr};
+    int rc = gemm_validate(g);
+    if (rc) return rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    GemmPlan plan;
+    if ((rc = gemm_plan(g, *ds, &plan))) return rc;
+    out[0] = plan.BN;
+    out[1] = plan.split;
+    out[2] = plan.stages;
+    out[3] = plan.group_m;
+    out[4] = plan.grid;
+    out[5] = static_cast<int>(plan.smem);
+    return ISAM_OK;
+}
+
+int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x, const isam_bf16 *W,
+                     const isam_bf16 *U, const float *b, const float *h0, float *h_out) {
+    if (T < 1 || batch < 1 || hidden < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward: sizes must be >= 1");
+    if (!x || !W || !U || !b || !h_out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward: null pointer");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gru_launch(T, batch, hidden, x, W, U, b, h0, h_out, *ds, current_stream());
+}
+
+int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
+                    const isam_bf16 *dw_w, const isam_bf16 *pw_w, float *out) {
+    if (N < 1 || H < 1 || W < 1 || Cin < 1 || Cout < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_dwsep_conv: sizes must be >= 1");
+    if (!x || !dw_w || !pw_w || !out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_dwsep_conv: null pointer");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return dwsep_launch(N, H, W, Cin, Cout, x, dw_w, pw_w, out, *ds, current_stream());
+}
+
+}  // extern "C"

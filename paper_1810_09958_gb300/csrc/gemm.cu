@@ -1,0 +1,635 @@
+// gemm.cu -- tcgen05 GEMM for sm_103a:  C = alpha * op(A) * op(B) + beta * C
+//
+// The matrix-multiplication kernel of Listing 1 / Listing 4, scheduled the
+// GB300 way:
+//   * a persistent grid, one CTA (or one cluster of CTAs) per SM, walking
+//     output tiles in an L2-friendly grouped order (the paper's "unrolling"
+//     places compute tiles that share memory close together, Section 3.3);
+//   * warp specialisation: warp 0 streams A/B tiles with TMA into a
+//     multi-stage shared-memory ring, warp 1 issues tcgen05.mma from one
+//     thread into a double-buffered TMEM accumulator, warps 2-5 drain TMEM
+//     and apply alpha/beta/bias while the next tile is being multiplied;
+//   * split-K for skinny problems: the CTAs of one thread-block cluster take
+//     disjoint K ranges of the same tile and reduce their partial tiles
+//     through distributed shared memory in a fixed rank order (deterministic);
+//   * the tile width, split and ring depth come from a small analytic cost
+//     model (the paper's "Approach" interface for tiling and device
+//     allocation choices, Sections 3.4 and 4).
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace isam {
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+constexpr int kABytes = kBM * kBK * 2;  // 16 KB
+
+enum : uint32_t {
+    SITE_PROD_EMPTY = 0x101,
+    SITE_PROD_DRAIN = 0x102,
+    SITE_MMA_TEMPTY = 0x111,
+    SITE_MMA_FULL = 0x112,
+    SITE_EPI_TFULL = 0x121,
+    SITE_EPI_REDFREE = 0x122,
+    SITE_EPI_REDFULL = 0x123,
+};
+
+struct GemmParams {
+    int M, N, K;
+    int m_tiles, n_tiles, kb_total;
+    int split, stages, group_m;
+    int n_vec4;  // 1 when N % 4 == 0 (16-byte stores in the split-K reduce)
+    float alpha, beta;
+    float *C;
+    const float *bias;
+    unsigned long long timeout_ns;
+    uint32_t *err;
+};
+
+template <int BN, bool B_MN>
+struct Cfg {
+    static constexpr int kBBytes = B_MN ? ((BN + 63) / 64) * 8192 : BN * 128;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kTmemCols = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
+    static constexpr int kCW = BN < 32 ? BN : 32;  // epilogue column chunk
+};
+
+__host__ __device__ inline size_t epi_bytes(int BN, int split) {
+    return split > 1 ? static_cast<size_t>(kBM) * (BN + 4) * 4 : static_cast<size_t>(4) * 32 * 33 * 4;
+}
+
+__device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int group_m,
+                                            int &mt, int &nt) {
+    const int per_group = group_m * n_tiles;
+    const int g = tile / per_group;
+    const int first_m = g * group_m;
+    const int gm = min(group_m, m_tiles - first_m);
+    const int local = tile - g * per_group;
+    mt = first_m + local % gm;
+    nt = local / gm;
+}
+
+// Waits ignoring the abort flag (used only to let copies already issued land).
+__device__ bool drain_wait(uint64_t *bar, uint32_t parity, unsigned long long timeout_ns) {
+    const uint32_t a = smem_u32(bar);
+    const unsigned long long t0 = globaltimer();
+    while (!mbar_try_wait(a, parity)) {
+        if (globaltimer() - t0 > timeout_ns) return false;
+    }
+    return true;
+}
+
+template <int BN, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const GemmParams p) {
+    using C = Cfg<BN, B_MN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    const int S = p.split;
+    const int ST = p.stages;
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + static_cast<size_t>(ST) * kABytes;
+    float *ebuf = reinterpret_cast<float *>(sB + static_cast<size_t>(ST) * C::kBBytes);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(ebuf) + epi_bytes(BN, S));
+    uint64_t *full = bars;
+    uint64_t *empty = bars + ST;
+    uint64_t *tfull = empty + ST;
+    uint64_t *tempty = tfull + 2;
+    uint64_t *red_full = tempty + 2;
+    uint64_t *red_free = red_full + 1;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(red_free + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = S > 1 ? cluster_ctarank() : 0u;
+    const int cluster_id = blockIdx.x / S;
+    const int num_clusters = gridDim.x / S;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < ST; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        mbar_init(red_full, S);
+        mbar_init(red_free, S);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (S > 1) cluster_sync_all();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const WaitCtx w{p.timeout_ns, p.err, abort_flag};
+
+    const int kb_begin = static_cast<int>((static_cast<long long>(rank) * p.kb_total) / S);
+    const int kb_end = static_cast<int>((static_cast<long long>(rank + 1) * p.kb_total) / S);
+    const int num_tiles = p.m_tiles * p.n_tiles;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            int issued = 0;
+            bool ok = true;
+            for (int tile = cluster_id; ok && tile < num_tiles; tile += num_clusters) {
+                int mt, nt;
+                tile_coords(tile, p.m_tiles, p.n_tiles, p.group_m, mt, nt);
+                for (int kb = kb_begin; kb < kb_end; ++kb) {
+                    if (!bounded_wait(&empty[stage], phase ^ 1u, w, SITE_PROD_EMPTY)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+                    uint8_t *a = sA + static_cast<size_t>(stage) * kABytes;
+                    uint8_t *b = sB + static_cast<size_t>(stage) * C::kBBytes;
+                    const int k0 = kb * kBK;
+                    if (A_MN) {
+                        tma_load_2d(&tmA, &full[stage], a, mt * kBM, k0);
+                        tma_load_2d(&tmA, &full[stage], a + 8192, mt * kBM + 64, k0);
+                    } else {
+                        tma_load_2d(&tmA, &full[stage], a, k0, mt * kBM);
+                    }
+                    if (B_MN) {
+#pragma unroll
+                        for (int c = 0; c < (BN + 63) / 64; ++c)
+                            tma_load_2d(&tmB, &full[stage], b + c * 8192, nt * BN + c * 64, k0);
+                    } else {
+                        tma_load_2d(&tmB, &full[stage], b, k0, nt * BN);
+                    }
+                    ++issued;
+                    if (++stage == ST) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                // Let every copy already issued land before the CTA can exit.
+                const int pending = min(issued, ST);
+                int s = stage;
+                uint32_t ph = phase;
+                for (int i = 0; i < pending; ++i) {
+                    if (--s < 0) {
+                        s = ST - 1;
+                        ph ^= 1u;
+                    }
+                    drain_wait(&full[s], ph, p.timeout_ns);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(kBM, BN, A_MN, B_MN);
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            for (int tile = cluster_id; ok && tile < num_tiles; tile += num_clusters) {
+                if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_MMA_TEMPTY)) break;
+                tc_fence_after();
+                const uint32_t d = tmem_base + static_cast<uint32_t>(acc * BN);
+                for (int kb = kb_begin; kb < kb_end; ++kb) {
+                    if (!bounded_wait(&full[stage], phase, w, SITE_MMA_FULL)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(sA + static_cast<size_t>(stage) * kABytes);
+                    const uint32_t b0 = smem_u32(sB + static_cast<size_t>(stage) * C::kBBytes);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, 8192, 1024)
+                                                 : sdesc_sw128(a0 + k * 32, 16, 1024);
+                        const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
+                                                 : sdesc_sw128(b0 + k * 32, 16, 1024);
+                        umma_bf16(d, ad, bd, idesc, (kb > kb_begin || k > 0) ? 1u : 0u);
+                    }
+                    umma_commit(&empty[stage]);
+                    if (++stage == ST) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                umma_commit(&tfull[acc]);
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+            }
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 2-5)
+        const int ew = warp - 2;          // 0..3
+        const int q = warp & 3;           // TMEM lane quadrant this warp may read
+        const int row_local = q * 32 + lane;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        int iter = 0;
+        bool ok = true;
+        for (int tile = cluster_id; tile < num_tiles; tile += num_clusters, ++iter) {
+            int mt, nt;
+            tile_coords(tile, p.m_tiles, p.n_tiles, p.group_m, mt, nt);
+            if (!bounded_wait(&tfull[acc], acc_phase, w, SITE_EPI_TFULL)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                   static_cast<uint32_t>(acc * BN);
+            if (S == 1) {
+                float *tb = ebuf + ew * (32 * 33);
+                constexpr int CW = C::kCW;
+                constexpr int RPI = 32 / CW;  // rows per store iteration
+                const int sub = lane / CW;
+                const int col = lane % CW;
+#pragma unroll 1
+                for (int c = 0; c < BN; c += CW) {
+                    uint32_t r[CW];
+                    if constexpr (CW == 32) {
+                        tmem_ld32(tbase + c, r);
+                    } else {
+                        tmem_ld16(tbase + c, r);
+                    }
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < CW; ++j) tb[lane * 33 + j] = __uint_as_float(r[j]);
+                    __syncwarp();
+                    const int gcol = nt * BN + c + col;
+                    const float bias = (p.bias != nullptr && gcol < p.N) ? p.bias[gcol] : 0.0f;
+#pragma unroll 4
+                    for (int rr = sub; rr < 32; rr += RPI) {
+                        const int grow = mt * kBM + q * 32 + rr;
+                        if (grow < p.M && gcol < p.N) {
+                            const size_t idx = static_cast<size_t>(grow) * p.N + gcol;
+                            float v = p.alpha * tb[rr * 33 + col] + bias;
+                            if (p.beta != 0.0f) v += p.beta * p.C[idx];
+                            p.C[idx] = v;
+                        }
+                    }
+                    __syncwarp();
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[acc]);
+            } else {
+                // Split-K: park this CTA's partial tile in shared memory, then
+                // every CTA of the cluster reduces its own row slice over all
+                // ranks in rank order.
+                if (iter > 0 &&
+                    !bounded_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w,
+                                        SITE_EPI_REDFREE)) {
+                    ok = false;
+                    break;
+                }
+                float *prow = ebuf + static_cast<size_t>(row_local) * (BN + 4);
+#pragma unroll 1
+                for (int c = 0; c < BN; c += C::kCW) {
+                    uint32_t r[C::kCW];
+                    if constexpr (C::kCW == 32) {
+                        tmem_ld32(tbase + c, r);
+                    } else {
+                        tmem_ld16(tbase + c, r);
+                    }
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < C::kCW; j += 4)
+                        *reinterpret_cast<float4 *>(prow + c + j) =
+                            make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
+                                        __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[acc]);
+                named_bar(1, 128);
+                if (ew == 0 && lane == 0) {
+                    for (int r = 0; r < S; ++r) mbar_arrive_remote(red_full, static_cast<uint32_t>(r));
+                }
+                if (!bounded_wait<true>(red_full, static_cast<uint32_t>(iter & 1), w,
+                                        SITE_EPI_REDFULL)) {
+                    ok = false;
+                    break;
+                }
+                const int rows_per = kBM / S;
+                const int row0 = static_cast<int>(rank) * rows_per;
+                const int g4 = BN / 4;
+                const int groups = rows_per * g4;
+                for (int g = ew * 32 + lane; g < groups; g += 128) {
+                    const int rl = row0 + g / g4;
+                    const int c4 = (g % g4) * 4;
+                    const uint32_t local = smem_u32(ebuf + static_cast<size_t>(rl) * (BN + 4) + c4);
+                    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int r = 0; r < S; ++r) {
+                        const float4 v = ld_dsmem_f4(mapa_shared(local, static_cast<uint32_t>(r)));
+                        s.x += v.x;
+                        s.y += v.y;
+                        s.z += v.z;
+                        s.w += v.w;
+                    }
+                    const int grow = mt * kBM + rl;
+                    const int gcol = nt * BN + c4;
+                    if (grow >= p.M) continue;
+                    float *crow = p.C + static_cast<size_t>(grow) * p.N;
+                    float o[4] = {s.x, s.y, s.z, s.w};
+                    if (p.n_vec4 && gcol + 3 < p.N) {
+                        float4 v;
+                        float *vv = reinterpret_cast<float *>(&v);
+                        float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (p.beta != 0.0f) cin = *reinterpret_cast<const float4 *>(crow + gcol);
+                        const float *ci = reinterpret_cast<const float *>(&cin);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            float x = p.alpha * o[j] + (p.bias ? p.bias[gcol + j] : 0.0f);
+                            if (p.beta != 0.0f) x += p.beta * ci[j];
+                            vv[j] = x;
+                        }
+                        *reinterpret_cast<float4 *>(crow + gcol) = v;
+                    } else {
+                        for (int j = 0; j < 4; ++j) {
+                            if (gcol + j >= p.N) break;
+                            float x = p.alpha * o[j] + (p.bias ? p.bias[gcol + j] : 0.0f);
+                            if (p.beta != 0.0f) x += p.beta * crow[gcol + j];
+                            crow[gcol + j] = x;
+                        }
+                    }
+                }
+                named_bar(1, 128);
+                if (ew == 0 && lane == 0) {
+                    for (int r = 0; r < S; ++r) mbar_arrive_remote(red_free, static_cast<uint32_t>(r));
+                }
+            }
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+        // Split-K: no peer may still be reading this CTA's partial tile when it exits.
+        if (S > 1 && ok && iter > 0) {
+            bounded_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, C::kTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------- host side
+using KernelFn = void (*)(CUtensorMap, CUtensorMap, GemmParams);
+
+template <int BN>
+KernelFn pick3(bool a_mn, bool b_mn) {
+    if (a_mn) return b_mn ? gemm_tc_kernel<BN, true, true> : gemm_tc_kernel<BN, true, false>;
+    return b_mn ? gemm_tc_kernel<BN, false, true> : gemm_tc_kernel<BN, false, false>;
+}
+
+KernelFn pick_kernel(int BN, bool a_mn, bool b_mn) {
+    switch (BN) {
+        case 16: return pick3<16>(a_mn, b_mn);
+        case 32: return pick3<32>(a_mn, b_mn);
+        case 64: return pick3<64>(a_mn, b_mn);
+        case 128: return pick3<128>(a_mn, b_mn);
+        case 256: return pick3<256>(a_mn, b_mn);
+        default: return nullptr;
+    }
+}
+
+int b_bytes(int BN, bool b_mn) { return b_mn ? ((BN + 63) / 64) * 8192 : BN * 128; }
+
+size_t smem_bytes(int BN, bool b_mn, int split, int stages) {
+    return 1024 + static_cast<size_t>(stages) * (kABytes + b_bytes(BN, b_mn)) + epi_bytes(BN, split) +
+           (2 * stages + 6) * 8 + 16;
+}
+
+int max_stages(int BN, bool b_mn, int split, int smem_limit) {
+    int st = 8;
+    while (st > 2 && smem_bytes(BN, b_mn, split, st) > static_cast<size_t>(smem_limit)) --st;
+    return st;
+}
+
+int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
+
+// Rough machine constants for the cost model (GB300: measured dense bf16 and
+// copy bandwidth; per-SM shared-memory bandwidth 128 B/clk).
+constexpr double kPeakFlops = 1.9e15;
+constexpr double kHbmBw = 6.7e12;
+constexpr double kSmL2Bw = 110e9;   // sustainable L2 -> SM bytes/s per SM
+constexpr double kClock = 1.9e9;
+constexpr double kTileOverheadUs = 0.35;
+constexpr double kLaunchUs = 2.5;
+
+double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out) {
+    const int m_tiles = ceil_div(g.M, kBM);
+    const int n_tiles = ceil_div(g.N, BN);
+    const long long tiles = static_cast<long long>(m_tiles) * n_tiles;
+    const int kb = ceil_div(g.K, kBK);
+    const int kb_per = ceil_div(kb, S);
+    const int clusters_max = std::max(1, num_sms / S);
+    const int clusters = static_cast<int>(std::min<long long>(tiles, clusters_max));
+    *grid_out = clusters * S;
+    const int tiles_per_cluster = ceil_div(tiles, clusters);
+    // Tensor time of one tile slice: 128 x BN x 16 per k-step at 4096 MAC/clk,
+    // or shared-memory bound at 128 B/clk for the A and B slices.
+    const double cyc_k16 = std::max(BN / 2.0, (kBM * 32.0 + BN * 32.0) / 128.0);
+    const double t_mma = kb_per * 4 * cyc_k16 / kClock * 1e6;
+    const double bytes_unit = static_cast<double>(kBM + BN) * kb_per * kBK * 2.0;
+    const double active = std::min<double>(static_cast<double>(tiles) * S, num_sms);
+    const double sm_bw = std::min(kSmL2Bw, kHbmBw / active);
+    const double t_load = bytes_unit / sm_bw * 1e6;
+    const double t_unit = std::max(t_mma, t_load) + kTileOverheadUs +
+                          (S > 1 ? 0.5 + 128.0 * BN * 4.0 * (S - 1) / S / 60e9 * 1e6 : 0.0);
+    const double t_steady = tiles_per_cluster * t_unit;
+    const double uniq = 2.0 * g.M * g.K + 2.0 * g.K * g.N +
+                        4.0 * g.M * g.N * (g.beta != 0.0f ? 2.0 : 1.0);
+    const double t_hbm = uniq / kHbmBw * 1e6;
+    const double t_flops = 2.0 * g.M * g.N * g.K / kPeakFlops * 1e6;
+    return std::max({t_steady, t_hbm, t_flops}) + kLaunchUs;
+}
+
+struct AttrCache {
+    std::mutex mu;
+    KernelFn fn[64] = {};
+    int smem[64] = {};
+    int n = 0;
+} g_attr;
+
+int ensure_smem_attr(KernelFn fn, size_t smem) {
+    std::lock_guard<std::mutex> lk(g_attr.mu);
+    for (int i = 0; i < g_attr.n; ++i)
+        if (g_attr.fn[i] == fn) {
+            if (g_attr.smem[i] >= static_cast<int>(smem)) return ISAM_OK;
+            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(smem));
+            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
+            g_attr.smem[i] = static_cast<int>(smem);
+            return ISAM_OK;
+        }
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
+    if (g_attr.n < 64) {
+        g_attr.fn[g_attr.n] = fn;
+        g_attr.smem[g_attr.n] = static_cast<int>(smem);
+        ++g_attr.n;
+    }
+    return ISAM_OK;
+}
+
+}  // namespace
+
+int gemm_validate(const GemmDesc &g) {
+    if (g.M < 1 || g.N < 1 || g.K < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm: sizes must be >= 1 (M=%d N=%d K=%d)",
+                         g.M, g.N, g.K);
+    if ((g.transA != 0 && g.transA != 1) || (g.transB != 0 && g.transB != 1))
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm: transA/transB must be 0 or 1");
+    if (!g.A || !g.B || !g.C) return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm: null pointer");
+    if ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B) |
+         reinterpret_cast<uintptr_t>(g.C)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: A, B and C must be 16-byte aligned");
+    const int a_pitch = g.transA ? g.M : g.K;
+    const int b_pitch = g.transB ? g.K : g.N;
+    if (a_pitch % 8 != 0 || b_pitch % 8 != 0)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gemm: stored row pitch of A (%d) and B (%d) must be multiples of 8 "
+                         "elements (16 bytes)",
+                         a_pitch, b_pitch);
+    return ISAM_OK;
+}
+
+int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
+    const bool b_mn = g.transB == 0;
+    const int nsm = ds.num_sms;
+    const int kb = ceil_div(g.K, kBK);
+    double best = 1e300;
+    GemmPlan bp{};
+    const int bns[] = {16, 32, 64, 128, 256};
+    const int splits[] = {1, 2, 4, 8};
+    for (int BN : bns) {
+        if (BN > 16 && BN / 2 >= g.N) continue;  // wider than needed
+        for (int S : splits) {
+            if (S > kb) continue;
+            if (S > 1 && BN > 128) continue;
+            int grid = 0;
+            const double t = estimate_us(g, BN, S, nsm, &grid);
+            if (t < best * 0.999) {
+                best = t;
+                bp.BN = BN;
+                bp.split = S;
+                bp.grid = grid;
+                bp.est_us = t;
+            }
+        }
+    }
+    if (const char *f = getenv("ISAM_FORCE_TILE")) {
+        int fbn = 0, fs = 0, fst = 0;
+        if (sscanf(f, "%d,%d,%d", &fbn, &fs, &fst) >= 2 && pick_kernel(fbn, false, false) &&
+            (fs == 1 || fs == 2 || fs == 4 || fs == 8) && fs <= kb && !(fs > 1 && fbn > 128)) {
+            bp.BN = fbn;
+            bp.split = fs;
+            estimate_us(g, fbn, fs, nsm, &bp.grid);
+            if (fst >= 2) bp.stages = fst;
+        }
+    }
+    const int st_max = max_stages(bp.BN, b_mn, bp.split, ds.max_smem_optin);
+    if (bp.stages < 2 || bp.stages > st_max) bp.stages = st_max;
+    bp.smem = smem_bytes(bp.BN, b_mn, bp.split, bp.stages);
+    bp.group_m = 16;
+    if (bp.smem > static_cast<size_t>(ds.max_smem_optin))
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: tile does not fit shared memory");
+    *plan = bp;
+    return ISAM_OK;
+}
+
+int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t stream) {
+    const bool a_mn = g.transA == 1;
+    const bool b_mn = g.transB == 0;
+    CUtensorMap ta, tb;
+    int rc;
+    if (a_mn)
+        rc = make_tmap_2d_bf16(&ta, g.A, g.M, g.K, static_cast<uint64_t>(g.M) * 2, 64, 64);
+    else
+        rc = make_tmap_2d_bf16(&ta, g.A, g.K, g.M, static_cast<uint64_t>(g.K) * 2, 64, kBM);
+    if (rc) return rc;
+    if (b_mn)
+        rc = make_tmap_2d_bf16(&tb, g.B, g.N, g.K, static_cast<uint64_t>(g.N) * 2, 64, 64);
+    else
+        rc = make_tmap_2d_bf16(&tb, g.B, g.K, g.N, static_cast<uint64_t>(g.K) * 2, 64,
+                               static_cast<uint32_t>(plan.BN));
+    if (rc) return rc;
+
+    GemmParams p{};
+    p.M = g.M;
+    p.N = g.N;
+    p.K = g.K;
+    p.m_tiles = ceil_div(g.M, kBM);
+    p.n_tiles = ceil_div(g.N, plan.BN);
+    p.kb_total = ceil_div(g.K, kBK);
+    p.split = plan.split;
+    p.stages = plan.stages;
+    p.group_m = plan.group_m;
+    p.n_vec4 = (g.N % 4 == 0) ? 1 : 0;
+    p.alpha = g.alpha;
+    p.beta = g.beta;
+    p.C = g.C;
+    p.bias = g.bias_n;
+    p.timeout_ns = wait_timeout_ns();
+    p.err = ds.err_word;
+
+    KernelFn fn = pick_kernel(plan.BN, a_mn, b_mn);
+    if (!fn) return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: no kernel for BN=%d", plan.BN);
+    if ((rc = ensure_smem_attr(fn, plan.smem))) return rc;
+
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.gridDim = dim3(static_cast<unsigned>(plan.grid), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = plan.smem;
+    cfg.stream = stream;
+    cfg.numAttrs = 0;
+    cfg.attrs = attr;
+    if (plan.split > 1) {
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = static_cast<unsigned>(plan.split);
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.numAttrs = 1;
+    }
+    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, ta, tb, p);
+    if (e != cudaSuccess) return cuda_error(e, "launch gemm_tc_kernel");
+    return ISAM_OK;
+}
+
+}  // namespace isam

@@ -1,0 +1,74 @@
+// internal.h -- host-side declarations shared by the library's translation
+// units.  Not part of the public ABI (that is include/isam.h).
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "../../include/isam.h"
+
+namespace isam {
+
+// Per-device state, created on first use with that device current.
+struct DeviceState {
+    int device = -1;
+    int num_sms = 0;
+    int max_smem_optin = 0;
+    uint32_t *err_word = nullptr;  // 4 x uint32 on the device
+    // GRU workspaces (grown on demand).
+    float *gru_gx = nullptr;       // [T*batch][3H] fp32 input projection
+    size_t gru_gx_bytes = 0;
+    uint16_t *gru_hx = nullptr;    // 2 x [32][H] bf16 hidden-state exchange
+    size_t gru_hx_bytes = 0;
+    uint32_t *gru_counter = nullptr;  // step counter (1 x uint32, padded)
+};
+
+DeviceState *device_state(int *status);  // current device; null + status on failure
+cudaStream_t current_stream();
+unsigned long long wait_timeout_ns();
+
+int set_error(int code, const char *fmt, ...);
+int cuda_error(cudaError_t e, const char *what);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point, with a
+// small cache keyed on every encoded field.
+int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
+                      uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
+int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims[3],
+                      const uint64_t strides_bytes[2], const uint32_t box[3]);
+
+// GEMM C = alpha op(A) op(B) + beta C (+ bias[n] per column when bias != null).
+struct GemmDesc {
+    int M, N, K;
+    int transA, transB;
+    float alpha, beta;
+    const uint16_t *A;
+    const uint16_t *B;
+    float *C;
+    const float *bias_n;
+};
+
+// Tile plan chosen by the cost model (or forced through ISAM_FORCE_TILE).
+struct GemmPlan {
+    int BN;       // tile width (tile height is always 128)
+    int split;    // CTAs of one cluster sharing a tile along K (1, 2, 4 or 8)
+    int stages;   // shared-memory ring depth
+    int group_m;  // rasterisation group height (tiles)
+    int grid;     // CTAs launched (persistent)
+    size_t smem;  // dynamic shared memory bytes
+    double est_us;
+};
+
+int gemm_validate(const GemmDesc &g);
+int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan);
+int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t s);
+
+int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
+               const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
+               cudaStream_t s);
+
+int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
+                 const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t s);
+
+}  // namespace isam

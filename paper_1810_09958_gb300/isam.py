@@ -1,0 +1,154 @@
+"""Thin Python binding of libisam.so (include/isam.h): argument marshalling only.
+
+Each function takes torch tensors that already live on the current CUDA
+device, checks dtype/shape/contiguity, points the library at torch's current
+stream and passes raw device pointers through the C ABI.  Every step of the
+computation runs in the library's CUDA kernels; there is no fallback.  If the
+library has not been built, loading it raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libisam.so")
+HEADER = os.path.join(os.path.dirname(PKG), "include", "isam.h")
+
+ISAM_OK, ISAM_ERR_INVALID_ARG, ISAM_ERR_UNSUPPORTED, ISAM_ERR_CUDA, ISAM_ERR_TIMEOUT = range(5)
+
+_lock = threading.Lock()
+_lib = None
+
+
+class IsamError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"isam error {code}: {msg}")
+        self.code = code
+
+
+def declared_functions() -> list[str]:
+    """Names of every function declared in include/isam.h."""
+    with open(HEADER) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(isam_[a-z0-9_]+)\s*\(", text)))
+
+
+def load():
+    """Loads libisam.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(
+                f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+        lib = ctypes.CDLL(LIB_PATH)
+        i, f, P = ctypes.c_int, ctypes.c_float, ctypes.c_void_p
+        lib.isam_version.argtypes = []
+        lib.isam_set_stream.argtypes = [P]
+        lib.isam_sync.argtypes = []
+        lib.isam_last_error_string.argtypes = []
+        lib.isam_last_error_string.restype = ctypes.c_char_p
+        lib.isam_shutdown.argtypes = []
+        lib.isam_gemm.argtypes = [i, i, i, i, i, f, P, P, f, P]
+        lib.isam_gemm_plan_info.argtypes = [i, i, i, i, i, f, P]
+        lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
+        lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
+        for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
+                     "isam_gemm_plan_info", "isam_gru_forward", "isam_dwsep_conv"):
+            getattr(lib, name).restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def last_error() -> str:
+    return load().isam_last_error_string().decode(errors="replace")
+
+
+def check(rc: int) -> None:
+    if rc != ISAM_OK:
+        raise IsamError(rc, last_error())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _dev(t, dtype, numel, name):
+    import torch
+    if t.device.type != "cuda":
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if t.numel() != numel:
+        raise ValueError(f"{name} has {t.numel()} elements, expected {numel}")
+    if t.device.index != torch.cuda.current_device():
+        raise ValueError(f"{name} is not on the current device")
+
+
+def _use_current_stream(lib):
+    import torch
+    lib.isam_set_stream(ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+
+
+def sync() -> None:
+    check(load().isam_sync())
+
+
+def shutdown() -> None:
+    check(load().isam_shutdown())
+
+
+def gemm(M, N, K, transA, transB, alpha, A, B, beta, C) -> None:
+    """isam_gemm: C = alpha op(A) op(B) + beta C (A, B bf16; C fp32)."""
+    import torch
+    lib = load()
+    _dev(A, torch.bfloat16, M * K, "A")
+    _dev(B, torch.bfloat16, K * N, "B")
+    _dev(C, torch.float32, M * N, "C")
+    _use_current_stream(lib)
+    check(lib.isam_gemm(M, N, K, int(transA), int(transB), float(alpha), _ptr(A), _ptr(B),
+                        float(beta), _ptr(C)))
+
+
+def gemm_plan(M, N, K, transA, transB, beta=0.0) -> dict:
+    """The tile plan the library's cost model picks (nothing is launched)."""
+    lib = load()
+    out = (ctypes.c_int * 6)()
+    check(lib.isam_gemm_plan_info(M, N, K, int(transA), int(transB), float(beta), out))
+    return dict(zip(("BN", "split", "stages", "group_m", "grid", "smem"), list(out)))
+
+
+def gru_forward(T, batch, hidden, x, W, U, b, h0, h_out) -> None:
+    """isam_gru_forward (x, W, U bf16; b, h0, h_out fp32; h0 may be None)."""
+    import torch
+    lib = load()
+    H = hidden
+    _dev(x, torch.bfloat16, T * batch * H, "x")
+    _dev(W, torch.bfloat16, 3 * H * H, "W")
+    _dev(U, torch.bfloat16, 3 * H * H, "U")
+    _dev(b, torch.float32, 6 * H, "b")
+    if h0 is not None:
+        _dev(h0, torch.float32, batch * H, "h0")
+    _dev(h_out, torch.float32, T * batch * H, "h_out")
+    _use_current_stream(lib)
+    check(lib.isam_gru_forward(T, batch, H, _ptr(x), _ptr(W), _ptr(U), _ptr(b), _ptr(h0),
+                               _ptr(h_out)))
+
+
+def dwsep_conv(N, H, W, Cin, Cout, x, dw_w, pw_w, out) -> None:
+    """isam_dwsep_conv: NHWC 3x3 depthwise (pad 1) then 1x1 pointwise."""
+    import torch
+    lib = load()
+    _dev(x, torch.bfloat16, N * H * W * Cin, "x")
+    _dev(dw_w, torch.bfloat16, 9 * Cin, "dw_w")
+    _dev(pw_w, torch.bfloat16, Cin * Cout, "pw_w")
+    _dev(out, torch.float32, N * H * W * Cout, "out")
+    _use_current_stream(lib)
+    check(lib.isam_dwsep_conv(N, H, W, Cin, Cout, _ptr(x), _ptr(dw_w), _ptr(pw_w), _ptr(out)))
