@@ -1,9 +1,394 @@
-// gru.cu -- GRU forward (placeholder until the persistent recurrent kernel lands).
+// gru.cu -- GRU forward over T steps on sm_103a.
+//
+// Recurrent scheduling after Section 3.6 of the paper: the loop body is
+// scheduled once as a priming iteration (load the persistent weights and the
+// initial state onto the compute units), a recursive iteration run T times
+// that overwrites its own inputs, and a finish iteration (the last state is
+// already in place in h_out).  The paper credits its GRU speed-up to fusion
+// and to keeping reused data on chip (Section 5.1.2); here:
+//
+//   1. gx = x W^T + b_ih for all T steps is one GEMM (isam_gemm's kernel, bias
+//      fused in its epilogue), written to a library workspace;
+//   2. one cooperative persistent kernel runs the recurrence.  CTA c owns
+//      hidden units [16c, 16c+16): its 48 rows of U (gates r, z, n) stay in
+//      shared memory for all T steps.  Per step it TMA-loads bf16(h_{t-1})
+//      (all batch rows), multiplies U_slice * h^T on the tensor cores into
+//      TMEM, evaluates the gates in fp32 with h carried in fp32 registers,
+//      writes h_t to h_out and bf16(h_t) to an exchange buffer, and signals a
+//      grid-wide step counter.  Every wait is bounded in time.
+#include <cstdio>
+#include <cstdlib>
+
+#include <cuda_bf16.h>
+
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace isam {
-int gru_launch(int, int, int, const uint16_t *, const uint16_t *, const uint16_t *, const float *,
-               const float *, float *, DeviceState &, cudaStream_t) {
-    return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: not available in this build");
+
+namespace {
+
+constexpr int kUnits = 16;           // hidden units per CTA
+constexpr int kRows = 3 * kUnits;    // U rows per CTA (r, z, n)
+constexpr int kBatchPad = 32;        // MMA N (batch rows, padded)
+constexpr int kThreads = 128;
+constexpr int kAtomU = kRows * 128;  // bytes of one 64-wide K atom of the U slice (6 KB)
+constexpr int kAtomH = kBatchPad * 128;  // bytes of one K atom of h (4 KB)
+constexpr int kQuarters = 4;             // at most this many h pieces per step
+constexpr int kGhBytes = 6400;           // 48 x 33 fp32, rounded up to 64 bytes
+
+enum : uint32_t {
+    SITE_GRU_STEP = 0x201,
+    SITE_GRU_U = 0x202,
+    SITE_GRU_H = 0x203,
+    SITE_GRU_MMA = 0x204,
+};
+
+struct GruParams {
+    int T, batch, H, nk;       // nk = H / 64 K atoms
+    int nq, qk;                // h is loaded in nq pieces of qk atoms (nq * qk == nk)
+    int n_cta;
+    const float *gx;           // [T*batch][3H], includes b_ih
+    const float *b_hh;         // [3H]
+    const float *h0;           // [batch][H] or null
+    float *h_out;              // [T][batch][H]
+    uint16_t *hx;              // [2][32][H] bf16 exchange
+    uint32_t *counter;         // step counter (zeroed before launch)
+    int skip_publish_cta;      // debug: this CTA never publishes (-1: none)
+    unsigned long long timeout_ns;
+    uint32_t *err;
+};
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
+
+__device__ __forceinline__ void red_release_gpu_add(uint32_t *p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ float sigmoidf_fast(float v) { return 1.0f / (1.0f + __expf(-v)); }
+
+__device__ __forceinline__ uint16_t f32_to_bf16_rne(float f) {
+    return __bfloat16_as_ushort(__float2bfloat16_rn(f));
+}
+
+// Spins (bounded) until the step counter reaches target.
+__device__ bool wait_counter(const uint32_t *counter, uint32_t target, const WaitCtx &w) {
+    if (ld_acquire_gpu(counter) >= target) return true;
+    const unsigned long long t0 = globaltimer();
+    for (uint32_t i = 1;; ++i) {
+        if (ld_acquire_gpu(counter) >= target) return true;
+        if ((i & 15u) == 0u) {
+            if (*w.abort_flag) return false;
+            if (globaltimer() - t0 > w.timeout_ns) {
+                report_timeout(w, SITE_GRU_STEP);
+                return false;
+            }
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    gru_recurrent_kernel(const __grid_constant__ CUtensorMap tmU,
+                         const __grid_constant__ CUtensorMap tmH0,
+                         const __grid_constant__ CUtensorMap tmH1, const GruParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    // U slice: nk atoms of 48 rows x 128 B; the M = 128 MMA reads 80 rows past
+    // each atom, so the region is padded to keep the last atom's read inside.
+    const int u_bytes = p.nk * kAtomU + 10240;
+    uint8_t *sU = smem;
+    uint8_t *sH = smem + u_bytes;                        // nk atoms of 32 rows x 128 B
+    float *gh = reinterpret_cast<float *>(sH + p.nk * kAtomH);  // [48][33] fp32
+    uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(gh) + kGhBytes);
+    uint64_t *ubar = bars;                 // U slice landed
+    uint64_t *hbar = bars + 1;             // [kQuarters] h quarter landed
+    uint64_t *mma_done = hbar + kQuarters; // MMAs of the step complete
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mma_done + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5;
+    const int lane = tid & 31;
+    const int j0 = blockIdx.x * kUnits;
+    const int H = p.H;
+    const int G = 3 * H;
+    const WaitCtx w{p.timeout_ns, p.err, abort_flag};
+    const int qk = p.qk;
+    const int nq = p.nq;
+
+    if (tid == 0) {
+        mbar_init(ubar, 1);
+        for (int q = 0; q < kQuarters; ++q) mbar_init(&hbar[q], 1);
+        mbar_init(mma_done, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(tmem_slot, 32);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_d = *tmem_slot;
+
+    // ---- priming iteration: persistent weights and initial state.
+    if (tid == 0) {
+        tma_prefetch_desc(&tmU);
+        mbar_arrive_expect_tx(ubar, static_cast<uint32_t>(p.nk * kAtomU));
+        for (int ka = 0; ka < p.nk; ++ka) tma_load_3d(&tmU, ubar, sU + ka * kAtomU, ka * 64, j0, 0);
+    }
+    // Each thread owns one unit u and batch rows bb, bb + 8, bb + 16, bb + 24.
+    const int u = tid & 15;
+    const int bb = tid >> 4;
+    const int j = j0 + u;
+    const float bh_r = p.b_hh[j], bh_z = p.b_hh[H + j], bh_n = p.b_hh[2 * H + j];
+    float hprev[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int b = bb + 8 * k;
+        hprev[k] = (p.h0 != nullptr && b < p.batch) ? p.h0[static_cast<size_t>(b) * H + j] : 0.0f;
+        if (b < p.batch) p.hx[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hprev[k]);
+    }
+    fence_proxy_async_global();
+    __syncthreads();
+    if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta) red_release_gpu_add(p.counter, 1u);
+    bool ok = true;
+    if (tid == 32) ok = bounded_wait(ubar, 0, w, SITE_GRU_U);
+
+    const uint32_t idesc = idesc_bf16_f32(128, kBatchPad, false, false);
+    int issued_phase = -1;  // last step whose h loads were issued (for the drain)
+
+    // ---- recursive iteration, T times.
+    for (int t = 0; t < p.T; ++t) {
+        const uint32_t par = static_cast<uint32_t>(t & 1);
+        if (tid == 0 && !*abort_flag) {
+            if (wait_counter(p.counter, static_cast<uint32_t>((t + 1) * p.n_cta), w)) {
+                fence_proxy_async_global();
+                const CUtensorMap *m = (t & 1) ? &tmH1 : &tmH0;
+                for (int q = 0; q < nq; ++q) {
+                    mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(qk * kAtomH));
+                    tma_load_3d(m, &hbar[q], sH + q * qk * kAtomH, 0, 0, q * qk);
+                }
+                issued_phase = t;
+            }
+        }
+        // Input projection of this step (independent of h): prefetch.
+        float gxr[4], gxz[4], gxn[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int b = bb + 8 * k;
+            if (b < p.batch) {
+                const float *g = p.gx + (static_cast<size_t>(t) * p.batch + b) * G + j;
+                gxr[k] = g[0];
+                gxz[k] = g[H];
+                gxn[k] = g[2 * H];
+            } else {
+                gxr[k] = gxz[k] = gxn[k] = 0.0f;
+            }
+        }
+        if (tid == 32 && ok) {
+            for (int q = 0; q < nq && ok; ++q) {
+                if (!bounded_wait(&hbar[q], par, w, SITE_GRU_H)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                for (int a = q * qk; a < (q + 1) * qk; ++a) {
+                    const uint32_t ua = smem_u32(sU + a * kAtomU);
+                    const uint32_t ha = smem_u32(sH + a * kAtomH);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        umma_bf16(tmem_d, sdesc_sw128(ua + k * 32, 16, 1024),
+                                  sdesc_sw128(ha + k * 32, 16, 1024), idesc,
+                                  (a > 0 || k > 0) ? 1u : 0u);
+                }
+            }
+            if (ok) umma_commit(mma_done);
+        }
+        if (!bounded_wait(mma_done, par, w, SITE_GRU_MMA)) break;
+        tc_fence_after();
+        if (warp < 2) {
+            uint32_t r[32];
+            tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
+            tmem_ld_wait();
+            const int row = warp * 32 + lane;
+            if (row < kRows) {
+#pragma unroll
+                for (int c = 0; c < 32; ++c) gh[row * 33 + c] = __uint_as_float(r[c]);
+            }
+        }
+        tc_fence_before();
+        __syncthreads();
+        uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int b = bb + 8 * k;
+            if (b >= p.batch) continue;
+            const float ghr = gh[u * 33 + b] + bh_r;
+            const float ghz = gh[(kUnits + u) * 33 + b] + bh_z;
+            const float ghn = gh[(2 * kUnits + u) * 33 + b] + bh_n;
+            const float rg = sigmoidf_fast(gxr[k] + ghr);
+            const float zg = sigmoidf_fast(gxz[k] + ghz);
+            const float ng = tanhf(gxn[k] + rg * ghn);
+            const float hn = (1.0f - zg) * ng + zg * hprev[k];
+            hprev[k] = hn;
+            p.h_out[(static_cast<size_t>(t) * p.batch + b) * H + j] = hn;
+            hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
+        }
+        fence_proxy_async_global();
+        __syncthreads();
+        if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
+            red_release_gpu_add(p.counter, 1u);
+        tc_fence_after();
+        if (*abort_flag) break;
+    }
+
+    // ---- teardown: let issued copies land, release TMEM.
+    if (tid == 0 && issued_phase >= 0 && *abort_flag) {
+        for (int q = 0; q < nq; ++q) {
+            const uint32_t a = smem_u32(&hbar[q]);
+            const unsigned long long t0 = globaltimer();
+            while (!mbar_try_wait(a, static_cast<uint32_t>(issued_phase & 1)))
+                if (globaltimer() - t0 > p.timeout_ns) break;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem_d, 32);
+    }
+}
+
+size_t gru_smem_bytes(int H) {
+    const int nk = H / 64;
+    return 1024 + static_cast<size_t>(nk) * kAtomU + 10240 + static_cast<size_t>(nk) * kAtomH +
+           kGhBytes + 8 * (2 + kQuarters) + 16 + 16;
+}
+
+int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
+    if (*cap >= need) return ISAM_OK;
+    if (*ptr) cudaFree(*ptr);
+    *ptr = nullptr;
+    *cap = 0;
+    cudaError_t e = cudaMalloc(ptr, need);
+    if (e != cudaSuccess) return cuda_error(e, what);
+    *cap = need;
+    return ISAM_OK;
+}
+
+}  // namespace
+
+int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
+               const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
+               cudaStream_t stream) {
+    const int H = hidden;
+    if (batch > kBatchPad || H % 64 != 0 || H > 1024 || H < 64)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gru_forward: needs batch <= 32 and hidden a multiple of 64 in "
+                         "[64, 1024] (batch=%d hidden=%d)",
+                         batch, H);
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
+         reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |
+         reinterpret_cast<uintptr_t>(h0) | reinterpret_cast<uintptr_t>(h_out)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: pointers must be 16-byte aligned");
+    const int n_cta = H / kUnits;
+    if (n_cta > ds.num_sms)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: %d CTAs cannot be co-resident", n_cta);
+    const size_t smem = gru_smem_bytes(H);
+    if (smem > static_cast<size_t>(ds.max_smem_optin))
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: hidden too large for shared memory");
+
+    int rc;
+    const size_t gx_bytes = static_cast<size_t>(T) * batch * 3 * H * sizeof(float);
+    if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_gx), &ds.gru_gx_bytes, gx_bytes,
+                        "allocating the GRU projection workspace")))
+        return rc;
+    const size_t hx_bytes = static_cast<size_t>(2) * kBatchPad * H * sizeof(uint16_t);
+    if (ds.gru_hx_bytes < hx_bytes) {
+        if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_hx), &ds.gru_hx_bytes, hx_bytes,
+                            "allocating the GRU exchange buffer")))
+            return rc;
+        cudaError_t e = cudaMemset(ds.gru_hx, 0, hx_bytes);
+        if (e != cudaSuccess) return cuda_error(e, "clearing the GRU exchange buffer");
+    }
+    if (!ds.gru_counter) {
+        cudaError_t e = cudaMalloc(&ds.gru_counter, 256);
+        if (e != cudaSuccess) return cuda_error(e, "allocating the GRU step counter");
+    }
+
+    // 1. Input projection for all steps: gx = x W^T + b_ih  (M = T*batch, N = 3H, K = H).
+    GemmDesc g{T * batch, 3 * H, H, 0, 1, 1.0f, 0.0f, x, W, ds.gru_gx, b};
+    GemmPlan plan;
+    if ((rc = gemm_validate(g))) return rc;
+    if ((rc = gemm_plan(g, ds, &plan))) return rc;
+    if ((rc = gemm_launch(g, plan, ds, stream))) return rc;
+
+    // 2. Recurrence.
+    CUtensorMap tmU, tmH0, tmH1;
+    {
+        const uint64_t dims[3] = {static_cast<uint64_t>(H), static_cast<uint64_t>(H), 3};
+        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, static_cast<uint64_t>(H) * H * 2};
+        const uint32_t box[3] = {64, kUnits, 3};
+        if ((rc = make_tmap_3d_bf16(&tmU, U, dims, strides, box))) return rc;
+    }
+    const int nk = H / 64;
+    const int nq = (nk % 4 == 0) ? 4 : (nk % 2 == 0) ? 2 : 1;
+    for (int i = 0; i < 2; ++i) {
+        const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(nk)};
+        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
+        const uint32_t box[3] = {64, kBatchPad, static_cast<uint32_t>(nk / nq)};
+        if ((rc = make_tmap_3d_bf16(i ? &tmH1 : &tmH0, ds.gru_hx + static_cast<size_t>(i) * kBatchPad * H,
+                                    dims, strides, box)))
+            return rc;
+    }
+    GruParams p{};
+    p.T = T;
+    p.batch = batch;
+    p.H = H;
+    p.nk = nk;
+    p.nq = nq;
+    p.qk = nk / nq;
+    p.n_cta = n_cta;
+    p.gx = ds.gru_gx;
+    p.b_hh = b + 3 * H;
+    p.h0 = h0;
+    p.h_out = h_out;
+    p.hx = ds.gru_hx;
+    p.counter = ds.gru_counter;
+    p.skip_publish_cta = -1;
+    if (const char *s = getenv("ISAM_DEBUG_GRU_SKIP_CTA")) p.skip_publish_cta = atoi(s);
+    p.timeout_ns = wait_timeout_ns();
+    p.err = ds.err_word;
+
+    cudaError_t e = cudaMemsetAsync(ds.gru_counter, 0, sizeof(uint32_t), stream);
+    if (e != cudaSuccess) return cuda_error(e, "clearing the GRU step counter");
+    static bool attr_set = false;
+    if (!attr_set) {
+        e = cudaFuncSetAttribute(gru_recurrent_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 ds.max_smem_optin);
+        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
+        attr_set = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(n_cta), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
+    if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel");
+    return ISAM_OK;
+}
+
 }  // namespace isam

@@ -92,7 +92,7 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t par
     return ok != 0;
 }
 
-__device__ __noinline__ void report_timeout(const WaitCtx &w, uint32_t site) {
+static __device__ __noinline__ void report_timeout(const WaitCtx &w, uint32_t site) {
     *w.abort_flag = 1;
     if (atomicOr(w.err, DEV_ERR_TIMEOUT) == 0u) {
         w.err[1] = site;

@@ -1,0 +1,144 @@
+"""GRU forward parity on the GPU through the C ABI (isam_gru_forward) against
+the fp64 oracle.  Tolerance: normalised max error over every step's hidden
+state (all of h_out) <= 1e-2."""
+import os
+import subprocess
+import sys
+import textwrap
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_1810_09958_gb300 import isam, synth
+from gpu_util import Guarded, dev_bf16, nmax_err
+
+pytestmark = pytest.mark.gpu
+TOL = 1e-2
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import torch
+    from paper_1810_09958_gb300 import build
+    build.build()
+    isam.load()
+    torch.cuda.set_device(0)
+    yield
+    isam.sync()
+
+
+def run_gru(x, W, U, b, h0):
+    import torch
+    T, batch, H = x.shape
+    out = Guarded(T * batch * H)
+    h0d = None if h0 is None else torch.from_numpy(np.ascontiguousarray(h0, np.float32)).cuda()
+    isam.gru_forward(T, batch, H, dev_bf16(x), dev_bf16(W), dev_bf16(U),
+                     torch.from_numpy(b).cuda(), h0d, out.t)
+    isam.sync()
+    assert out.guards_intact(), "write outside h_out"
+    return out.numpy().reshape(T, batch, H)
+
+
+def test_gru_benchmark_shape_full_oracle():
+    """hidden = input = 1024, batch 32, 128 steps, h0 = 0 (the GRU benchmark shape)."""
+    T, batch, H = 128, 32, 1024
+    x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=synth.stream_seed(synth.BASE_SEED, 3))
+    got = run_gru(x, W, U, b, h0)
+    ref = oracle.gru_forward(x, W, U, b, h0)
+    err = nmax_err(got, ref)
+    assert err <= TOL, err
+    assert nmax_err(got[-1], ref[-1]) <= TOL
+
+
+@pytest.mark.parametrize("T,batch,H", [(1, 1, 64), (5, 3, 64), (7, 17, 192), (9, 32, 128),
+                                       (20, 32, 512), (3, 31, 320), (16, 8, 1024)])
+def test_gru_shapes_with_initial_state(T, batch, H):
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 1000 + batch * 10 + H)
+    h0 = synth.f32_uniform(T + batch + H, (batch, H))
+    got = run_gru(x, W, U, b, h0)
+    ref = oracle.gru_forward(x, W, U, b, h0)
+    assert nmax_err(got, ref) <= TOL
+
+
+def test_gru_null_h0_means_zeros():
+    T, batch, H = 4, 5, 128
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=44)
+    got = run_gru(x, W, U, b, None)
+    ref = oracle.gru_forward(x, W, U, b, None)
+    assert nmax_err(got, ref) <= TOL
+
+
+def test_gru_zero_weights_closed_form():
+    """W = U = 0: h_t = n + z**t (h0 - n) with r, z, n set by the biases alone."""
+    T, batch, H = 6, 4, 128
+    zero = np.zeros((3 * H, H), np.uint16)
+    x = synth.bf16_normal(1, (T, batch, H))
+    b = synth.f32_uniform(2, (6 * H,), -2.0, 2.0)
+    h0 = synth.f32_uniform(3, (batch, H))
+    got = run_gru(x, zero, zero, b, h0)
+    ref = oracle.gru_forward(x, zero, zero, b, h0)
+    assert np.max(np.abs(got - ref)) <= 1e-5
+
+
+def test_gru_saturated_update_gate_keeps_state():
+    T, batch, H = 10, 6, 256
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=7)
+    b = b.copy()
+    b[H:2 * H] = 30.0
+    h0 = synth.f32_uniform(8, (batch, H))
+    got = run_gru(x, W, U, b, h0)
+    assert np.max(np.abs(got - h0[None])) <= 1e-6
+
+
+def test_gru_repeat_calls_identical():
+    T, batch, H = 12, 32, 256
+    x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=12)
+    a = run_gru(x, W, U, b, h0)
+    c = run_gru(x, W, U, b, h0)
+    assert np.array_equal(a, c)
+
+
+def test_gru_unsupported_shapes_rejected():
+    import torch
+    z = torch.zeros(4096, dtype=torch.bfloat16, device="cuda")
+    f = torch.zeros(4096, dtype=torch.float32, device="cuda")
+    lib = isam.load()
+    import ctypes
+    p = lambda t: ctypes.c_void_p(t.data_ptr())
+    assert lib.isam_gru_forward(1, 33, 64, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_gru_forward(1, 1, 96, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
+
+
+def test_gru_missing_participant_times_out_cleanly():
+    """One CTA never signals the step counter (a flag nothing sets): every
+    bounded wait runs out, the kernel returns, isam_sync reports
+    ISAM_ERR_TIMEOUT, and the context stays usable for a correct call."""
+    code = textwrap.dedent(f"""
+        import sys, numpy as np, torch
+        sys.path.insert(0, {ROOT!r}); sys.path.insert(0, {os.path.join(ROOT, 'tests')!r})
+        import os
+        from paper_1810_09958_gb300 import isam, synth
+        import oracle
+        from gpu_util import dev_bf16, nmax_err
+        torch.cuda.set_device(0)
+        T, batch, H = 4, 8, 128
+        x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=3)
+        args = [dev_bf16(x), dev_bf16(W), dev_bf16(U), torch.from_numpy(b).cuda(), None]
+        out = torch.zeros(T * batch * H, device="cuda")
+        os.environ["ISAM_DEBUG_GRU_SKIP_CTA"] = "0"
+        isam.gru_forward(T, batch, H, *args, out)
+        rc = isam.load().isam_sync()
+        assert rc == isam.ISAM_ERR_TIMEOUT, rc
+        del os.environ["ISAM_DEBUG_GRU_SKIP_CTA"]
+        isam.gru_forward(T, batch, H, *args, out)
+        isam.sync()
+        ref = oracle.gru_forward(x, W, U, b, None)
+        assert nmax_err(out.cpu().numpy().reshape(T, batch, H), ref) <= 1e-2
+        print("TIMEOUT_OK")
+    """)
+    env = dict(os.environ, ISAM_WAIT_TIMEOUT_MS="300")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       timeout=300)
+    assert r.returncode == 0 and "TIMEOUT_OK" in r.stdout, r.stdout + r.stderr
