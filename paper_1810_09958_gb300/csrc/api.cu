@@ -46,7 +46,8 @@ int get_encoder() {
 }
 
 int encode(CUtensorMap *out, const uint64_t key[12], cuuint32_t rank, const void *base,
-           const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box) {
+           const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box,
+           CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
     {
         std::lock_guard<std::mutex> lk(g_tmap_mu);
         for (int i = 0; i < kTmapCache; ++i)
@@ -58,7 +59,7 @@ int encode(CUtensorMap *out, const uint64_t key[12], cuuint32_t rank, const void
     int rc = get_encoder();
     if (rc) return rc;
     cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = g_encode(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), dims,
+    CUresult r = g_encode(out, dtype, rank, const_cast<void *>(base), dims,
                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -153,6 +154,16 @@ int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64
     cuuint64_t strides[1] = {row_pitch_bytes};
     cuuint32_t box[2] = {box_inner, box_outer};
     return encode(out, key, 2, base, dims, strides, box);
+}
+
+int make_tmap_2d_f32(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
+                     uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer) {
+    const uint64_t key[12] = {0xF32, reinterpret_cast<uint64_t>(base), inner, outer,
+                              row_pitch_bytes, box_inner, box_outer, 0, 0, 0, 0, 0};
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_pitch_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    return encode(out, key, 2, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
 }
 
 int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims_in[3],

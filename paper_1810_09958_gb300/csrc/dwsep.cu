@@ -1,9 +1,361 @@
-// dwsep.cu -- separable depthwise convolution (placeholder until the fused kernel lands).
+// dwsep.cu -- separable depthwise convolution (Listing 3 with s = 1, c = 1,
+// zero border of one pixel) on sm_103a, in the factored form of Section 2.3:
+// the 3x3 depthwise sum is formed first and the result is multiplied by the
+// pointwise weights, a GEMM with M = N*H*W pixels, K = Cin, N = Cout.
+//
+// One persistent kernel, one CTA per SM, 128-pixel tiles:
+//   warps 0-3  depthwise producers: read the 3x3 neighbourhood of each pixel
+//              with 16-byte NHWC loads, accumulate in fp32, round to bf16 and
+//              write the A tile straight into the tensor cores' 128-byte
+//              swizzled K-major layout (two-stage ring);
+//   warp 4     loads the pointwise weights once (TMA, resident for the whole
+//              kernel) and issues tcgen05.mma from one thread into a
+//              double-buffered TMEM accumulator;
+//   warps 5-8  drain TMEM, stage 32x32 fp32 blocks in swizzled shared memory
+//              and write them out with TMA bulk tensor stores.
+// The depthwise intermediate never leaves the chip.
+#include <cuda_bf16.h>
+
+#include <cstdio>
+
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace isam {
-int dwsep_launch(int, int, int, int, int, const uint16_t *, const uint16_t *, const uint16_t *,
-                 float *, DeviceState &, cudaStream_t) {
-    return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: not available in this build");
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kThreads = 288;
+constexpr int kAStages = 2;
+constexpr int kStageBufs = 2;  // epilogue staging buffers per warp (4 KB each)
+
+enum : uint32_t {
+    SITE_DW_AEMPTY = 0x301,
+    SITE_DW_AFULL = 0x302,
+    SITE_DW_TEMPTY = 0x303,
+    SITE_DW_TFULL = 0x304,
+    SITE_DW_W = 0x305,
+};
+
+struct DwParams {
+    int N, H, W, Cin, Cout;
+    long long M;            // N*H*W pixels
+    int tiles;
+    int atoms;              // ceil(Cin / 64) K atoms of the A tile
+    int kb;                 // ceil(Cin / 64) k-blocks of the pointwise weights
+    int nchunks;            // ceil(Cout / 64) 64-wide column chunks of the weights
+    const uint16_t *x;
+    const uint16_t *dw;
+    unsigned long long timeout_ns;
+    uint32_t *err;
+};
+
+struct DwLayout {
+    int a_stage_bytes, w_bytes, dwf_bytes;
+    int off_a, off_w, off_stage, off_dwf, off_bars;
+    int total;
+};
+
+__host__ __device__ inline DwLayout dw_layout(int Cin, int Cout) {
+    DwLayout L;
+    const int atoms = (Cin + 63) / 64;
+    const int nchunks = (Cout + 63) / 64;
+    L.a_stage_bytes = atoms * kBM * 128;
+    L.w_bytes = atoms * nchunks * 8192;
+    L.dwf_bytes = ((9 * Cin * 4) + 1023) / 1024 * 1024;
+    L.off_a = 0;
+    L.off_w = L.off_a + kAStages * L.a_stage_bytes;
+    L.off_stage = L.off_w + L.w_bytes;
+    L.off_dwf = L.off_stage + 4 * kStageBufs * 4096;
+    L.off_bars = L.off_dwf + L.dwf_bytes;
+    L.total = L.off_bars + 256 + 1024;
+    return L;
 }
+
+__device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const uint32_t l = __bfloat16_as_ushort(__float2bfloat16_rn(lo));
+    const uint32_t h = __bfloat16_as_ushort(__float2bfloat16_rn(hi));
+    return l | (h << 16);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    dwsep_fused_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmOut,
+                       const DwParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    const DwLayout L = dw_layout(p.Cin, p.Cout);
+    uint8_t *sA = smem + L.off_a;
+    uint8_t *sW = smem + L.off_w;
+    uint8_t *sStage = smem + L.off_stage;
+    float *dwf = reinterpret_cast<float *>(smem + L.off_dwf);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L.off_bars);
+    uint64_t *a_full = bars;                 // [kAStages]
+    uint64_t *a_empty = bars + kAStages;     // [kAStages]
+    uint64_t *tfull = a_empty + kAStages;    // [2]
+    uint64_t *tempty = tfull + 2;            // [2]
+    uint64_t *wbar = tempty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(wbar + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5;
+    const int lane = tid & 31;
+    const int Cin = p.Cin, Cout = p.Cout;
+    const int ncols = Cout <= 64 ? 64 : (Cout <= 128 ? 128 : 256);  // accumulator width (pow2)
+    const uint32_t tmem_cols = 2u * static_cast<uint32_t>(ncols);
+
+    if (tid == 0) {
+        for (int s = 0; s < kAStages; ++s) {
+            mbar_init(&a_full[s], 128);
+            mbar_init(&a_empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        mbar_init(wbar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    for (int i = tid; i < 9 * Cin; i += kThreads)
+        dwf[i] = __uint_as_float(static_cast<uint32_t>(p.dw[i]) << 16);
+    if (warp == 4) {
+        tmem_alloc(tmem_slot, tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const WaitCtx w{p.timeout_ns, p.err, abort_flag};
+
+    if (warp < 4) {
+        // ------------------------------------------------ depthwise producers
+        const int groups = Cin / 8;           // 16-byte channel groups per pixel
+        const int items = kBM * groups;
+        const long long HW = static_cast<long long>(p.H) * p.W;
+        int stage = 0;
+        uint32_t phase = 0;
+        for (int tile = blockIdx.x; tile < p.tiles; tile += gridDim.x) {
+            if (!bounded_wait(&a_empty[stage], phase ^ 1u, w, SITE_DW_AEMPTY)) break;
+            uint8_t *a = sA + stage * L.a_stage_bytes;
+            const long long p0 = static_cast<long long>(tile) * kBM;
+            for (int it = tid; it < items; it += 128) {
+                const int r = it / groups;
+                const int g = it - r * groups;
+                const long long pix = p0 + r;
+                if (pix >= p.M) continue;
+                const int n = static_cast<int>(pix / HW);
+                const long long rem = pix - static_cast<long long>(n) * HW;
+                const int y = static_cast<int>(rem / p.W);
+                const int xx = static_cast<int>(rem - static_cast<long long>(y) * p.W);
+                float acc[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
+#pragma unroll
+                for (int di = 0; di < 3; ++di) {
+                    const int yy = y + di - 1;
+                    if (yy < 0 || yy >= p.H) continue;
+#pragma unroll
+                    for (int dj = 0; dj < 3; ++dj) {
+                        const int xc = xx + dj - 1;
+                        if (xc < 0 || xc >= p.W) continue;
+                        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(
+                            p.x + ((static_cast<long long>(n) * p.H + yy) * p.W + xc) * Cin + g * 8));
+                        const float *wt = dwf + (di * 3 + dj) * Cin + g * 8;
+                        const float4 w0 = *reinterpret_cast<const float4 *>(wt);
+                        const float4 w1 = *reinterpret_cast<const float4 *>(wt + 4);
+                        acc[0] = fmaf(bf_lo(v.x), w0.x, acc[0]);
+                        acc[1] = fmaf(bf_hi(v.x), w0.y, acc[1]);
+                        acc[2] = fmaf(bf_lo(v.y), w0.z, acc[2]);
+                        acc[3] = fmaf(bf_hi(v.y), w0.w, acc[3]);
+                        acc[4] = fmaf(bf_lo(v.z), w1.x, acc[4]);
+                        acc[5] = fmaf(bf_hi(v.z), w1.y, acc[5]);
+                        acc[6] = fmaf(bf_lo(v.w), w1.z, acc[6]);
+                        acc[7] = fmaf(bf_hi(v.w), w1.w, acc[7]);
+                    }
+                }
+                uint4 o;
+                o.x = pack_bf16x2(acc[0], acc[1]);
+                o.y = pack_bf16x2(acc[2], acc[3]);
+                o.z = pack_bf16x2(acc[4], acc[5]);
+                o.w = pack_bf16x2(acc[6], acc[7]);
+                // K-major, 128-byte swizzle: atom g/8, row r, 16-byte chunk (g%8) ^ (r%8).
+                const int atom = g >> 3;
+                const int chunk = (g & 7) ^ (r & 7);
+                *reinterpret_cast<uint4 *>(a + atom * (kBM * 128) + r * 128 + chunk * 16) = o;
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(&a_full[stage]);
+            if (++stage == kAStages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+    } else if (warp == 4) {
+        // ------------------------------------------------ weights + MMA issuer
+        if (lane == 0) {
+            bool ok = true;
+            tma_prefetch_desc(&tmW);
+            mbar_arrive_expect_tx(wbar, static_cast<uint32_t>(L.w_bytes));
+            for (int kb = 0; kb < p.kb; ++kb)
+                for (int c = 0; c < p.nchunks; ++c)
+                    tma_load_2d(&tmW, wbar, sW + (kb * p.nchunks + c) * 8192, c * 64, kb * 64);
+            ok = bounded_wait(wbar, 0, w, SITE_DW_W);
+            const uint32_t idesc = idesc_bf16_f32(kBM, Cout, false, true);
+            const int ksteps = Cin / 16;
+            int stage = 0, acc = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            for (int tile = blockIdx.x; ok && tile < p.tiles; tile += gridDim.x) {
+                if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_DW_TEMPTY)) break;
+                if (!bounded_wait(&a_full[stage], phase, w, SITE_DW_AFULL)) break;
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA + stage * L.a_stage_bytes);
+                const uint32_t w0 = smem_u32(sW);
+                const uint32_t d = tmem_base + static_cast<uint32_t>(acc * ncols);
+                for (int ks = 0; ks < ksteps; ++ks) {
+                    const int atom = ks >> 2, kk = ks & 3;
+                    const uint64_t ad = sdesc_sw128(a0 + atom * (kBM * 128) + kk * 32, 16, 1024);
+                    const uint64_t bd = sdesc_sw128(w0 + atom * (p.nchunks * 8192) + kk * 2048, 8192, 1024);
+                    umma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
+                }
+                umma_commit(&a_empty[stage]);
+                umma_commit(&tfull[acc]);
+                if (++stage == kAStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+            }
+        }
+    } else {
+        // ------------------------------------------------ epilogue (warps 5-8)
+        const int q = warp & 3;
+        const int ew = warp - 5;
+        uint8_t *stg = sStage + ew * (kStageBufs * 4096);
+        int acc = 0, buf = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < p.tiles; tile += gridDim.x) {
+            if (!bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL)) break;
+            tc_fence_after();
+            const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                static_cast<uint32_t>(acc * ncols);
+            const int row0 = tile * kBM + q * 32;
+            for (int c = 0; c < Cout; c += 32) {
+                uint32_t r[32];
+                if (Cout - c >= 32) {
+                    tmem_ld32(tb + c, r);
+                } else {
+                    uint32_t h[16];
+                    tmem_ld16(tb + c, h);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        r[i] = h[i];
+                        r[16 + i] = 0u;
+                    }
+                }
+                tmem_ld_wait();
+                // Reuse of this staging buffer: its previous bulk store must have read it.
+                if (lane == 0) bulk_wait_read<kStageBufs - 1>();
+                __syncwarp();
+                uint8_t *sb = stg + buf * 4096;
+#pragma unroll
+                for (int ch = 0; ch < 8; ++ch) {
+                    const int pos = ch ^ (lane & 7);
+                    *reinterpret_cast<uint4 *>(sb + lane * 128 + pos * 16) =
+                        make_uint4(r[4 * ch], r[4 * ch + 1], r[4 * ch + 2], r[4 * ch + 3]);
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&tmOut, sb, c, row0);
+                    bulk_commit();
+                }
+                buf = (buf + 1) % kStageBufs;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+        if (lane == 0) bulk_wait_all<0>();
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 4) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, tmem_cols);
+    }
+}
+
+}  // namespace
+
+int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
+                 const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t stream) {
+    if (Cin % 16 != 0 || Cin < 16 || Cin > 256 || Cout % 16 != 0 || Cout < 16 || Cout > 256)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_dwsep_conv: needs Cin and Cout multiples of 16 in [16, 256] "
+                         "(Cin=%d Cout=%d)",
+                         Cin, Cout);
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dw) |
+         reinterpret_cast<uintptr_t>(pw) | reinterpret_cast<uintptr_t>(out)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: pointers must be 16-byte aligned");
+    const long long M = static_cast<long long>(N) * H * W;
+    if (M > (1ll << 31) - 256)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: N*H*W too large");
+    const DwLayout L = dw_layout(Cin, Cout);
+    if (L.total > ds.max_smem_optin)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_dwsep_conv: Cin=%d, Cout=%d does not fit shared memory", Cin, Cout);
+    int rc;
+    CUtensorMap tmW, tmOut;
+    if ((rc = make_tmap_2d_bf16(&tmW, pw, static_cast<uint64_t>(Cout), static_cast<uint64_t>(Cin),
+                                static_cast<uint64_t>(Cout) * 2, 64, 64)))
+        return rc;
+    if ((rc = make_tmap_2d_f32(&tmOut, out, static_cast<uint64_t>(Cout), static_cast<uint64_t>(M),
+                               static_cast<uint64_t>(Cout) * 4, 32, 32)))
+        return rc;
+    DwParams p{};
+    p.N = N;
+    p.H = H;
+    p.W = W;
+    p.Cin = Cin;
+    p.Cout = Cout;
+    p.M = M;
+    p.tiles = static_cast<int>((M + kBM - 1) / kBM);
+    p.atoms = (Cin + 63) / 64;
+    p.kb = (Cin + 63) / 64;
+    p.nchunks = (Cout + 63) / 64;
+    p.x = x;
+    p.dw = dw;
+    p.timeout_ns = wait_timeout_ns();
+    p.err = ds.err_word;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(dwsep_fused_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             ds.max_smem_optin);
+        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(dwsep)");
+        attr_set = true;
+    }
+    const int grid = p.tiles < ds.num_sms ? p.tiles : ds.num_sms;
+    dwsep_fused_kernel<<<grid, kThreads, L.total, stream>>>(tmW, tmOut, p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "launch dwsep_fused_kernel");
+    return ISAM_OK;
+}
+
 }  // namespace isam

@@ -144,6 +144,31 @@ __device__ __forceinline__ void tma_load_3d(const void *map, uint64_t *bar, void
         : "memory");
 }
 
+// Bulk tensor store shared -> global (rows/cols outside the tensor are clipped).
+__device__ __forceinline__ void tma_store_2d(const void *map, const void *src, int32_t c0, int32_t c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(smem_u32(src)), "r"(c0), "r"(c1)
+        : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+
+// Waits until at most N committed bulk groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+
+// Waits until at most N committed bulk groups are still in flight.
+template <int N>
+__device__ __forceinline__ void bulk_wait_all() {
+    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // Generic-proxy writes to global memory become visible to later async-proxy
 // (TMA) reads.
 __device__ __forceinline__ void fence_proxy_async_global() {

@@ -1,0 +1,92 @@
+"""Separable depthwise convolution parity on the GPU through the C ABI
+(isam_dwsep_conv) against the fp64 oracle.  Tolerance: normalised max error
+<= 5e-3; integer-valued inputs (depthwise sums exactly representable in bf16)
+must match bit for bit."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_1810_09958_gb300 import isam, synth
+from gpu_util import Guarded, dev_bf16, nmax_err
+
+pytestmark = pytest.mark.gpu
+TOL = 5e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import torch
+    from paper_1810_09958_gb300 import build
+    build.build()
+    isam.load()
+    torch.cuda.set_device(0)
+    yield
+    isam.sync()
+
+
+def run_dwsep(x, dw, pw):
+    N, H, W, Cin = x.shape
+    Cout = pw.shape[1]
+    out = Guarded(N * H * W * Cout)
+    isam.dwsep_conv(N, H, W, Cin, Cout, dev_bf16(x), dev_bf16(dw), dev_bf16(pw), out.t)
+    isam.sync()
+    assert out.guards_intact(), "write outside out"
+    return out.numpy().reshape(N, H, W, Cout)
+
+
+def test_dwsep_benchmark_layer_full_oracle():
+    """N = 32, 56 x 56, 128 -> 256 channels (the benchmark layer)."""
+    N, H, W, Cin, Cout = 32, 56, 56, 128, 256
+    x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=synth.stream_seed(synth.BASE_SEED, 4))
+    got = run_dwsep(x, dw, pw)
+    ref = oracle.dwsep(x, dw, pw)
+    assert nmax_err(got, ref) <= TOL
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1, 16, 32), (1, 5, 7, 16, 16), (2, 9, 8, 32, 48),
+                                   (3, 4, 33, 64, 96), (2, 13, 11, 128, 256), (1, 3, 130, 48, 16),
+                                   (1, 7, 19, 256, 64), (4, 2, 3, 80, 144)])
+def test_dwsep_shapes(shape):
+    N, H, W, Cin, Cout = shape
+    x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=sum(shape) * 31 + Cin)
+    got = run_dwsep(x, dw, pw)
+    ref = oracle.dwsep(x, dw, pw)
+    assert nmax_err(got, ref) <= TOL, shape
+
+
+def test_dwsep_integer_bit_exact():
+    N, H, W, Cin, Cout = 3, 10, 17, 64, 96
+    x = synth.bf16_integers(1, (N, H, W, Cin), -3, 3)
+    dw = synth.bf16_integers(2, (3, 3, Cin), -2, 2)
+    pw = synth.bf16_integers(3, (Cin, Cout), -2, 2)
+    got = run_dwsep(x, dw, pw)
+    ref = oracle.dwsep(x, dw, pw)
+    assert np.array_equal(got.astype(np.float64), ref)
+
+
+def test_dwsep_ones_window_boundary_pattern():
+    """All-ones window on a constant image with an identity pointwise stage:
+    9c inside, 6c on edges, 4c in corners."""
+    N, H, W, C = 2, 6, 9, 32
+    c = 1.5
+    x = synth.to_bf16_bits(np.full((N, H, W, C), c))
+    dw = synth.to_bf16_bits(np.ones((3, 3, C)))
+    pw = synth.to_bf16_bits(np.eye(C))
+    got = run_dwsep(x, dw, pw)
+    rows = np.array([2] + [3] * (H - 2) + [2])
+    cols = np.array([2] + [3] * (W - 2) + [2])
+    want = c * np.outer(rows, cols)
+    for k in range(C):
+        assert np.array_equal(got[0, :, :, k].astype(np.float64), want)
+
+
+def test_dwsep_unsupported_rejected():
+    import ctypes
+    import torch
+    z = torch.zeros(1 << 16, dtype=torch.bfloat16, device="cuda")
+    f = torch.zeros(1 << 16, dtype=torch.float32, device="cuda")
+    lib = isam.load()
+    p = lambda t: ctypes.c_void_p(t.data_ptr())
+    assert lib.isam_dwsep_conv(1, 4, 4, 24, 16, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_dwsep_conv(1, 4, 4, 16, 272, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_dwsep_conv(1, 4, 4, 256, 256, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
