@@ -1,0 +1,576 @@
+#!/usr/bin/env python3
+"""Benchmark of the GB300 hot path (isam C ABI) -- one JSON line on rank 0.
+
+Timed workload (one "step"): the tall-skinny GEMM sweep of the paper's
+DeepBench-sized GEMM benchmark (Section 5.1.1): (M, K) in {(1760,1760),
+(2560,2560), (4096,4096), (7680,2560)} x N in {16, 32, 64, 128} x {NN, TN},
+bf16 operands U[-1,1], fp32 accumulate and output, beta = 0.  32 GEMMs per
+step, each on its own operands (0.74 GB of inputs per step, larger than L2,
+so no GEMM finds its operands in L2 from the step before).
+
+value  = GEMM TFLOP/s over the sweep (all ranks' flops / max rank time).
+e2e    = the same through host buffers: pinned host -> device copies of every
+         operand, the GEMMs, device -> host copies of every result, per step.
+roofline: the sweep's kernel (gemm_tc_kernel) is HBM-bound: algorithmic bytes
+         (2MK + 2KN + 4MN per GEMM) / summed per-launch CUDA-event time, against
+         the measured copy bandwidth.
+hot_path: the other rows measured in the same run (not part of value): the
+         8192^3 GEMM with beta = 1 (TFLOP/s vs dense bf16), the GRU forward
+         (hidden 1024, batch 32, 128 steps: timesteps/s), the fused separable
+         depthwise layer (32x56x56, 128 -> 256: GB/s vs HBM).
+cpu_baseline: the fp64 oracle on the host cores, on a row sample of the sweep.
+
+--impl reference times the oracle itself (the only reference this build has)
+on the same workload's row sample, K steps after W warm-up steps.
+Multi-GPU (torchrun): every rank runs the whole sweep on its own GPU with no
+collective on the data path (weak scaling); timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+SWEEP_MK = [(1760, 1760), (2560, 2560), (4096, 4096), (7680, 2560)]
+SWEEP_N = [16, 32, 64, 128]
+METRIC = "GEMM TFLOP/s (tall-skinny sweep) and GRU timesteps/s on 1 GB300; % of roofline"
+WORKLOAD = ("tall-skinny GEMM sweep: (M,K) in {(1760,1760),(2560,2560),(4096,4096),(7680,2560)} "
+            "x N in {16,32,64,128} x {NN,TN}; bf16 U[-1,1]; fp32 accumulate/output; beta=0")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# --------------------------------------------------------------------------- host logic
+def sweep_problems():
+    """(M, N, K, transA) of the 32 GEMMs of one step, in launch order."""
+    return [(M, N, K, tA) for tA in (0, 1) for (M, K) in SWEEP_MK for N in SWEEP_N]
+
+
+def gemm_flops(M, N, K):
+    return 2.0 * M * N * K
+
+
+def gemm_bytes(M, N, K, beta=False):
+    return 2.0 * M * K + 2.0 * K * N + 4.0 * M * N * (2 if beta else 1)
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def reduce_max(x: float, backend_device=None) -> float:
+    """Max of a float over all ranks (identity without torch.distributed)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=backend_device or "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained")}, "measured"
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def row_sample(M: int, stride: int):
+    import numpy as np
+    return np.arange(0, M, stride, dtype=np.int32)
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampled every 200 ms in the background."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.rows = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return self
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.time(), [c.strip() for c in line.split(",")]))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            if self.thread:
+                self.thread.join(timeout=2)
+
+    def summary(self, t0: float, t1: float):
+        inside = [r for (t, r) in self.rows if t0 <= t <= t1]
+        window = "timed"
+        if not inside and self.rows:
+            mid = 0.5 * (t0 + t1)
+            inside = [min(self.rows, key=lambda tr: abs(tr[0] - mid))[1]]
+            window = "nearest"
+        if not inside:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm = [float(r[1]) for r in inside if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in inside if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i in range(4)
+                          if len(r) > 5 + i and r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(inside), "window": window}
+
+
+# --------------------------------------------------------------------------- GPU arm
+def make_sweep(dev):
+    import torch
+    from paper_1810_09958_gb300 import synth
+    probs = []
+    for (M, N, K, tA) in sweep_problems():
+        seed = synth.stream_seed(synth.BASE_SEED, 1, M, K, N, tA)
+        A = synth.bf16_uniform_torch(synth.stream_seed(seed, 1), M * K, dev)
+        B = synth.bf16_uniform_torch(synth.stream_seed(seed, 2), K * N, dev)
+        C = torch.empty(M * N, dtype=torch.float32, device=dev)
+        probs.append({"M": M, "N": N, "K": K, "tA": tA, "A": A, "B": B, "C": C,
+                      "flops": gemm_flops(M, N, K), "bytes": gemm_bytes(M, N, K)})
+    return probs
+
+
+def run_sweep(isam, probs):
+    for p in probs:
+        isam.gemm(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
+
+
+def time_sweep(isam, probs, steps, warmup):
+    """K steps of the sweep, each one replay of a CUDA graph holding the 32
+    GEMM launches (so host launch cost does not leak into microsecond kernels);
+    CUDA events on the replay stream bracket the timed region."""
+    import torch
+    for _ in range(warmup):
+        run_sweep(isam, probs)
+    isam.sync()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        run_sweep(isam, probs)
+    for _ in range(warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    start.record(stream)
+    for _ in range(steps):
+        graph.replay()
+    end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    isam.sync()
+    return start.elapsed_time(end), graph
+
+
+def time_e2e(isam, probs, steps, warmup):
+    """Same sweep through host buffers: H2D of operands, GEMMs, D2H of results."""
+    import torch
+    host = []
+    for p in probs:
+        host.append({"A": p["A"].cpu().pin_memory(), "B": p["B"].cpu().pin_memory(),
+                     "C": torch.empty(p["M"] * p["N"], dtype=torch.float32).pin_memory()})
+    h2d = sum(h["A"].numel() * 2 + h["B"].numel() * 2 for h in host)
+    d2h = sum(h["C"].numel() * 4 for h in host)
+
+    def one():
+        for p, h in zip(probs, host):
+            p["A"].copy_(h["A"], non_blocking=True)
+            p["B"].copy_(h["B"], non_blocking=True)
+            isam.gemm(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
+            h["C"].copy_(p["C"], non_blocking=True)
+
+    for _ in range(warmup):
+        one()
+    torch.cuda.synchronize()
+    barrier()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record()
+    for _ in range(steps):
+        one()
+    end.record()
+    torch.cuda.synchronize()
+    isam.sync()
+    return start.elapsed_time(end), h2d, d2h
+
+
+def time_call(fn, reps, warmup, flush=None):
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        if flush is not None:
+            flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        b.synchronize()
+        ts.append(a.elapsed_time(b))
+    return statistics.median(ts)
+
+
+def hot_path_rows(isam, dev, peaks):
+    """The remaining rows of the hot path, each timed on its benchmark shape."""
+    import torch
+    from paper_1810_09958_gb300 import synth
+    out = {}
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)  # 256 MB > L2
+    # 8192^3, beta = 1, N(0,1)*0.02 operands, C U[-1,1].
+    n = 8192
+    A = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 2, 1), n * n, dev, 0.0, 0.02)
+    B = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 2, 2), n * n, dev, 0.0, 0.02)
+    C = synth.f32_uniform_torch(synth.stream_seed(synth.BASE_SEED, 2, 3), n * n, dev)
+    ms = time_call(lambda: isam.gemm(n, n, n, 0, 0, 1.0, A, B, 1.0, C), reps=10, warmup=3)
+    tf = gemm_flops(n, n, n) / ms / 1e9
+    out["gemm_8192_beta1"] = {"ms": round(ms, 4), "tflops": round(tf, 1),
+                              "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4),
+                              "frac_bf16_sustained": round(tf / peaks["bf16_tflops_sustained"], 4),
+                              "plan": isam.gemm_plan(n, n, n, 0, 0, 1.0)}
+    del A, B, C
+    # GRU: hidden = input = 1024, batch 32, T = 128.
+    T, batch, H = 128, 32, 1024
+    s = 1.0 / 32.0
+    x = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 3, 1), T * batch * H, dev)
+    W = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 3, 2), 3 * H * H, dev, -s, s)
+    U = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 3, 3), 3 * H * H, dev, -s, s)
+    b = synth.f32_uniform_torch(synth.stream_seed(synth.BASE_SEED, 3, 4), 6 * H, dev, -0.1, 0.1)
+    h0 = torch.zeros(batch * H, dtype=torch.float32, device=dev)
+    hout = torch.empty(T * batch * H, dtype=torch.float32, device=dev)
+    ms = time_call(lambda: isam.gru_forward(T, batch, H, x, W, U, b, h0, hout), reps=10, warmup=3,
+                   flush=flush)
+    gflop = 2.0 * T * batch * 3 * H * (H + H) / 1e9
+    tf = gflop / ms
+    out["gru_h1024_b32_t128"] = {"ms": round(ms, 4), "timesteps_per_s": round(T / (ms / 1e3), 1),
+                                 "us_per_step": round(ms * 1e3 / T, 3), "tflops": round(tf, 2),
+                                 "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4)}
+    del x, W, U, b, h0, hout
+    # Separable depthwise layer.
+    N, Hh, Ww, Cin, Cout = 32, 56, 56, 128, 256
+    xd = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 4, 1), N * Hh * Ww * Cin, dev)
+    dw = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 4, 2), 9 * Cin, dev, -1 / 3, 1 / 3)
+    pw = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 4, 3), Cin * Cout, dev,
+                                  -Cin ** -0.5, Cin ** -0.5)
+    od = torch.empty(N * Hh * Ww * Cout, dtype=torch.float32, device=dev)
+    ms = time_call(lambda: isam.dwsep_conv(N, Hh, Ww, Cin, Cout, xd, dw, pw, od), reps=20, warmup=3,
+                   flush=flush)
+    byts = N * Hh * Ww * (Cin * 2 + Cout * 4) + 9 * Cin * 2 + Cin * Cout * 2
+    gbs = byts / ms / 1e6
+    out["dwsep_32x56x56_128_256"] = {"ms": round(ms, 4), "gbs": round(gbs, 1),
+                                     "frac_hbm": round(gbs / peaks["hbm_gbs"], 4),
+                                     "tflops": round(2.0 * N * Hh * Ww * Cin * (9 + Cout) / ms / 1e9, 2)}
+    isam.sync()
+    return out
+
+
+# --------------------------------------------------------------------------- CPU (oracle) arm
+def sample_operands(stride):
+    """Every stride-th row i of op(A) of each sweep GEMM, with its full B, drawn
+    from the same streams as the GPU arm's operands (the generator is
+    counter-based, so only the sampled entries are drawn).  Row r of the
+    returned A_sub is row rows[r] of op(A); the oracle then computes exactly
+    rows[r] of C as a (len(rows) x N x K) problem."""
+    import numpy as np
+    from paper_1810_09958_gb300 import synth
+    ops = []
+    for (M, N, K, tA) in sweep_problems():
+        seed = synth.stream_seed(synth.BASE_SEED, 1, M, K, N, tA)
+        rows = row_sample(M, stride).astype(np.uint64)
+        ks = np.arange(K, dtype=np.uint64)
+        idx = (ks[None, :] * np.uint64(M) + rows[:, None]) if tA else (rows[:, None] * np.uint64(K) + ks[None, :])
+        A_sub = synth.to_bf16_bits(synth.uniform_at(synth.stream_seed(seed, 1), idx))
+        B = synth.bf16_uniform(synth.stream_seed(seed, 2), (K, N))
+        ops.append((rows.size, N, K, A_sub, B))
+    return ops
+
+
+def oracle_sample_run(ops):
+    """The oracle on a row sample of every sweep GEMM; returns (seconds, flops)."""
+    import oracle
+    t0 = time.perf_counter()
+    flops = 0.0
+    for (R, N, K, A_sub, B) in ops:
+        oracle.gemm(R, N, K, 0, 0, 1.0, A_sub, B)
+        flops += 2.0 * R * N * K
+    return time.perf_counter() - t0, flops
+
+
+def full_pass_seconds():
+    """Oracle time of one full pass over the sweep, extrapolated from a
+    stride-64 row sample."""
+    probe = 64
+    t, _ = oracle_sample_run(sample_operands(probe))
+    return t * probe
+
+
+def stride_for(target_s, t_full):
+    return max(1, int(round(t_full / max(target_s, 1e-3))))
+
+
+def cpu_baseline(target_s=12.0):
+    """The oracle as it stands on this host's cores: a row sample of the sweep
+    (all rows when a full pass is short), repeated to about target_s."""
+    import oracle
+    t_full = full_pass_seconds()
+    stride = stride_for(target_s, t_full)
+    ops = sample_operands(stride)
+    reps = max(1, int(round(target_s / max(t_full / stride, 1e-3)))) if stride == 1 else 1
+    t, flops = 0.0, 0.0
+    for _ in range(reps):
+        dt, df = oracle_sample_run(ops)
+        t += dt
+        flops += df
+    rows = "all rows" if stride == 1 else f"every {stride}th row"
+    return {"value": flops / t / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"fp64 oracle, {rows} of each of the 32 sweep GEMMs, {reps} pass(es): "
+                      f"{flops / 1e9:.2f} GFLOP in {t:.1f} s"}
+
+
+def reference_arm(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    # Each step a row sample sized so that all W + K steps take about two minutes.
+    t_full = full_pass_seconds()
+    per_step = min(4.0, 120.0 / max(1, args.steps + args.warmup))
+    stride = stride_for(per_step, t_full)
+    ops = sample_operands(stride)
+    warm = sample_operands(stride * 8)
+    for _ in range(args.warmup):
+        oracle_sample_run(warm)
+    t_all, f_all = 0.0, 0.0
+    for _ in range(args.steps):
+        t, f = oracle_sample_run(ops)
+        t_all += t
+        f_all += f
+    v = f_all / t_all / 1e12
+    sample = (f"fp64 oracle, every {stride}th row of each of the 32 sweep GEMMs per step "
+              f"({f_all / args.steps / 1e9:.2f} GFLOP per step)")
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_all / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, "gemms_per_step": 32},
+            "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": oracle.num_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------------- single case
+def run_case(args):
+    """Times one hot-path call on its own (for profiling and sweeps):
+    gemm:M,N,K,transA,transB,beta | gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]."""
+    import torch
+    from paper_1810_09958_gb300 import build, isam, synth
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    if not os.path.exists(isam.LIB_PATH):
+        build.build()
+    isam.load()
+    kind, _, rest = args.case.partition(":")
+    vals = [float(v) for v in rest.split(",")] if rest else []
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)
+    if kind == "gemm":
+        M, N, K, tA, tB = (int(v) for v in vals[:5])
+        beta = vals[5] if len(vals) > 5 else 0.0
+        A = synth.bf16_uniform_torch(11, M * K, dev)
+        B = synth.bf16_uniform_torch(12, K * N, dev)
+        C = synth.f32_uniform_torch(13, M * N, dev)
+        fn = lambda: isam.gemm(M, N, K, tA, tB, 1.0, A, B, beta, C)
+        work = {"tflops": gemm_flops(M, N, K) / 1e12, "gb": gemm_bytes(M, N, K, beta != 0) / 1e9,
+                "plan": isam.gemm_plan(M, N, K, tA, tB, beta)}
+    elif kind == "gru":
+        T, batch, H = (int(v) for v in vals) if vals else (128, 32, 1024)
+        s = H ** -0.5
+        x = synth.bf16_normal_torch(21, T * batch * H, dev)
+        W = synth.bf16_uniform_torch(22, 3 * H * H, dev, -s, s)
+        U = synth.bf16_uniform_torch(23, 3 * H * H, dev, -s, s)
+        b = synth.f32_uniform_torch(24, 6 * H, dev, -0.1, 0.1)
+        hout = torch.empty(T * batch * H, dtype=torch.float32, device=dev)
+        fn = lambda: isam.gru_forward(T, batch, H, x, W, U, b, None, hout)
+        work = {"tflops": 2.0 * T * batch * 3 * H * 2 * H / 1e12, "timesteps": T}
+    elif kind == "dwsep":
+        N, H, W, Cin, Cout = (int(v) for v in vals) if vals else (32, 56, 56, 128, 256)
+        x = synth.bf16_normal_torch(31, N * H * W * Cin, dev)
+        dw = synth.bf16_uniform_torch(32, 9 * Cin, dev, -1 / 3, 1 / 3)
+        pw = synth.bf16_uniform_torch(33, Cin * Cout, dev, -Cin ** -0.5, Cin ** -0.5)
+        out = torch.empty(N * H * W * Cout, dtype=torch.float32, device=dev)
+        fn = lambda: isam.dwsep_conv(N, H, W, Cin, Cout, x, dw, pw, out)
+        work = {"gb": (N * H * W * (2 * Cin + 4 * Cout) + 18 * Cin + 2 * Cin * Cout) / 1e9,
+                "tflops": 2.0 * N * H * W * Cin * (9 + Cout) / 1e12}
+    else:
+        raise SystemExit(f"unknown case {args.case}")
+    ms = time_call(fn, reps=args.steps, warmup=args.warmup, flush=flush)
+    isam.sync()
+    res = {"case": args.case, "ms": round(ms, 5)}
+    if "tflops" in work:
+        res["tflops_per_s"] = round(work["tflops"] / (ms / 1e3), 2)
+    if "gb" in work:
+        res["gb_per_s"] = round(work["gb"] / (ms / 1e3), 1)
+    if "timesteps" in work:
+        res["timesteps_per_s"] = round(work["timesteps"] / (ms / 1e3), 1)
+    if "plan" in work:
+        res["plan"] = work["plan"]
+    print(json.dumps(res), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------------- main
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["isam", "reference"], default="isam")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-hot-path", action="store_true")
+    ap.add_argument("--case", default=None,
+                    help="time one call instead of the benchmark: gemm:M,N,K,tA,tB,beta | "
+                         "gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.case:
+        return run_case(args)
+
+    if args.impl == "reference":
+        return reference_arm(args)
+
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    from paper_1810_09958_gb300 import build, isam
+    if not os.path.exists(isam.LIB_PATH):
+        build.build()
+    isam.load()
+    peaks, peaks_src = read_peaks()
+
+    probs = make_sweep(dev)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(dev.index).start() if rank == 0 else None
+    time.sleep(0.3)
+    t0 = time.time()
+    total_ms, graph = time_sweep(isam, probs, args.steps, args.warmup)
+    t1 = time.time()
+    kern_ms = total_ms
+    total_ms = reduce_max(total_ms, dev)
+    flops_step = sum(p["flops"] for p in probs)
+    bytes_step = sum(p["bytes"] for p in probs)
+    value = flops_step * args.steps * world / (total_ms / 1e3) / 1e12
+    launches = args.steps * len(probs)
+
+    e2e_ms, h2d, d2h = time_e2e(isam, probs, max(3, args.steps // 20), 2)
+    e2e_ms = reduce_max(e2e_ms, dev)
+    e2e_steps = max(3, args.steps // 20)
+    e2e_value = flops_step * e2e_steps * world / (e2e_ms / 1e3) / 1e12
+
+    hot = None
+    if not args.no_hot_path:
+        hot = hot_path_rows(isam, dev, peaks)
+    if sampler:
+        sampler.stop()
+    del probs, graph
+    torch.cuda.empty_cache()
+
+    if rank == 0:
+        achieved = bytes_step * args.steps / (kern_ms / 1e3) / 1e9
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "gemms_per_step": 32,
+                       "l2": "inputs larger than L2: each GEMM has its own operands, "
+                             f"{bytes_step / 1e9:.2f} GB per step",
+                       "parallelism": f"replica x{world}"},
+            "roofline": {"kernel": "gemm_tc_kernel", "bound": "hbm", "achieved": round(achieved, 1),
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None,
+                         "peak_source": peaks_src,
+                         "algorithmic_bytes_per_step": bytes_step,
+                         "launches_per_step": 32,
+                         "timing": "the sweep is this kernel's 32 launches back to back in a CUDA "
+                                   "graph; duration = timed-region events / steps (inter-launch "
+                                   "gaps included)"},
+            "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+            "gpu_launches": launches,
+            "clocks": sampler.summary(t0, t1) if sampler else None,
+        }
+        if hot is not None:
+            line["hot_path"] = hot
+        if not args.no_cpu_baseline and world == 1:
+            import oracle
+            oracle.build()
+            line["cpu_baseline"] = cpu_baseline()
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -53,6 +53,16 @@ def uniform(seed: int, n: int, lo: float = -1.0, hi: float = 1.0) -> np.ndarray:
     return out
 
 
+def uniform_at(seed: int, idx: np.ndarray, lo: float = -1.0, hi: float = 1.0) -> np.ndarray:
+    """Draws number ``idx`` (any shape of non-negative indices) of the stream, as
+    uniform() would return them: uniform(seed, n)[idx] == uniform_at(seed, idx)."""
+    with np.errstate(over="ignore"):
+        z = _mix64(np.uint64(seed & 0xFFFFFFFFFFFFFFFF) +
+                   (np.asarray(idx, dtype=np.uint64) + np.uint64(1)) * _GOLDEN)
+    u = (z >> np.uint64(11)).astype(np.float64) * (1.0 / 9007199254740992.0)
+    return lo + (hi - lo) * u
+
+
 def normal(seed: int, n: int, mean: float = 0.0, std: float = 1.0) -> np.ndarray:
     """``n`` float64 normal values; value i uses draws 2i and 2i+1 (Box-Muller)."""
     out = np.empty(n, dtype=np.float64)
@@ -73,10 +83,10 @@ def integers(seed: int, n: int, lo: int, hi: int) -> np.ndarray:
 
 
 def to_bf16_bits(x: np.ndarray) -> np.ndarray:
-    """Rounds values to bfloat16 (round-to-nearest-even) and returns uint16 bits."""
+    """Rounds finite values to bfloat16 (round-to-nearest-even); uint16 bits."""
     f = np.ascontiguousarray(x, dtype=np.float32)
-    b = f.view(np.uint32).astype(np.uint64)
-    b = (b + np.uint64(0x7FFF) + ((b >> np.uint64(16)) & np.uint64(1))) >> np.uint64(16)
+    b = f.view(np.uint32)
+    b = (b + (np.uint32(0x7FFF) + ((b >> np.uint32(16)) & np.uint32(1)))) >> np.uint32(16)
     return b.astype(np.uint16).reshape(np.shape(x))
 
 
@@ -114,6 +124,71 @@ def bf16_integers(seed: int, shape, lo: int, hi: int) -> np.ndarray:
 def f32_uniform(seed: int, shape, lo=-1.0, hi=1.0) -> np.ndarray:
     n = int(np.prod(shape))
     return uniform(seed, n, lo, hi).astype(np.float32).reshape(shape)
+
+
+# ---------------------------------------------------------------------------
+# The same streams drawn with torch on any device (used to fill large device
+# buffers quickly).  Uniform draws are bit-identical to uniform()/bf16_uniform();
+# torch int64 arithmetic wraps modulo 2**64 like the uint64 version and right
+# shifts are made logical by masking.
+# ---------------------------------------------------------------------------
+def _to_i64(v: int) -> int:
+    v &= 0xFFFFFFFFFFFFFFFF
+    return v - (1 << 64) if v >= (1 << 63) else v
+
+
+def _lshr(z, s: int):
+    return (z >> s) & ((1 << (64 - s)) - 1)
+
+
+def splitmix64_torch(seed: int, start: int, count: int, device):
+    import torch
+    idx = torch.arange(start + 1, start + count + 1, dtype=torch.int64, device=device)
+    z = idx * _to_i64(0x9E3779B97F4A7C15) + _to_i64(seed)
+    z = (z ^ _lshr(z, 30)) * _to_i64(0xBF58476D1CE4E5B9)
+    z = (z ^ _lshr(z, 27)) * _to_i64(0x94D049BB133111EB)
+    return z ^ _lshr(z, 31)
+
+
+def bf16_uniform_torch(seed: int, n: int, device, lo=-1.0, hi=1.0):
+    """A flat torch.bfloat16 tensor on ``device``, bit-identical to bf16_uniform(seed, (n,))."""
+    import torch
+    out = torch.empty(n, dtype=torch.bfloat16, device=device)
+    chunk = 1 << 24
+    for s in range(0, n, chunk):
+        c = min(chunk, n - s)
+        z = splitmix64_torch(seed, s, c, device)
+        u = _lshr(z, 11).to(torch.float64) * (1.0 / 9007199254740992.0)
+        out[s:s + c] = (lo + (hi - lo) * u).to(torch.float32).to(torch.bfloat16)
+    return out
+
+
+def bf16_normal_torch(seed: int, n: int, device, mean=0.0, std=1.0):
+    """A flat torch.bfloat16 tensor of normal draws from the same stream as
+    normal() (device libm may differ from numpy's in the last bit of a rare
+    value; used only to fill timing inputs)."""
+    import torch
+    out = torch.empty(n, dtype=torch.bfloat16, device=device)
+    chunk = 1 << 23
+    for s in range(0, n, chunk):
+        c = min(chunk, n - s)
+        z = splitmix64_torch(seed, 2 * s, 2 * c, device)
+        u = (_lshr(z, 11).to(torch.float64) + 1.0) * (1.0 / 9007199254740992.0)
+        v = mean + std * torch.sqrt(-2.0 * torch.log(u[0::2])) * torch.cos(2.0 * math.pi * u[1::2])
+        out[s:s + c] = v.to(torch.float32).to(torch.bfloat16)
+    return out
+
+
+def f32_uniform_torch(seed: int, n: int, device, lo=-1.0, hi=1.0):
+    import torch
+    out = torch.empty(n, dtype=torch.float32, device=device)
+    chunk = 1 << 24
+    for s in range(0, n, chunk):
+        c = min(chunk, n - s)
+        z = splitmix64_torch(seed, s, c, device)
+        u = _lshr(z, 11).to(torch.float64) * (1.0 / 9007199254740992.0)
+        out[s:s + c] = (lo + (hi - lo) * u).to(torch.float32)
+    return out
 
 
 # ---------------------------------------------------------------------------

@@ -289,3 +289,25 @@ def test_bf16_rounding_is_nearest_even():
     bits = synth.to_bf16_bits(vals)
     back = synth.bf16_bits_to_f32(bits)
     assert back.tolist() == [1.0, 1.0, 1.0 + 2 ** -6, -2.5, 1.0]
+
+
+def test_torch_generator_matches_numpy():
+    torch = pytest.importorskip("torch")
+    n = 100_003
+    seed = synth.stream_seed(synth.BASE_SEED, 1, 7)
+    a = synth.bf16_uniform(seed, (n,))
+    b = synth.bf16_uniform_torch(seed, n, "cpu").view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(a, b)
+    c = synth.f32_uniform(seed, (n,))
+    d = synth.f32_uniform_torch(seed, n, "cpu").numpy()
+    assert np.array_equal(c, d)
+    e = synth.bf16_normal(seed, (n,)).astype(np.int32)
+    f = synth.bf16_normal_torch(seed, n, "cpu").view(torch.int16).numpy().view(np.uint16).astype(np.int32)
+    assert np.mean(e == f) > 0.999
+
+
+def test_uniform_at_matches_stream():
+    seed = synth.stream_seed(synth.BASE_SEED, 9)
+    full = synth.uniform(seed, 5000)
+    idx = np.array([[0, 4999, 17], [2500, 3, 3]])
+    assert np.array_equal(synth.uniform_at(seed, idx), full[idx])
