@@ -134,6 +134,39 @@ int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
                      const float *h0, float *h_out);
 
 /*
+ * GRU forward that allocates nothing.  The paper has no counterpart: this is a
+ * deployment variant of isam_gru_forward for callers that cannot let a library
+ * call cudaMalloc -- a process whose device memory is all reserved up front by
+ * its framework's caching allocator (a raw cudaMalloc would fail or fragment
+ * that pool), or a latency-bound request path that forbids cudaMalloc/cudaFree
+ * because they can synchronise the whole device.
+ *
+ * Same arguments, layouts, equations and support limits as isam_gru_forward
+ * (1 <= batch <= 32, hidden a multiple of 64 in [64, 1024], any T >= 1).  The
+ * caller still passes every input and h_out.  The workspaces live in one
+ * static 8 MiB device array inside libisam.so, which every GPU that loads the
+ * library holds until the process exits; the input projection is computed in
+ * chunks of time steps that fit it (20 steps at batch 32, hidden 1024), with h
+ * carried between chunks through h_out.  No cudaMalloc, cudaFree or other
+ * allocating routine is called.
+ *
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ *   - Every call shares the one array: calls that overlap on the GPU (other
+ *     streams, other host threads) race and corrupt each other.  The call
+ *     clears the parts that must start at zero (error word, step counter).
+ *   - Unlike the other calls it waits for its own work on the stream before
+ *     returning, so that it can report a device-side timeout itself:
+ *     ISAM_OK, ISAM_ERR_TIMEOUT (h_out undefined), ISAM_ERR_CUDA,
+ *     ISAM_ERR_INVALID_ARG or ISAM_ERR_UNSUPPORTED (sizes beyond the limits
+ *     above, misaligned pointers, a device other than sm_103a).
+ */
+int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam_bf16 *x,
+                             const isam_bf16 *W, const isam_bf16 *U, const float *b,
+                             const float *h0, float *h_out);
+
+/*
  * Separable depthwise convolution, NHWC: a 3x3 depthwise stage (stride 1,
  * zero border of one pixel, channel multiplier 1) followed by a pointwise
  * 1x1 stage, i.e. Listing 3 with s = 1 and c = 1, executed in the factored

@@ -18,6 +18,7 @@
 //      grid-wide step counter.  Every wait is bounded in time.
 #include <cstdio>
 #include <cstdlib>
+#include <mutex>
 
 #include <cuda_bf16.h>
 
@@ -392,3 +393,216 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
 }
 
 }  // namespace isam
+
+// ===========================================================================
+// Allocation-free variant of the GRU forward.
+//
+// Some callers cannot let a library call cudaMalloc: a serving process whose
+// device memory is all reserved up front by its framework's caching allocator
+// (a raw cudaMalloc would fail or fragment that pool), or a latency-bound
+// request path that forbids cudaMalloc/cudaFree because they can synchronise
+// the whole device.  isam_gru_forward_noalloc serves them: its workspaces
+// (device error word, step counter, hidden-state exchange buffer, and the
+// input projection of up to a chunk of time steps) live in the fixed array
+// below, so the call allocates nothing.  It launches the same two kernels as
+// isam_gru_forward, one time chunk after another, carrying h from one chunk to
+// the next through h_out.
+// ===========================================================================
+namespace isam {
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = static_cast<size_t>(8) << 20;  // 8 MiB
+constexpr size_t kNaErrOff = 0;      // 16-byte device error word
+constexpr size_t kNaCounterOff = 256;
+constexpr size_t kNaHxOff = 512;     // 2 x [32][H] bf16 exchange buffer
+
+}  // namespace
+}  // namespace isam
+
+// Every GPU that loads this library holds these 8 MiB until the process exits.
+static __device__ __align__(256) unsigned char g_gru_noalloc_scratch[isam::kNoAllocScratchBytes];
+
+namespace isam {
+namespace {
+
+struct NoAllocDevice {
+    bool ready = false;
+    unsigned char *scratch = nullptr;  // device address of g_gru_noalloc_scratch
+    int num_sms = 0;
+    int smem_optin = 0;
+};
+NoAllocDevice g_noalloc[64];
+std::mutex g_noalloc_mu;
+bool g_noalloc_attr = false;
+
+// Once per device, with that device current: the array's device address and
+// the device limits the launches need.  No allocation happens here.
+int noalloc_setup(int dev, NoAllocDevice *nd) {
+    int major = 0, minor = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (e != cudaSuccess) return cuda_error(e, "isam_gru_forward_noalloc: device attributes");
+    if (major != 10 || minor != 3)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gru_forward_noalloc: built for sm_103a (GB300); device %d is sm_%d%d",
+                         dev, major, minor);
+    void *ptr = nullptr;
+    e = cudaGetSymbolAddress(&ptr, g_gru_noalloc_scratch);
+    if (e != cudaSuccess || ptr == nullptr)
+        return cuda_error(e, "isam_gru_forward_noalloc: cudaGetSymbolAddress(scratch)");
+    if ((e = cudaDeviceGetAttribute(&nd->num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&nd->smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) !=
+            cudaSuccess)
+        return cuda_error(e, "isam_gru_forward_noalloc: device attributes");
+    nd->scratch = static_cast<unsigned char *>(ptr);
+    nd->ready = true;
+    return ISAM_OK;
+}
+
+}  // namespace
+}  // namespace isam
+
+extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam_bf16 *x,
+                                        const isam_bf16 *W, const isam_bf16 *U, const float *b,
+                                        const float *h0, float *h_out) {
+    using namespace isam;
+    const int H = hidden;
+    if (T < 1 || batch < 1 || H < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_noalloc: sizes must be >= 1");
+    if (!x || !W || !U || !b || !h_out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_noalloc: null pointer");
+    if (batch > kBatchPad || H % 64 != 0 || H > 1024 || H < 64)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gru_forward_noalloc: needs batch <= 32 and hidden a multiple of 64 "
+                         "in [64, 1024] (batch=%d hidden=%d)",
+                         batch, H);
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
+         reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |
+         reinterpret_cast<uintptr_t>(h0) | reinterpret_cast<uintptr_t>(h_out)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gru_forward_noalloc: pointers must be 16-byte aligned");
+    // Scratch layout: error word | step counter | exchange buffer | projection chunk.
+    const size_t hx_bytes = static_cast<size_t>(2) * kBatchPad * H * sizeof(uint16_t);
+    const size_t gx_off = (kNaHxOff + hx_bytes + 255) / 256 * 256;
+    const size_t step_bytes = static_cast<size_t>(batch) * 3 * H * sizeof(float);
+    const long long chunk = static_cast<long long>((kNoAllocScratchBytes - gx_off) / step_bytes);
+    if (chunk < 1)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gru_forward_noalloc: one step's projection (%zu bytes) exceeds the "
+                         "%zu-byte scratch",
+                         step_bytes, kNoAllocScratchBytes - gx_off);
+
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64)
+        return set_error(ISAM_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+    NoAllocDevice nd;
+    {
+        std::lock_guard<std::mutex> lk(g_noalloc_mu);
+        if (!g_noalloc[dev].ready) {
+            int rc = noalloc_setup(dev, &g_noalloc[dev]);
+            if (rc) return rc;
+        }
+        nd = g_noalloc[dev];
+        if (!g_noalloc_attr) {
+            e = cudaFuncSetAttribute(gru_recurrent_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     nd.smem_optin);
+            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
+            g_noalloc_attr = true;
+        }
+    }
+    const int n_cta = H / kUnits;
+    const size_t smem = gru_smem_bytes(H);
+    if (n_cta > nd.num_sms || smem > static_cast<size_t>(nd.smem_optin))
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward_noalloc: hidden too large");
+
+    uint32_t *err = reinterpret_cast<uint32_t *>(nd.scratch + kNaErrOff);
+    uint32_t *counter = reinterpret_cast<uint32_t *>(nd.scratch + kNaCounterOff);
+    uint16_t *hx = reinterpret_cast<uint16_t *>(nd.scratch + kNaHxOff);
+    float *gx = reinterpret_cast<float *>(nd.scratch + gx_off);
+    cudaStream_t stream = current_stream();
+
+    // A device view for the shared GEMM launcher: limits plus the scratch error word.
+    DeviceState view;
+    view.device = dev;
+    view.num_sms = nd.num_sms;
+    view.max_smem_optin = nd.smem_optin;
+    view.err_word = err;
+
+    int rc;
+    if ((e = cudaMemsetAsync(err, 0, 16, stream)) != cudaSuccess)
+        return cuda_error(e, "clearing the scratch error word");
+    CUtensorMap tmU, tmH0, tmH1;
+    {
+        const uint64_t dims[3] = {static_cast<uint64_t>(H), static_cast<uint64_t>(H), 3};
+        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, static_cast<uint64_t>(H) * H * 2};
+        const uint32_t box[3] = {64, kUnits, 3};
+        if ((rc = make_tmap_3d_bf16(&tmU, U, dims, strides, box))) return rc;
+    }
+    const int nk = H / 64;
+    const int nq = (nk % 4 == 0) ? 4 : (nk % 2 == 0) ? 2 : 1;
+    for (int i = 0; i < 2; ++i) {
+        const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(nk)};
+        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
+        const uint32_t box[3] = {64, kBatchPad, static_cast<uint32_t>(nk / nq)};
+        if ((rc = make_tmap_3d_bf16(i ? &tmH1 : &tmH0, hx + static_cast<size_t>(i) * kBatchPad * H,
+                                    dims, strides, box)))
+            return rc;
+    }
+    const size_t step_elems = static_cast<size_t>(batch) * H;
+    for (long long t0 = 0; t0 < T; t0 += chunk) {
+        const int tc = static_cast<int>(T - t0 < chunk ? T - t0 : chunk);
+        // Input projection of steps [t0, t0 + tc): gx = x W^T + b_ih.
+        GemmDesc g{tc * batch, 3 * H, H, 0, 1, 1.0f, 0.0f, x + static_cast<size_t>(t0) * step_elems, W,
+                   gx, b};
+        GemmPlan plan;
+        if ((rc = gemm_validate(g))) return rc;
+        if ((rc = gemm_plan(g, view, &plan))) return rc;
+        if ((rc = gemm_launch(g, plan, view, stream))) return rc;
+        // Recurrence over the chunk, starting from h_{t0 - 1} (h0 for the first chunk).
+        if ((e = cudaMemsetAsync(counter, 0, sizeof(uint32_t), stream)) != cudaSuccess)
+            return cuda_error(e, "clearing the scratch step counter");
+        GruParams p{};
+        p.T = tc;
+        p.batch = batch;
+        p.H = H;
+        p.nk = nk;
+        p.nq = nq;
+        p.qk = nk / nq;
+        p.n_cta = n_cta;
+        p.gx = gx;
+        p.b_hh = b + 3 * H;
+        p.h0 = t0 == 0 ? h0 : h_out + static_cast<size_t>(t0 - 1) * step_elems;
+        p.h_out = h_out + static_cast<size_t>(t0) * step_elems;
+        p.hx = hx;
+        p.counter = counter;
+        p.skip_publish_cta = -1;
+        p.timeout_ns = wait_timeout_ns();
+        p.err = err;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeCooperative;
+        attr[0].val.cooperative = 1;
+        cfg.gridDim = dim3(static_cast<unsigned>(n_cta), 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = stream;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
+        if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel (noalloc)");
+    }
+    // Report device-side timeouts of this call before returning.
+    if ((e = cudaStreamSynchronize(stream)) != cudaSuccess)
+        return cuda_error(e, "isam_gru_forward_noalloc: cudaStreamSynchronize");
+    uint32_t w[4] = {0, 0, 0, 0};
+    if ((e = cudaMemcpy(w, err, sizeof w, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_error(e, "isam_gru_forward_noalloc: reading the scratch error word");
+    if (w[0] != 0)
+        return set_error(ISAM_ERR_TIMEOUT,
+                         "isam_gru_forward_noalloc: a bounded device wait ran out (site 0x%x, "
+                         "block %u); h_out is undefined",
+                         w[1], w[2]);
+    return ISAM_OK;
+}
