@@ -125,9 +125,10 @@ int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta,
  * resident in shared memory and multiplies bf16(h_{t-1}) on the tensor cores
  * (h itself is carried in fp32).  Gates are evaluated in fp32.
  *
- * Supported: T >= 1, 1 <= batch <= 32, hidden a multiple of 128 with
- * hidden <= 2048 (hidden / 16 cooperating CTAs must be co-resident); all
- * pointers 16-byte aligned.  Otherwise ISAM_ERR_UNSUPPORTED.
+ * Supported: T >= 1, 1 <= batch <= 32, hidden a multiple of 64 in
+ * [64, 1024] (hidden / 16 cooperating CTAs, launched cooperatively so they
+ * are co-resident); all pointers 16-byte aligned.  Otherwise
+ * ISAM_ERR_UNSUPPORTED.
  */
 int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
                      const isam_bf16 *W, const isam_bf16 *U, const float *b,

@@ -4,14 +4,15 @@
 // pointwise weights, a GEMM with M = N*H*W pixels, K = Cin, N = Cout.
 //
 // One persistent kernel, one CTA per SM, 128-pixel tiles:
-//   warps 0-3  depthwise producers: read the 3x3 neighbourhood of each pixel
-//              with 16-byte NHWC loads, accumulate in fp32, round to bf16 and
-//              write the A tile straight into the tensor cores' 128-byte
-//              swizzled K-major layout (two-stage ring);
-//   warp 4     loads the pointwise weights once (TMA, resident for the whole
+//   warps 0-7  depthwise producers: for two pixels at a time issue all nine
+//              16-byte NHWC tap loads at once (clamped addresses, masked
+//              afterwards), accumulate in fp32, round to bf16 and write the A
+//              tile straight into the tensor cores' 128-byte swizzled K-major
+//              layout (two-stage ring);
+//   warp 8     loads the pointwise weights once (TMA, resident for the whole
 //              kernel) and issues tcgen05.mma from one thread into a
 //              double-buffered TMEM accumulator;
-//   warps 5-8  drain TMEM, stage 32x32 fp32 blocks in swizzled shared memory
+//   warps 9-12 drain TMEM, stage 32x32 fp32 blocks in swizzled shared memory
 //              and write them out with TMA bulk tensor stores.
 // The depthwise intermediate never leaves the chip.
 #include <cuda_bf16.h>
@@ -26,7 +27,11 @@ namespace isam {
 namespace {
 
 constexpr int kBM = 128;
-constexpr int kThreads = 288;
+constexpr int kProdWarps = 8;                 // depthwise producer warps 0-7
+constexpr int kProd = kProdWarps * 32;
+constexpr int kMmaWarp = kProdWarps;          // warp 8
+constexpr int kEpiWarp0 = kProdWarps + 1;     // warps 9-12
+constexpr int kThreads = (kProdWarps + 5) * 32;
 constexpr int kAStages = 2;
 constexpr int kStageBufs = 2;  // epilogue staging buffers per warp (4 KB each)
 
@@ -111,7 +116,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (tid == 0) {
         for (int s = 0; s < kAStages; ++s) {
-            mbar_init(&a_full[s], 128);
+            mbar_init(&a_full[s], kProd);
             mbar_init(&a_empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -124,7 +129,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = tid; i < 9 * Cin; i += kThreads)
         dwf[i] = __uint_as_float(static_cast<uint32_t>(p.dw[i]) << 16);
-    if (warp == 4) {
+    __syncwarp();
+    if (warp == kMmaWarp) {
         tmem_alloc(tmem_slot, tmem_cols);
         tmem_relinquish();
     }
@@ -134,61 +140,80 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx w{p.timeout_ns, p.err, abort_flag};
 
-    if (warp < 4) {
+    if (warp < kProdWarps) {
         // ------------------------------------------------ depthwise producers
         const int groups = Cin / 8;           // 16-byte channel groups per pixel
         const int items = kBM * groups;
-        const long long HW = static_cast<long long>(p.H) * p.W;
+        const int H = p.H, W = p.W, HW = p.H * p.W;
+        const int M = static_cast<int>(p.M);
+        const uint4 zero4 = make_uint4(0u, 0u, 0u, 0u);
         int stage = 0;
         uint32_t phase = 0;
         for (int tile = blockIdx.x; tile < p.tiles; tile += gridDim.x) {
             if (!bounded_wait(&a_empty[stage], phase ^ 1u, w, SITE_DW_AEMPTY)) break;
             uint8_t *a = sA + stage * L.a_stage_bytes;
-            const long long p0 = static_cast<long long>(tile) * kBM;
-            for (int it = tid; it < items; it += 128) {
-                const int r = it / groups;
-                const int g = it - r * groups;
-                const long long pix = p0 + r;
-                if (pix >= p.M) continue;
-                const int n = static_cast<int>(pix / HW);
-                const long long rem = pix - static_cast<long long>(n) * HW;
-                const int y = static_cast<int>(rem / p.W);
-                const int xx = static_cast<int>(rem - static_cast<long long>(y) * p.W);
-                float acc[8];
+            const int p0 = tile * kBM;
+            for (int it0 = tid; it0 < items; it0 += 2 * kProd) {
+                uint4 v[2][9];
+                int rr[2], gg[2];
+                bool live[2];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
+                for (int u = 0; u < 2; ++u) {
+                    const int it = it0 + u * kProd;
+                    const int r = it / groups;
+                    const int g = it - r * groups;
+                    const int pix = p0 + r;
+                    live[u] = it < items && pix < M;
+                    rr[u] = r;
+                    gg[u] = g;
+                    const int n = live[u] ? pix / HW : 0;
+                    const int rem = live[u] ? pix - n * HW : 0;
+                    const int y = rem / W;
+                    const int xx = rem - y * W;
+                    const uint16_t *img = p.x + static_cast<size_t>(n) * HW * Cin + g * 8;
 #pragma unroll
-                for (int di = 0; di < 3; ++di) {
-                    const int yy = y + di - 1;
-                    if (yy < 0 || yy >= p.H) continue;
-#pragma unroll
-                    for (int dj = 0; dj < 3; ++dj) {
-                        const int xc = xx + dj - 1;
-                        if (xc < 0 || xc >= p.W) continue;
-                        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(
-                            p.x + ((static_cast<long long>(n) * p.H + yy) * p.W + xc) * Cin + g * 8));
-                        const float *wt = dwf + (di * 3 + dj) * Cin + g * 8;
-                        const float4 w0 = *reinterpret_cast<const float4 *>(wt);
-                        const float4 w1 = *reinterpret_cast<const float4 *>(wt + 4);
-                        acc[0] = fmaf(bf_lo(v.x), w0.x, acc[0]);
-                        acc[1] = fmaf(bf_hi(v.x), w0.y, acc[1]);
-                        acc[2] = fmaf(bf_lo(v.y), w0.z, acc[2]);
-                        acc[3] = fmaf(bf_hi(v.y), w0.w, acc[3]);
-                        acc[4] = fmaf(bf_lo(v.z), w1.x, acc[4]);
-                        acc[5] = fmaf(bf_hi(v.z), w1.y, acc[5]);
-                        acc[6] = fmaf(bf_lo(v.w), w1.z, acc[6]);
-                        acc[7] = fmaf(bf_hi(v.w), w1.w, acc[7]);
+                    for (int t = 0; t < 9; ++t) {
+                        const int yy = y + t / 3 - 1;
+                        const int xc = xx + t % 3 - 1;
+                        const bool ok = live[u] && static_cast<unsigned>(yy) < static_cast<unsigned>(H) &&
+                                        static_cast<unsigned>(xc) < static_cast<unsigned>(W);
+                        const uint16_t *src = ok ? img + (static_cast<size_t>(yy) * W + xc) * Cin : p.x;
+                        const uint4 t4 = __ldg(reinterpret_cast<const uint4 *>(src));
+                        v[u][t] = ok ? t4 : zero4;
                     }
                 }
-                uint4 o;
-                o.x = pack_bf16x2(acc[0], acc[1]);
-                o.y = pack_bf16x2(acc[2], acc[3]);
-                o.z = pack_bf16x2(acc[4], acc[5]);
-                o.w = pack_bf16x2(acc[6], acc[7]);
-                // K-major, 128-byte swizzle: atom g/8, row r, 16-byte chunk (g%8) ^ (r%8).
-                const int atom = g >> 3;
-                const int chunk = (g & 7) ^ (r & 7);
-                *reinterpret_cast<uint4 *>(a + atom * (kBM * 128) + r * 128 + chunk * 16) = o;
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (!live[u]) continue;
+                    const int g = gg[u], r = rr[u];
+                    float acc[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
+#pragma unroll
+                    for (int t = 0; t < 9; ++t) {
+                        const float *wt = dwf + t * Cin + g * 8;
+                        const float4 w0 = *reinterpret_cast<const float4 *>(wt);
+                        const float4 w1 = *reinterpret_cast<const float4 *>(wt + 4);
+                        const uint4 q = v[u][t];
+                        acc[0] = fmaf(bf_lo(q.x), w0.x, acc[0]);
+                        acc[1] = fmaf(bf_hi(q.x), w0.y, acc[1]);
+                        acc[2] = fmaf(bf_lo(q.y), w0.z, acc[2]);
+                        acc[3] = fmaf(bf_hi(q.y), w0.w, acc[3]);
+                        acc[4] = fmaf(bf_lo(q.z), w1.x, acc[4]);
+                        acc[5] = fmaf(bf_hi(q.z), w1.y, acc[5]);
+                        acc[6] = fmaf(bf_lo(q.w), w1.z, acc[6]);
+                        acc[7] = fmaf(bf_hi(q.w), w1.w, acc[7]);
+                    }
+                    uint4 o;
+                    o.x = pack_bf16x2(acc[0], acc[1]);
+                    o.y = pack_bf16x2(acc[2], acc[3]);
+                    o.z = pack_bf16x2(acc[4], acc[5]);
+                    o.w = pack_bf16x2(acc[6], acc[7]);
+                    // K-major, 128-byte swizzle: atom g/8, row r, 16-byte chunk (g%8) ^ (r%8).
+                    const int atom = g >> 3;
+                    const int chunk = (g & 7) ^ (r & 7);
+                    *reinterpret_cast<uint4 *>(a + atom * (kBM * 128) + r * 128 + chunk * 16) = o;
+                }
             }
             fence_proxy_async_smem();
             mbar_arrive(&a_full[stage]);
@@ -197,7 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 phase ^= 1u;
             }
         }
-    } else if (warp == 4) {
+        __syncwarp();
+    } else if (warp == kMmaWarp) {
         // ------------------------------------------------ weights + MMA issuer
         if (lane == 0) {
             bool ok = true;
@@ -236,15 +262,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
+        __syncwarp();
     } else {
         // ------------------------------------------------ epilogue (warps 5-8)
         const int q = warp & 3;
-        const int ew = warp - 5;
+        const int ew = warp - kEpiWarp0;
         uint8_t *stg = sStage + ew * (kStageBufs * 4096);
         int acc = 0, buf = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < p.tiles; tile += gridDim.x) {
-            if (!bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL)) break;
+            if (!__all_sync(0xffffffffu, bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL) ? 1 : 0)) break;
             tc_fence_after();
             const uint32_t tb = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                 static_cast<uint32_t>(acc * ncols);
@@ -295,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     tc_fence_before();
     __syncthreads();
-    if (warp == 4) {
+    if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tmem_base, tmem_cols);
     }

@@ -48,7 +48,10 @@ struct GemmParams {
     int M, N, K;
     int m_tiles, n_tiles, kb_total;
     int split, stages, group_m;
+    int ka;      // 64-wide K atoms per pipeline stage (1, 2 or 4)
+    int kg_total;  // k-groups of ka atoms
     int n_vec4;  // 1 when N % 4 == 0 (16-byte stores in the split-K reduce)
+    int tma_c;   // 1: epilogue moves C with TMA (N % 4 == 0, BN >= 32, no split)
     float alpha, beta;
     float *C;
     const float *bias;
@@ -58,14 +61,16 @@ struct GemmParams {
 
 template <int BN, bool B_MN>
 struct Cfg {
-    static constexpr int kBBytes = B_MN ? ((BN + 63) / 64) * 8192 : BN * 128;
-    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kBAtom = B_MN ? ((BN + 63) / 64) * 8192 : BN * 128;  // one K atom of B
     static constexpr int kTmemCols = (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
     static constexpr int kCW = BN < 32 ? BN : 32;  // epilogue column chunk
 };
 
+// Epilogue shared memory: split-K partial tile, or per-warp staging (TMA
+// path: 2 x 4 KB per epilogue warp; plain path: a 32 x 33 fp32 transpose).
 __host__ __device__ inline size_t epi_bytes(int BN, int split) {
-    return split > 1 ? static_cast<size_t>(kBM) * (BN + 4) * 4 : static_cast<size_t>(4) * 32 * 33 * 4;
+    if (split > 1) return static_cast<size_t>(kBM) * (BN + 4) * 4;
+    return BN >= 32 ? static_cast<size_t>(4) * 2 * 4096 : static_cast<size_t>(4) * 32 * 33 * 4;
 }
 
 __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, int group_m,
@@ -89,19 +94,30 @@ __device__ bool drain_wait(uint64_t *bar, uint32_t parity, unsigned long long ti
     return true;
 }
 
+// bounded_wait by every lane of a warp, with a warp-uniform result.
+template <bool cluster_scope = false>
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, const WaitCtx &w,
+                                          uint32_t site) {
+    const bool ok = bounded_wait<cluster_scope>(bar, parity, w, site);
+    return __all_sync(0xffffffffu, ok) != 0;
+}
+
 template <int BN, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmParams p) {
+                   const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
     using C = Cfg<BN, B_MN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
     const int S = p.split;
     const int ST = p.stages;
+    const int KA = p.ka;
+    const int a_stage = KA * kABytes;
+    const int b_stage = KA * C::kBAtom;
     uint8_t *sA = smem;
-    uint8_t *sB = smem + static_cast<size_t>(ST) * kABytes;
-    float *ebuf = reinterpret_cast<float *>(sB + static_cast<size_t>(ST) * C::kBBytes);
+    uint8_t *sB = smem + static_cast<size_t>(ST) * a_stage;
+    float *ebuf = reinterpret_cast<float *>(sB + static_cast<size_t>(ST) * b_stage);
     uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(ebuf) + epi_bytes(BN, S));
     uint64_t *full = bars;
     uint64_t *empty = bars + ST;
@@ -109,7 +125,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *tempty = tfull + 2;
     uint64_t *red_full = tempty + 2;
     uint64_t *red_free = red_full + 1;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(red_free + 1);
+    uint64_t *cbar = red_free + 1;  // [4 epilogue warps][2] C-load barriers
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(cbar + 8);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -129,13 +146,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(red_full, S);
         mbar_init(red_free, S);
+        for (int i = 0; i < 8; ++i) mbar_init(&cbar[i], 1);
         *abort_flag = 0;
         fence_mbar_init();
-    }
-    if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
+        if (p.tma_c) tma_prefetch_desc(&tmC);
     }
+    __syncwarp();
     if (warp == 1) {
         tmem_alloc(tmem_slot, C::kTmemCols);
         tmem_relinquish();
@@ -147,8 +165,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx w{p.timeout_ns, p.err, abort_flag};
 
-    const int kb_begin = static_cast<int>((static_cast<long long>(rank) * p.kb_total) / S);
-    const int kb_end = static_cast<int>((static_cast<long long>(rank + 1) * p.kb_total) / S);
+    const int kg_begin = static_cast<int>((static_cast<long long>(rank) * p.kg_total) / S);
+    const int kg_end = static_cast<int>((static_cast<long long>(rank + 1) * p.kg_total) / S);
     const int num_tiles = p.m_tiles * p.n_tiles;
 
     if (warp == 0) {
@@ -161,27 +179,31 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int tile = cluster_id; ok && tile < num_tiles; tile += num_clusters) {
                 int mt, nt;
                 tile_coords(tile, p.m_tiles, p.n_tiles, p.group_m, mt, nt);
-                for (int kb = kb_begin; kb < kb_end; ++kb) {
+                for (int kg = kg_begin; kg < kg_end; ++kg) {
                     if (!bounded_wait(&empty[stage], phase ^ 1u, w, SITE_PROD_EMPTY)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
-                    uint8_t *a = sA + static_cast<size_t>(stage) * kABytes;
-                    uint8_t *b = sB + static_cast<size_t>(stage) * C::kBBytes;
-                    const int k0 = kb * kBK;
-                    if (A_MN) {
-                        tma_load_2d(&tmA, &full[stage], a, mt * kBM, k0);
-                        tma_load_2d(&tmA, &full[stage], a + 8192, mt * kBM + 64, k0);
-                    } else {
-                        tma_load_2d(&tmA, &full[stage], a, k0, mt * kBM);
-                    }
-                    if (B_MN) {
+                    mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(a_stage + b_stage));
+                    uint8_t *a = sA + static_cast<size_t>(stage) * a_stage;
+                    uint8_t *b = sB + static_cast<size_t>(stage) * b_stage;
+                    for (int at = 0; at < KA; ++at) {
+                        const int k0 = (kg * KA + at) * kBK;
+                        uint8_t *aa = a + at * kABytes;
+                        uint8_t *bb = b + at * C::kBAtom;
+                        if (A_MN) {
+                            tma_load_2d(&tmA, &full[stage], aa, mt * kBM, k0);
+                            tma_load_2d(&tmA, &full[stage], aa + 8192, mt * kBM + 64, k0);
+                        } else {
+                            tma_load_2d(&tmA, &full[stage], aa, k0, mt * kBM);
+                        }
+                        if (B_MN) {
 #pragma unroll
-                        for (int c = 0; c < (BN + 63) / 64; ++c)
-                            tma_load_2d(&tmB, &full[stage], b + c * 8192, nt * BN + c * 64, k0);
-                    } else {
-                        tma_load_2d(&tmB, &full[stage], b, k0, nt * BN);
+                            for (int c = 0; c < (BN + 63) / 64; ++c)
+                                tma_load_2d(&tmB, &full[stage], bb + c * 8192, nt * BN + c * 64, k0);
+                        } else {
+                            tma_load_2d(&tmB, &full[stage], bb, k0, nt * BN);
+                        }
                     }
                     ++issued;
                     if (++stage == ST) {
@@ -204,6 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
+        __syncwarp();
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
@@ -217,21 +240,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_MMA_TEMPTY)) break;
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(acc * BN);
-                for (int kb = kb_begin; kb < kb_end; ++kb) {
+                for (int kg = kg_begin; kg < kg_end; ++kg) {
                     if (!bounded_wait(&full[stage], phase, w, SITE_MMA_FULL)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a0 = smem_u32(sA + static_cast<size_t>(stage) * kABytes);
-                    const uint32_t b0 = smem_u32(sB + static_cast<size_t>(stage) * C::kBBytes);
+                    const uint32_t a0 = smem_u32(sA + static_cast<size_t>(stage) * a_stage);
+                    const uint32_t b0 = smem_u32(sB + static_cast<size_t>(stage) * b_stage);
+                    for (int at = 0; at < KA; ++at) {
+                        const uint32_t aa = a0 + at * kABytes;
+                        const uint32_t bb = b0 + at * C::kBAtom;
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        const uint64_t ad = A_MN ? sdesc_sw128(a0 + k * 2048, 8192, 1024)
-                                                 : sdesc_sw128(a0 + k * 32, 16, 1024);
-                        const uint64_t bd = B_MN ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
-                                                 : sdesc_sw128(b0 + k * 32, 16, 1024);
-                        umma_bf16(d, ad, bd, idesc, (kb > kb_begin || k > 0) ? 1u : 0u);
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint64_t ad = A_MN ? sdesc_sw128(aa + k * 2048, 8192, 1024)
+                                                     : sdesc_sw128(aa + k * 32, 16, 1024);
+                            const uint64_t bd = B_MN ? sdesc_sw128(bb + k * 2048, 8192, 1024)
+                                                     : sdesc_sw128(bb + k * 32, 16, 1024);
+                            umma_bf16(d, ad, bd, idesc, (kg > kg_begin || at > 0 || k > 0) ? 1u : 0u);
+                        }
                     }
                     umma_commit(&empty[stage]);
                     if (++stage == ST) {
@@ -247,11 +274,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
+        __syncwarp();
     } else {
         // ------------------------------------------------ epilogue (warps 2-5)
         const int ew = warp - 2;          // 0..3
         const int q = warp & 3;           // TMEM lane quadrant this warp may read
         const int row_local = q * 32 + lane;
+        const bool use_tma = (S == 1) && (BN >= 32) && (p.tma_c != 0);
+        const bool load_c = use_tma && (p.beta != 0.0f);
+        uint8_t *stg = reinterpret_cast<uint8_t *>(ebuf) + ew * 8192;  // TMA path: 2 x 4 KB
+        uint64_t *cb = cbar + ew * 2;
+        uint32_t cpar[2] = {0u, 0u};
+        bool cpend[2] = {false, false};
+        int gbuf = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
         int iter = 0;
@@ -259,14 +294,89 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int tile = cluster_id; tile < num_tiles; tile += num_clusters, ++iter) {
             int mt, nt;
             tile_coords(tile, p.m_tiles, p.n_tiles, p.group_m, mt, nt);
-            if (!bounded_wait(&tfull[acc], acc_phase, w, SITE_EPI_TFULL)) {
+            const int row0 = mt * kBM + q * 32;
+            const int col0 = nt * BN;
+            if (load_c) {
+                // Prefetch the first C chunk of this tile while its MMAs run.
+                if (lane == 0) {
+                    bulk_wait_read<0>();
+                    const int b = gbuf & 1;
+                    mbar_arrive_expect_tx(&cb[b], 4096);
+                    tma_load_2d(&tmC, &cb[b], stg + b * 4096, col0, row0);
+                }
+                cpend[gbuf & 1] = true;
+                __syncwarp();
+            }
+            if (!warp_wait(&tfull[acc], acc_phase, w, SITE_EPI_TFULL)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN);
-            if (S == 1) {
+            if (use_tma) {
+                if constexpr (BN >= 32) {
+#pragma unroll 1
+                    for (int j = 0; j < BN / 32; ++j) {
+                        const int b = gbuf & 1;
+                        if (load_c && j + 1 < BN / 32) {
+                            if (lane == 0) {
+                                bulk_wait_read<0>();  // buffer b^1: its last store has read it
+                                mbar_arrive_expect_tx(&cb[b ^ 1], 4096);
+                                tma_load_2d(&tmC, &cb[b ^ 1], stg + (b ^ 1) * 4096, col0 + (j + 1) * 32, row0);
+                            }
+                            cpend[b ^ 1] = true;
+                        }
+                        if (!load_c && lane == 0) bulk_wait_read<1>();  // buffer b: store of 2 chunks ago
+                        uint32_t r[32];
+                        tmem_ld32(tbase + j * 32, r);
+                        tmem_ld_wait();
+                        if (load_c) {
+                            if (!warp_wait(&cb[b], cpar[b], w, SITE_EPI_TFULL)) {
+                                ok = false;
+                                break;
+                            }
+                            cpar[b] ^= 1u;
+                            cpend[b] = false;
+                        }
+                        __syncwarp();
+                        uint8_t *sb = stg + b * 4096;
+                        const int cbase = col0 + j * 32;
+#pragma unroll
+                        for (int ch = 0; ch < 8; ++ch) {
+                            const int pos = ch ^ (lane & 7);
+                            float4 *slot = reinterpret_cast<float4 *>(sb + lane * 128 + pos * 16);
+                            float4 v = make_float4(p.alpha * __uint_as_float(r[4 * ch]),
+                                                   p.alpha * __uint_as_float(r[4 * ch + 1]),
+                                                   p.alpha * __uint_as_float(r[4 * ch + 2]),
+                                                   p.alpha * __uint_as_float(r[4 * ch + 3]));
+                            if (p.bias != nullptr && cbase + 4 * ch < p.N) {
+                                const float4 bv = __ldg(reinterpret_cast<const float4 *>(p.bias + cbase + 4 * ch));
+                                v.x += bv.x;
+                                v.y += bv.y;
+                                v.z += bv.z;
+                                v.w += bv.w;
+                            }
+                            if (load_c) {
+                                const float4 cv = *slot;
+                                v.x += p.beta * cv.x;
+                                v.y += p.beta * cv.y;
+                                v.z += p.beta * cv.z;
+                                v.w += p.beta * cv.w;
+                            }
+                            *slot = v;
+                        }
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tmC, sb, cbase, row0);
+                            bulk_commit();
+                        }
+                        ++gbuf;
+                    }
+                    if (!ok) break;
+                }
+            } else if (S == 1) {
                 float *tb = ebuf + ew * (32 * 33);
                 constexpr int CW = C::kCW;
                 constexpr int RPI = 32 / CW;  // rows per store iteration
@@ -284,30 +394,34 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < CW; ++j) tb[lane * 33 + j] = __uint_as_float(r[j]);
                     __syncwarp();
-                    const int gcol = nt * BN + c + col;
+                    const int gcol = col0 + c + col;
                     const float bias = (p.bias != nullptr && gcol < p.N) ? p.bias[gcol] : 0.0f;
-#pragma unroll 4
-                    for (int rr = sub; rr < 32; rr += RPI) {
-                        const int grow = mt * kBM + q * 32 + rr;
+                    float cin[32 / RPI];
+                    if (p.beta != 0.0f) {
+#pragma unroll
+                        for (int i = 0; i < 32 / RPI; ++i) {
+                            const int grow = row0 + sub + i * RPI;
+                            cin[i] = (grow < p.M && gcol < p.N) ? p.C[static_cast<size_t>(grow) * p.N + gcol] : 0.0f;
+                        }
+                    }
+#pragma unroll
+                    for (int i = 0; i < 32 / RPI; ++i) {
+                        const int rr = sub + i * RPI;
+                        const int grow = row0 + rr;
                         if (grow < p.M && gcol < p.N) {
-                            const size_t idx = static_cast<size_t>(grow) * p.N + gcol;
                             float v = p.alpha * tb[rr * 33 + col] + bias;
-                            if (p.beta != 0.0f) v += p.beta * p.C[idx];
-                            p.C[idx] = v;
+                            if (p.beta != 0.0f) v += p.beta * cin[i];
+                            p.C[static_cast<size_t>(grow) * p.N + gcol] = v;
                         }
                     }
                     __syncwarp();
                 }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&tempty[acc]);
             } else {
                 // Split-K: park this CTA's partial tile in shared memory, then
                 // every CTA of the cluster reduces its own row slice over all
                 // ranks in rank order.
                 if (iter > 0 &&
-                    !bounded_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w,
-                                        SITE_EPI_REDFREE)) {
+                    !warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE)) {
                     ok = false;
                     break;
                 }
@@ -330,22 +444,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&tempty[acc]);
+                __syncwarp();
                 named_bar(1, 128);
                 if (ew == 0 && lane == 0) {
                     for (int r = 0; r < S; ++r) mbar_arrive_remote(red_full, static_cast<uint32_t>(r));
                 }
-                if (!bounded_wait<true>(red_full, static_cast<uint32_t>(iter & 1), w,
-                                        SITE_EPI_REDFULL)) {
+                __syncwarp();
+                if (!warp_wait<true>(red_full, static_cast<uint32_t>(iter & 1), w, SITE_EPI_REDFULL)) {
                     ok = false;
                     break;
                 }
                 const int rows_per = kBM / S;
-                const int row0 = static_cast<int>(rank) * rows_per;
+                const int rl0 = static_cast<int>(rank) * rows_per;
                 const int g4 = BN / 4;
                 const int groups = rows_per * g4;
                 for (int g = ew * 32 + lane; g < groups; g += 128) {
-                    const int rl = row0 + g / g4;
+                    const int rl = rl0 + g / g4;
                     const int c4 = (g % g4) * 4;
+                    const int grow = mt * kBM + rl;
+                    const int gcol = col0 + c4;
+                    if (grow >= p.M) continue;
+                    float *crow = p.C + static_cast<size_t>(grow) * p.N;
+                    float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
+                    const bool vec = p.n_vec4 && gcol + 3 < p.N;
+                    if (p.beta != 0.0f && vec) cin = *reinterpret_cast<const float4 *>(crow + gcol);
                     const uint32_t local = smem_u32(ebuf + static_cast<size_t>(rl) * (BN + 4) + c4);
                     float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
                     for (int r = 0; r < S; ++r) {
@@ -355,16 +477,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         s.z += v.z;
                         s.w += v.w;
                     }
-                    const int grow = mt * kBM + rl;
-                    const int gcol = nt * BN + c4;
-                    if (grow >= p.M) continue;
-                    float *crow = p.C + static_cast<size_t>(grow) * p.N;
                     float o[4] = {s.x, s.y, s.z, s.w};
-                    if (p.n_vec4 && gcol + 3 < p.N) {
+                    if (vec) {
                         float4 v;
                         float *vv = reinterpret_cast<float *>(&v);
-                        float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
-                        if (p.beta != 0.0f) cin = *reinterpret_cast<const float4 *>(crow + gcol);
                         const float *ci = reinterpret_cast<const float *>(&cin);
 #pragma unroll
                         for (int j = 0; j < 4; ++j) {
@@ -382,10 +498,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
+                __syncwarp();
                 named_bar(1, 128);
                 if (ew == 0 && lane == 0) {
                     for (int r = 0; r < S; ++r) mbar_arrive_remote(red_free, static_cast<uint32_t>(r));
                 }
+                __syncwarp();
+            }
+            if (S == 1) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty[acc]);
+                __syncwarp();
             }
             if (++acc == 2) {
                 acc = 0;
@@ -393,9 +517,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         // Split-K: no peer may still be reading this CTA's partial tile when it exits.
-        if (S > 1 && ok && iter > 0) {
-            bounded_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE);
+        if (S > 1 && ok && iter > 0)
+            warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE);
+        // TMA path: C loads still in flight land, stores complete, before exit.
+        if (use_tma) {
+            for (int b = 0; b < 2; ++b)
+                if (cpend[b] && lane == 0) drain_wait(&cb[b], cpar[b], p.timeout_ns);
+            if (lane == 0) bulk_wait_all<0>();
         }
+        __syncwarp();
     }
 
     tc_fence_before();
@@ -407,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------- host side
-using KernelFn = void (*)(CUtensorMap, CUtensorMap, GemmParams);
+using KernelFn = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams);
 
 template <int BN>
 KernelFn pick3(bool a_mn, bool b_mn) {
@@ -428,14 +558,14 @@ KernelFn pick_kernel(int BN, bool a_mn, bool b_mn) {
 
 int b_bytes(int BN, bool b_mn) { return b_mn ? ((BN + 63) / 64) * 8192 : BN * 128; }
 
-size_t smem_bytes(int BN, bool b_mn, int split, int stages) {
-    return 1024 + static_cast<size_t>(stages) * (kABytes + b_bytes(BN, b_mn)) + epi_bytes(BN, split) +
-           (2 * stages + 6) * 8 + 16;
+size_t smem_bytes(int BN, bool b_mn, int split, int stages, int ka) {
+    return 1024 + static_cast<size_t>(stages) * ka * (kABytes + b_bytes(BN, b_mn)) +
+           epi_bytes(BN, split) + (2 * stages + 14) * 8 + 16;
 }
 
-int max_stages(int BN, bool b_mn, int split, int smem_limit) {
+int max_stages(int BN, bool b_mn, int split, int ka, int smem_limit) {
     int st = 8;
-    while (st > 2 && smem_bytes(BN, b_mn, split, st) > static_cast<size_t>(smem_limit)) --st;
+    while (st > 2 && smem_bytes(BN, b_mn, split, st, ka) > static_cast<size_t>(smem_limit)) --st;
     return st;
 }
 
@@ -553,19 +683,25 @@ int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
             }
         }
     }
+    bp.ka = 1;
     if (const char *f = getenv("ISAM_FORCE_TILE")) {
-        int fbn = 0, fs = 0, fst = 0;
-        if (sscanf(f, "%d,%d,%d", &fbn, &fs, &fst) >= 2 && pick_kernel(fbn, false, false) &&
-            (fs == 1 || fs == 2 || fs == 4 || fs == 8) && fs <= kb && !(fs > 1 && fbn > 128)) {
-            bp.BN = fbn;
-            bp.split = fs;
-            estimate_us(g, fbn, fs, nsm, &bp.grid);
-            if (fst >= 2) bp.stages = fst;
+        // "BN,split[,stages[,atoms per stage]]" (0 = the model's choice).
+        int fbn = 0, fs = 0, fst = 0, fka = 0;
+        if (sscanf(f, "%d,%d,%d,%d", &fbn, &fs, &fst, &fka) >= 2 && pick_kernel(fbn, false, false) &&
+            (fs == 1 || fs == 2 || fs == 4 || fs == 8) && !(fs > 1 && fbn > 128)) {
+            const int ka = (fka == 2 || fka == 4) ? fka : 1;
+            if (fs <= ceil_div(kb, ka)) {
+                bp.BN = fbn;
+                bp.split = fs;
+                bp.ka = ka;
+                estimate_us(g, fbn, fs, nsm, &bp.grid);
+                if (fst >= 2) bp.stages = fst;
+            }
         }
     }
-    const int st_max = max_stages(bp.BN, b_mn, bp.split, ds.max_smem_optin);
+    const int st_max = max_stages(bp.BN, b_mn, bp.split, bp.ka, ds.max_smem_optin);
     if (bp.stages < 2 || bp.stages > st_max) bp.stages = st_max;
-    bp.smem = smem_bytes(bp.BN, b_mn, bp.split, bp.stages);
+    bp.smem = smem_bytes(bp.BN, b_mn, bp.split, bp.stages, bp.ka);
     bp.group_m = 16;
     if (bp.smem > static_cast<size_t>(ds.max_smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: tile does not fit shared memory");
@@ -576,7 +712,8 @@ int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
 int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t stream) {
     const bool a_mn = g.transA == 1;
     const bool b_mn = g.transB == 0;
-    CUtensorMap ta, tb;
+    CUtensorMap ta, tb, tc;
+    memset(&tc, 0, sizeof tc);
     int rc;
     if (a_mn)
         rc = make_tmap_2d_bf16(&ta, g.A, g.M, g.K, static_cast<uint64_t>(g.M) * 2, 64, 64);
@@ -589,6 +726,11 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
         rc = make_tmap_2d_bf16(&tb, g.B, g.K, g.N, static_cast<uint64_t>(g.K) * 2, 64,
                                static_cast<uint32_t>(plan.BN));
     if (rc) return rc;
+    // The epilogue moves C with TMA when rows are 16-byte aligned (N % 4 == 0)
+    // and the tile is at least one 32-column chunk wide.
+    const int tma_c = (g.N % 4 == 0 && plan.BN >= 32 && plan.split == 1) ? 1 : 0;
+    if (tma_c && (rc = make_tmap_2d_f32(&tc, g.C, g.N, g.M, static_cast<uint64_t>(g.N) * 4, 32, 32)))
+        return rc;
 
     GemmParams p{};
     p.M = g.M;
@@ -597,6 +739,9 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
     p.m_tiles = ceil_div(g.M, kBM);
     p.n_tiles = ceil_div(g.N, plan.BN);
     p.kb_total = ceil_div(g.K, kBK);
+    p.ka = plan.ka;
+    p.kg_total = ceil_div(p.kb_total, plan.ka);
+    p.tma_c = tma_c;
     p.split = plan.split;
     p.stages = plan.stages;
     p.group_m = plan.group_m;
@@ -627,7 +772,7 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
         attr[0].val.clusterDim.z = 1;
         cfg.numAttrs = 1;
     }
-    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, ta, tb, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, ta, tb, tc, p);
     if (e != cudaSuccess) return cuda_error(e, "launch gemm_tc_kernel");
     return ISAM_OK;
 }

@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         fence_mbar_init();
     }
+    __syncwarp();
     if (warp == 0) {
         tmem_alloc(tmem_slot, 32);
         tmem_relinquish();
@@ -157,10 +158,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (b < p.batch) p.hx[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hprev[k]);
     }
     fence_proxy_async_global();
+    __syncwarp();
     __syncthreads();
     if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta) red_release_gpu_add(p.counter, 1u);
     bool ok = true;
     if (tid == 32) ok = bounded_wait(ubar, 0, w, SITE_GRU_U);
+    __syncwarp();
 
     const uint32_t idesc = idesc_bf16_f32(128, kBatchPad, false, false);
     int issued_phase = -1;  // last step whose h loads were issued (for the drain)
@@ -179,6 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issued_phase = t;
             }
         }
+        __syncwarp();
         // Input projection of this step (independent of h): prefetch.
         float gxr[4], gxz[4], gxn[4];
 #pragma unroll
@@ -212,7 +216,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (ok) umma_commit(mma_done);
         }
-        if (!bounded_wait(mma_done, par, w, SITE_GRU_MMA)) break;
+        __syncwarp();
+        // Block-uniform decision: every thread leaves the loop at the same step.
+        if (!__syncthreads_and(bounded_wait(mma_done, par, w, SITE_GRU_MMA) ? 1 : 0)) break;
         tc_fence_after();
         if (warp < 2) {
             uint32_t r[32];
@@ -246,8 +252,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
         if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
             red_release_gpu_add(p.counter, 1u);
+        __syncwarp();
         tc_fence_after();
-        if (*abort_flag) break;
     }
 
     // ---- teardown: let issued copies land, release TMEM.
@@ -259,6 +265,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (globaltimer() - t0 > p.timeout_ns) break;
         }
     }
+    __syncwarp();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {

@@ -54,6 +54,7 @@ struct GemmDesc {
 // Tile plan chosen by the cost model (or forced through ISAM_FORCE_TILE).
 struct GemmPlan {
     int BN;       // tile width (tile height is always 128)
+    int ka;       // 64-wide K atoms per pipeline stage
     int split;    // CTAs of one cluster sharing a tile along K (1, 2, 4 or 8)
     int stages;   // shared-memory ring depth
     int group_m;  // rasterisation group height (tiles)
