@@ -126,7 +126,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint64_t *red_full = tempty + 2;
     uint64_t *red_free = red_full + 1;
     uint64_t *cbar = red_free + 1;  // [4 epilogue warps][2] C-load barriers
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(cbar + 8);
+    uint64_t *done = cbar + 8;      // epilogue warps finished with TMEM
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -144,9 +145,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&tfull[i], 1);
             mbar_init(&tempty[i], 4);
         }
-        mbar_init(red_full, S);
+        mbar_init(red_full, kBM);
         mbar_init(red_free, S);
         for (int i = 0; i < 8; ++i) mbar_init(&cbar[i], 1);
+        mbar_init(done, 4);
         *abort_flag = 0;
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
@@ -168,6 +170,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kg_begin = static_cast<int>((static_cast<long long>(rank) * p.kg_total) / S);
     const int kg_end = static_cast<int>((static_cast<long long>(rank + 1) * p.kg_total) / S);
     const int num_tiles = p.m_tiles * p.n_tiles;
+
+    // Dependent launch: this grid may be resident while the previous kernel on
+    // the stream finishes.  Before waiting for it, pull this CTA's first
+    // stages into L2 (a prefetch only fills L2, the point of coherence, so it
+    // cannot observe stale data); every global load or store comes after.
+    griddep_launch_dependents();
+    if (threadIdx.x == 0 && cluster_id < num_tiles) {
+        int mt, nt;
+        tile_coords(cluster_id, p.m_tiles, p.n_tiles, p.group_m, mt, nt);
+        const int kg_pf = min(kg_end, kg_begin + ST);
+        for (int kg = kg_begin; kg < kg_pf; ++kg)
+            for (int at = 0; at < KA; ++at) {
+                const int k0 = (kg * KA + at) * kBK;
+                if (A_MN) {
+                    tma_prefetch_l2_2d(&tmA, mt * kBM, k0);
+                    tma_prefetch_l2_2d(&tmA, mt * kBM + 64, k0);
+                } else {
+                    tma_prefetch_l2_2d(&tmA, k0, mt * kBM);
+                }
+                if (B_MN) {
+                    for (int c = 0; c < (BN + 63) / 64; ++c) tma_prefetch_l2_2d(&tmB, nt * BN + c * 64, k0);
+                } else {
+                    tma_prefetch_l2_2d(&tmB, k0, nt * BN);
+                }
+            }
+    }
+    __syncwarp();
+    griddep_wait();
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
@@ -417,61 +447,72 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
             } else {
-                // Split-K: park this CTA's partial tile in shared memory, then
-                // every CTA of the cluster reduces its own row slice over all
-                // ranks in rank order.
+                // Split-K, push style: row slice o (128 / S rows) of the tile is
+                // reduced by cluster rank o.  Every epilogue thread stores its
+                // partial row straight into the owner's shared memory and then
+                // release-arrives on the owner's red_full (128 arrivals per
+                // tile: S sources x 128 / S rows); each owner sums the S slices
+                // it received in rank order (deterministic) and stores its rows
+                // of C.
                 if (iter > 0 &&
                     !warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE)) {
                     ok = false;
                     break;
                 }
-                float *prow = ebuf + static_cast<size_t>(row_local) * (BN + 4);
+                const int rows_per = kBM / S;
+                {
+                    const uint32_t owner = static_cast<uint32_t>(row_local / rows_per);
+                    const int rr = row_local - static_cast<int>(owner) * rows_per;
+                    const uint32_t dst = mapa_shared(
+                        smem_u32(ebuf + static_cast<size_t>(static_cast<int>(rank) * rows_per + rr) * (BN + 4)), owner);
+                    // Up to 64 columns per TMEM round trip (loads issued together).
+                    constexpr int CH = BN < 64 ? BN : 64;
 #pragma unroll 1
-                for (int c = 0; c < BN; c += C::kCW) {
-                    uint32_t r[C::kCW];
-                    if constexpr (C::kCW == 32) {
-                        tmem_ld32(tbase + c, r);
-                    } else {
-                        tmem_ld16(tbase + c, r);
-                    }
-                    tmem_ld_wait();
+                    for (int c = 0; c < BN; c += CH) {
+                        uint32_t r[CH];
+                        if constexpr (CH == 16) {
+                            uint32_t (&r0)[16] = *reinterpret_cast<uint32_t(*)[16]>(&r[0]);
+                            tmem_ld16(tbase + c, r0);
+                        } else {
 #pragma unroll
-                    for (int j = 0; j < C::kCW; j += 4)
-                        *reinterpret_cast<float4 *>(prow + c + j) =
-                            make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
-                                        __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3]));
+                            for (int h = 0; h < CH / 32; ++h) {
+                                uint32_t (&rh)[32] = *reinterpret_cast<uint32_t(*)[32]>(&r[h * 32]);
+                                tmem_ld32(tbase + c + h * 32, rh);
+                            }
+                        }
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int j = 0; j < CH; j += 4)
+                            st_dsmem_f4(dst + static_cast<uint32_t>((c + j) * 4),
+                                        make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]),
+                                                    __uint_as_float(r[j + 2]), __uint_as_float(r[j + 3])));
+                    }
+                    mbar_arrive_remote(red_full, owner);
                 }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&tempty[acc]);
                 __syncwarp();
-                named_bar(1, 128);
-                if (ew == 0 && lane == 0) {
-                    for (int r = 0; r < S; ++r) mbar_arrive_remote(red_full, static_cast<uint32_t>(r));
-                }
-                __syncwarp();
                 if (!warp_wait<true>(red_full, static_cast<uint32_t>(iter & 1), w, SITE_EPI_REDFULL)) {
                     ok = false;
                     break;
                 }
-                const int rows_per = kBM / S;
-                const int rl0 = static_cast<int>(rank) * rows_per;
                 const int g4 = BN / 4;
                 const int groups = rows_per * g4;
                 for (int g = ew * 32 + lane; g < groups; g += 128) {
-                    const int rl = rl0 + g / g4;
+                    const int rr = g / g4;
                     const int c4 = (g % g4) * 4;
-                    const int grow = mt * kBM + rl;
+                    const int grow = mt * kBM + static_cast<int>(rank) * rows_per + rr;
                     const int gcol = col0 + c4;
                     if (grow >= p.M) continue;
                     float *crow = p.C + static_cast<size_t>(grow) * p.N;
-                    float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
                     const bool vec = p.n_vec4 && gcol + 3 < p.N;
+                    float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
                     if (p.beta != 0.0f && vec) cin = *reinterpret_cast<const float4 *>(crow + gcol);
-                    const uint32_t local = smem_u32(ebuf + static_cast<size_t>(rl) * (BN + 4) + c4);
                     float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
                     for (int r = 0; r < S; ++r) {
-                        const float4 v = ld_dsmem_f4(mapa_shared(local, static_cast<uint32_t>(r)));
+                        const float4 v = *reinterpret_cast<const float4 *>(
+                            ebuf + static_cast<size_t>(r * rows_per + rr) * (BN + 4) + c4);
                         s.x += v.x;
                         s.y += v.y;
                         s.z += v.z;
@@ -498,12 +539,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
-                __syncwarp();
-                named_bar(1, 128);
-                if (ew == 0 && lane == 0) {
-                    for (int r = 0; r < S; ++r) mbar_arrive_remote(red_free, static_cast<uint32_t>(r));
+                // Release the slot to every pusher, unless nobody pushes again
+                // (after the cluster's last tile no remote arrive may target an
+                // exited CTA).
+                if (tile + num_clusters < num_tiles) {
+                    __syncwarp();
+                    named_bar(1, 128);
+                    if (ew == 0 && lane == 0) {
+                        for (int r = 0; r < S; ++r) mbar_arrive_remote(red_free, static_cast<uint32_t>(r));
+                    }
+                    __syncwarp();
                 }
-                __syncwarp();
             }
             if (S == 1) {
                 tc_fence_before();
@@ -516,21 +562,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                 acc_phase ^= 1u;
             }
         }
-        // Split-K: no peer may still be reading this CTA's partial tile when it exits.
-        if (S > 1 && ok && iter > 0)
-            warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE);
         // TMA path: C loads still in flight land, stores complete, before exit.
         if (use_tma) {
             for (int b = 0; b < 2; ++b)
                 if (cpend[b] && lane == 0) drain_wait(&cb[b], cpar[b], p.timeout_ns);
             if (lane == 0) bulk_wait_all<0>();
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(done);
         __syncwarp();
     }
 
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
+        // TMEM is released only after every epilogue warp has stopped reading it.
+        bounded_wait(done, 0, w, SITE_EPI_TFULL);
+        __syncwarp();
         tc_fence_after();
         tmem_dealloc(tmem_base, C::kTmemCols);
     }
@@ -560,7 +609,7 @@ int b_bytes(int BN, bool b_mn) { return b_mn ? ((BN + 63) / 64) * 8192 : BN * 12
 
 size_t smem_bytes(int BN, bool b_mn, int split, int stages, int ka) {
     return 1024 + static_cast<size_t>(stages) * ka * (kABytes + b_bytes(BN, b_mn)) +
-           epi_bytes(BN, split) + (2 * stages + 14) * 8 + 16;
+           epi_bytes(BN, split) + (2 * stages + 15) * 8 + 16;
 }
 
 int max_stages(int BN, bool b_mn, int split, int ka, int smem_limit) {
@@ -571,14 +620,20 @@ int max_stages(int BN, bool b_mn, int split, int ka, int smem_limit) {
 
 int ceil_div(long long a, long long b) { return static_cast<int>((a + b - 1) / b); }
 
-// Rough machine constants for the cost model (GB300: measured dense bf16 and
-// copy bandwidth; per-SM shared-memory bandwidth 128 B/clk).
+// Machine constants of the cost model, calibrated on GB300 with the
+// kernel's own timeline (globaltimer stamps per CTA): ~2.3 us from launch to
+// the first TMA data; TMA operand streaming saturates at ~47 GB/s per SM from
+// four stages in flight (a per-SM cap, so bandwidth comes from using many
+// SMs); ~1.3 us between launches; measured dense bf16 and copy peaks.
 constexpr double kPeakFlops = 1.9e15;
 constexpr double kHbmBw = 6.7e12;
-constexpr double kSmL2Bw = 110e9;   // sustainable L2 -> SM bytes/s per SM
+constexpr double kSmStreamBw = 47e9;   // operand bytes/s one SM sustains
+constexpr double kSmStoreBw = 30e9;    // epilogue bytes/s one SM sustains
 constexpr double kClock = 1.9e9;
-constexpr double kTileOverheadUs = 0.35;
-constexpr double kLaunchUs = 2.5;
+constexpr double kFirstDataUs = 2.3;
+constexpr double kLaunchGapUs = 1.3;
+constexpr double kTileOverheadUs = 0.3;
+constexpr double kSplitTailUs = 1.5;   // push + owner reduce of a split tile
 
 double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out) {
     const int m_tiles = ceil_div(g.M, kBM);
@@ -595,17 +650,15 @@ double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out)
     const double cyc_k16 = std::max(BN / 2.0, (kBM * 32.0 + BN * 32.0) / 128.0);
     const double t_mma = kb_per * 4 * cyc_k16 / kClock * 1e6;
     const double bytes_unit = static_cast<double>(kBM + BN) * kb_per * kBK * 2.0;
-    const double active = std::min<double>(static_cast<double>(tiles) * S, num_sms);
-    const double sm_bw = std::min(kSmL2Bw, kHbmBw / active);
-    const double t_load = bytes_unit / sm_bw * 1e6;
-    const double t_unit = std::max(t_mma, t_load) + kTileOverheadUs +
-                          (S > 1 ? 0.5 + 128.0 * BN * 4.0 * (S - 1) / S / 60e9 * 1e6 : 0.0);
+    const double t_load = bytes_unit / kSmStreamBw * 1e6;
+    const double t_unit = std::max(t_mma, t_load) + kTileOverheadUs;
     const double t_steady = tiles_per_cluster * t_unit;
-    const double uniq = 2.0 * g.M * g.K + 2.0 * g.K * g.N +
-                        4.0 * g.M * g.N * (g.beta != 0.0f ? 2.0 : 1.0);
+    const double out_bytes = 4.0 * g.M * g.N * (g.beta != 0.0f ? 2.0 : 1.0);
+    const double uniq = 2.0 * g.M * g.K + 2.0 * g.K * g.N + out_bytes;
     const double t_hbm = uniq / kHbmBw * 1e6;
     const double t_flops = 2.0 * g.M * g.N * g.K / kPeakFlops * 1e6;
-    return std::max({t_steady, t_hbm, t_flops}) + kLaunchUs;
+    const double tail = (S > 1 ? kSplitTailUs : 0.0) + kBM * BN * 4.0 / S / kSmStoreBw * 1e6;
+    return kFirstDataUs + std::max({t_steady, t_hbm, t_flops}) + tail + kLaunchGapUs;
 }
 
 struct AttrCache {
@@ -758,19 +811,21 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
     if ((rc = ensure_smem_attr(fn, plan.smem))) return rc;
 
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     cfg.gridDim = dim3(static_cast<unsigned>(plan.grid), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = plan.smem;
     cfg.stream = stream;
-    cfg.numAttrs = 0;
     cfg.attrs = attr;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 1;
     if (plan.split > 1) {
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = static_cast<unsigned>(plan.split);
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.numAttrs = 1;
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = static_cast<unsigned>(plan.split);
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
     }
     cudaError_t e = cudaLaunchKernelEx(&cfg, fn, ta, tb, tc, p);
     if (e != cudaSuccess) return cuda_error(e, "launch gemm_tc_kernel");
