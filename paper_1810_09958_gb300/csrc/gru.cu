@@ -9,13 +9,21 @@
 //
 //   1. gx = x W^T + b_ih for all T steps is one GEMM (isam_gemm's kernel, bias
 //      fused in its epilogue), written to a library workspace;
-//   2. one cooperative persistent kernel runs the recurrence.  CTA c owns
-//      hidden units [16c, 16c+16): its 48 rows of U (gates r, z, n) stay in
-//      shared memory for all T steps.  Per step it TMA-loads bf16(h_{t-1})
-//      (all batch rows), multiplies U_slice * h^T on the tensor cores into
-//      TMEM, evaluates the gates in fp32 with h carried in fp32 registers,
-//      writes h_t to h_out and bf16(h_t) to an exchange buffer, and signals a
-//      grid-wide step counter.  Every wait is bounded in time.
+//   2. one persistent kernel runs the recurrence.  Hidden units are taken in
+//      groups of 32; a group is a cluster of KS CTAs (KS = 4 at hidden 1024)
+//      that split the reduction dimension of U h: CTA r keeps the 96 rows of U
+//      for the group's r, z and n gates over its K quarter resident in shared
+//      memory for all T steps.  Per step each CTA TMA-loads its quarter of
+//      bf16(h_{t-1}) (all batch rows), runs 16 tcgen05.mma (M = 128 with 96
+//      rows used, N = 32 batch) into TMEM, and pushes the partial rows of the
+//      units owned by each cluster peer straight into that peer's shared
+//      memory; the owner sums the KS partials in rank order, evaluates the
+//      gates in fp32 (h carried in fp32 registers), publishes bf16(h_t) to an
+//      exchange buffer, signals a grid-wide step counter, then writes h_t to
+//      h_out.  Splitting K keeps the per-step tensor instruction count per CTA
+//      low: at this size each M = 128 instruction costs about the same
+//      whatever its N, so the step time is set by instructions per CTA.
+//      Every wait is bounded in time.
 #include <cstdio>
 #include <cstdlib>
 #include <mutex>
@@ -29,26 +37,31 @@ namespace isam {
 
 namespace {
 
-constexpr int kUnits = 16;           // hidden units per CTA
-constexpr int kRows = 3 * kUnits;    // U rows per CTA (r, z, n)
-constexpr int kBatchPad = 32;        // MMA N (batch rows, padded)
+constexpr int kGroup = 32;               // hidden units per group (one cluster)
+constexpr int kRowsG = 3 * kGroup;       // 96 U rows per group (r, z, n)
+constexpr int kBatchPad = 32;            // MMA N (batch rows, padded)
 constexpr int kThreads = 128;
-constexpr int kAtomU = kRows * 128;  // bytes of one 64-wide K atom of the U slice (6 KB)
-constexpr int kAtomH = kBatchPad * 128;  // bytes of one K atom of h (4 KB)
-constexpr int kQuarters = 4;             // at most this many h pieces per step
-constexpr int kGhBytes = 6400;           // 48 x 33 fp32, rounded up to 64 bytes
+constexpr int kAtomU = kRowsG * 128;     // one 64-wide K atom of the U slice (12 KB)
+constexpr int kAtomH = kBatchPad * 128;  // one K atom of h (4 KB)
+constexpr int kUPad = 32 * 128;          // the M = 128 MMA reads 32 rows past an atom
+constexpr int kRecvBytes = kRowsG * kBatchPad * 4;  // partial rows received per step (12 KB)
+constexpr int kMaxPieces = 4;
 
 enum : uint32_t {
     SITE_GRU_STEP = 0x201,
     SITE_GRU_U = 0x202,
     SITE_GRU_H = 0x203,
     SITE_GRU_MMA = 0x204,
+    SITE_GRU_RED = 0x205,
 };
 
 struct GruParams {
-    int T, batch, H, nk;       // nk = H / 64 K atoms
-    int nq, qk;                // h is loaded in nq pieces of qk atoms (nq * qk == nk)
-    int n_cta;
+    int T, batch, H;
+    int ks;                    // K splits per unit group = cluster size
+    int ka;                    // 64-wide K atoms per CTA (H / ks / 64)
+    int uo;                    // units whose gates one CTA evaluates (32 / ks)
+    int n_cta;                 // (H / 32) * ks
+    int nq, qk;                // h arrives in nq pieces of qk atoms (nq * qk == ka)
     const float *gx;           // [T*batch][3H], includes b_ih
     const float *b_hh;         // [3H]
     const float *h0;           // [batch][H] or null
@@ -92,6 +105,22 @@ __device__ bool wait_counter(const uint32_t *counter, uint32_t target, const Wai
     }
 }
 
+struct GruLayout {
+    int off_u, off_h, off_recv, off_bars, total;
+};
+
+__host__ __device__ inline GruLayout gru_layout(int ka) {
+    GruLayout L;
+    L.off_u = 0;
+    L.off_h = ka * kAtomU + kUPad;
+    L.off_recv = L.off_h + ka * kAtomH;
+    L.off_bars = L.off_recv + kRecvBytes;
+    L.total = L.off_bars + 128 + 1024;
+    return L;
+}
+
+constexpr int kMaxPairs = 8;  // (unit, batch) pairs per thread when one CTA owns all 32 units
+
 __global__ void __launch_bounds__(kThreads, 1)
     gru_recurrent_kernel(const __grid_constant__ CUtensorMap tmU,
                          const __grid_constant__ CUtensorMap tmH0,
@@ -99,33 +128,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
-    // U slice: nk atoms of 48 rows x 128 B; the M = 128 MMA reads 80 rows past
-    // each atom, so the region is padded to keep the last atom's read inside.
-    const int u_bytes = p.nk * kAtomU + 10240;
-    uint8_t *sU = smem;
-    uint8_t *sH = smem + u_bytes;                        // nk atoms of 32 rows x 128 B
-    float *gh = reinterpret_cast<float *>(sH + p.nk * kAtomH);  // [48][33] fp32
-    uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(gh) + kGhBytes);
-    uint64_t *ubar = bars;                 // U slice landed
-    uint64_t *hbar = bars + 1;             // [kQuarters] h quarter landed
-    uint64_t *mma_done = hbar + kQuarters; // MMAs of the step complete
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mma_done + 1);
+    const GruLayout L = gru_layout(p.ka);
+    uint8_t *sU = smem + L.off_u;
+    uint8_t *sH = smem + L.off_h;
+    float *recv = reinterpret_cast<float *>(smem + L.off_recv);  // [ks src][3 gates][uo][32 batch]
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L.off_bars);
+    uint64_t *ubar = bars;                  // U slice landed
+    uint64_t *hbar = bars + 1;              // [kMaxPieces] h piece landed
+    uint64_t *mma_done = hbar + kMaxPieces; // MMAs of the step complete
+    uint64_t *red_full = mma_done + 1;      // all partial rows of my units arrived
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(red_full + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
-    const int j0 = blockIdx.x * kUnits;
     const int H = p.H;
     const int G = 3 * H;
+    const int KS = p.ks;
+    const int UO = p.uo;
+    const int group = blockIdx.x / KS;
+    const uint32_t rank = KS > 1 ? cluster_ctarank() : 0u;
+    const int unit0 = group * kGroup;
+    const int atom0 = static_cast<int>(rank) * p.ka;
     const WaitCtx w{p.timeout_ns, p.err, abort_flag};
-    const int qk = p.qk;
-    const int nq = p.nq;
 
     if (tid == 0) {
         mbar_init(ubar, 1);
-        for (int q = 0; q < kQuarters; ++q) mbar_init(&hbar[q], 1);
+        for (int q = 0; q < kMaxPieces; ++q) mbar_init(&hbar[q], 1);
         mbar_init(mma_done, 1);
+        mbar_init(red_full, kRowsG);
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -136,26 +168,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc_fence_before();
     __syncthreads();
+    if (KS > 1) cluster_sync_all();  // peers' barriers exist before any remote arrive
     tc_fence_after();
     const uint32_t tmem_d = *tmem_slot;
 
     // ---- priming iteration: persistent weights and initial state.
     if (tid == 0) {
         tma_prefetch_desc(&tmU);
-        mbar_arrive_expect_tx(ubar, static_cast<uint32_t>(p.nk * kAtomU));
-        for (int ka = 0; ka < p.nk; ++ka) tma_load_3d(&tmU, ubar, sU + ka * kAtomU, ka * 64, j0, 0);
+        tma_prefetch_desc(&tmH0);
+        tma_prefetch_desc(&tmH1);
+        mbar_arrive_expect_tx(ubar, static_cast<uint32_t>(p.ka * kAtomU));
+        for (int a = 0; a < p.ka; ++a)
+            tma_load_3d(&tmU, ubar, sU + a * kAtomU, (atom0 + a) * 64, unit0, 0);
     }
-    // Each thread owns one unit u and batch rows bb, bb + 8, bb + 16, bb + 24.
-    const int u = tid & 15;
-    const int bb = tid >> 4;
-    const int j = j0 + u;
+    __syncwarp();
+    // This CTA evaluates the gates of units unit0 + rank*UO + [0, UO); thread
+    // tid takes unit ui = tid % UO and batch rows b = tid / UO + k * (128 / UO).
+    const int ui = tid % UO;
+    const int bstep = kThreads / UO;
+    const int np = UO * kBatchPad / kThreads;
+    const int j = unit0 + static_cast<int>(rank) * UO + ui;
     const float bh_r = p.b_hh[j], bh_z = p.b_hh[H + j], bh_n = p.b_hh[2 * H + j];
-    float hprev[4];
+    float hprev[kMaxPairs];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int b = bb + 8 * k;
-        hprev[k] = (p.h0 != nullptr && b < p.batch) ? p.h0[static_cast<size_t>(b) * H + j] : 0.0f;
-        if (b < p.batch) p.hx[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hprev[k]);
+    for (int k = 0; k < kMaxPairs; ++k) {
+        const int b = tid / UO + k * bstep;
+        hprev[k] = (k < np && p.h0 != nullptr && b < p.batch) ? p.h0[static_cast<size_t>(b) * H + j] : 0.0f;
+        if (k < np && b < p.batch) p.hx[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hprev[k]);
     }
     fence_proxy_async_global();
     __syncwarp();
@@ -175,20 +214,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (wait_counter(p.counter, static_cast<uint32_t>((t + 1) * p.n_cta), w)) {
                 fence_proxy_async_global();
                 const CUtensorMap *m = (t & 1) ? &tmH1 : &tmH0;
-                for (int q = 0; q < nq; ++q) {
-                    mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(qk * kAtomH));
-                    tma_load_3d(m, &hbar[q], sH + q * qk * kAtomH, 0, 0, q * qk);
+                for (int q = 0; q < p.nq; ++q) {
+                    mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(p.qk * kAtomH));
+                    tma_load_3d(m, &hbar[q], sH + q * p.qk * kAtomH, 0, 0, atom0 + q * p.qk);
                 }
                 issued_phase = t;
             }
         }
         __syncwarp();
         // Input projection of this step (independent of h): prefetch.
-        float gxr[4], gxz[4], gxn[4];
+        float gxr[kMaxPairs], gxz[kMaxPairs], gxn[kMaxPairs];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int b = bb + 8 * k;
-            if (b < p.batch) {
+        for (int k = 0; k < kMaxPairs; ++k) {
+            const int b = tid / UO + k * bstep;
+            if (k < np && b < p.batch) {
                 const float *g = p.gx + (static_cast<size_t>(t) * p.batch + b) * G + j;
                 gxr[k] = g[0];
                 gxz[k] = g[H];
@@ -198,13 +237,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         if (tid == 32 && ok) {
-            for (int q = 0; q < nq && ok; ++q) {
+            for (int q = 0; q < p.nq && ok; ++q) {
                 if (!bounded_wait(&hbar[q], par, w, SITE_GRU_H)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                for (int a = q * qk; a < (q + 1) * qk; ++a) {
+                for (int a = q * p.qk; a < (q + 1) * p.qk; ++a) {
                     const uint32_t ua = smem_u32(sU + a * kAtomU);
                     const uint32_t ha = smem_u32(sH + a * kAtomH);
 #pragma unroll
@@ -220,45 +259,63 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Block-uniform decision: every thread leaves the loop at the same step.
         if (!__syncthreads_and(bounded_wait(mma_done, par, w, SITE_GRU_MMA) ? 1 : 0)) break;
         tc_fence_after();
-        if (warp < 2) {
+        // Push: row gate*32 + u of the partial product (TMEM lane = row) goes to
+        // the cluster CTA that owns unit u, into its slot for this source rank.
+        if (warp < 3) {
             uint32_t r[32];
             tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
             tmem_ld_wait();
-            const int row = warp * 32 + lane;
-            if (row < kRows) {
+            const uint32_t owner = static_cast<uint32_t>(lane / UO);
+            const int oui = lane % UO;
+            const uint32_t dst = mapa_shared(
+                smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kBatchPad), owner);
 #pragma unroll
-                for (int c = 0; c < 32; ++c) gh[row * 33 + c] = __uint_as_float(r[c]);
-            }
+            for (int c = 0; c < 8; ++c)
+                st_dsmem_f4(dst + c * 16, make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
+                                                      __uint_as_float(r[4 * c + 2]),
+                                                      __uint_as_float(r[4 * c + 3])));
+            mbar_arrive_remote(red_full, owner);
         }
         tc_fence_before();
-        __syncthreads();
+        __syncwarp();
+        if (!__syncthreads_and(bounded_wait<true>(red_full, par, w, SITE_GRU_RED) ? 1 : 0)) break;
         uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int b = bb + 8 * k;
-            if (b >= p.batch) continue;
-            const float ghr = gh[u * 33 + b] + bh_r;
-            const float ghz = gh[(kUnits + u) * 33 + b] + bh_z;
-            const float ghn = gh[(2 * kUnits + u) * 33 + b] + bh_n;
+        for (int k = 0; k < kMaxPairs; ++k) {
+            const int b = tid / UO + k * bstep;
+            if (k >= np || b >= p.batch) continue;
+            float ghr = bh_r, ghz = bh_z, ghn = bh_n;
+            for (int s = 0; s < KS; ++s) {
+                const float *rs = recv + (s * 3 * UO + ui) * kBatchPad + b;
+                ghr += rs[0];
+                ghz += rs[UO * kBatchPad];
+                ghn += rs[2 * UO * kBatchPad];
+            }
             const float rg = sigmoidf_fast(gxr[k] + ghr);
             const float zg = sigmoidf_fast(gxz[k] + ghz);
             const float ng = tanhf(gxn[k] + rg * ghn);
             const float hn = (1.0f - zg) * ng + zg * hprev[k];
             hprev[k] = hn;
-            p.h_out[(static_cast<size_t>(t) * p.batch + b) * H + j] = hn;
             hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
         }
+        // Publish first (the release then waits only for the exchange-buffer
+        // stores), then write this step's h_t to h_out.
         fence_proxy_async_global();
         __syncthreads();
         if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
             red_release_gpu_add(p.counter, 1u);
         __syncwarp();
+#pragma unroll
+        for (int k = 0; k < kMaxPairs; ++k) {
+            const int b = tid / UO + k * bstep;
+            if (k < np && b < p.batch) p.h_out[(static_cast<size_t>(t) * p.batch + b) * H + j] = hprev[k];
+        }
         tc_fence_after();
     }
 
     // ---- teardown: let issued copies land, release TMEM.
     if (tid == 0 && issued_phase >= 0 && *abort_flag) {
-        for (int q = 0; q < nq; ++q) {
+        for (int q = 0; q < p.nq; ++q) {
             const uint32_t a = smem_u32(&hbar[q]);
             const unsigned long long t0 = globaltimer();
             while (!mbar_try_wait(a, static_cast<uint32_t>(issued_phase & 1)))
@@ -274,11 +331,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-size_t gru_smem_bytes(int H) {
-    const int nk = H / 64;
-    return 1024 + static_cast<size_t>(nk) * kAtomU + 10240 + static_cast<size_t>(nk) * kAtomH +
-           kGhBytes + 8 * (2 + kQuarters) + 16 + 16;
-}
+// K splits for a hidden size: each CTA's K range must be whole 64-wide atoms.
+int gru_splits(int H) { return (H % 256 == 0) ? 4 : (H % 128 == 0) ? 2 : 1; }
+
+size_t gru_smem_bytes(int H) { return static_cast<size_t>(gru_layout(H / gru_splits(H) / 64).total); }
+
+int gru_cta_count(int H) { return H / kGroup * gru_splits(H); }
 
 int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
     if (*cap >= need) return ISAM_OK;
@@ -288,6 +346,74 @@ int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
     cudaError_t e = cudaMalloc(ptr, need);
     if (e != cudaSuccess) return cuda_error(e, what);
     *cap = need;
+    return ISAM_OK;
+}
+
+// Tensor maps of the recurrence: U as [3 gates][H rows][H] (box: 96 rows of
+// one group over one 64-wide K atom) and the two exchange buffers as
+// [H/64 atoms][32 batch rows][64] (box: one CTA's h piece).
+int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tmU, CUtensorMap *tmH0,
+                   CUtensorMap *tmH1) {
+    int rc;
+    const int ka = H / gru_splits(H) / 64;
+    const int nq = (ka % 4 == 0) ? 4 : (ka % 3 == 0) ? 3 : (ka % 2 == 0) ? 2 : 1;
+    {
+        const uint64_t dims[3] = {static_cast<uint64_t>(H), static_cast<uint64_t>(H), 3};
+        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, static_cast<uint64_t>(H) * H * 2};
+        const uint32_t box[3] = {64, kGroup, 3};
+        if ((rc = make_tmap_3d_bf16(tmU, U, dims, strides, box))) return rc;
+    }
+    for (int i = 0; i < 2; ++i) {
+        const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(H / 64)};
+        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
+        const uint32_t box[3] = {64, kBatchPad, static_cast<uint32_t>(ka / nq)};
+        if ((rc = make_tmap_3d_bf16(i ? tmH1 : tmH0, hx + static_cast<size_t>(i) * kBatchPad * H, dims,
+                                    strides, box)))
+            return rc;
+    }
+    return ISAM_OK;
+}
+
+// Fills the shape fields of p and launches the recurrence: one cluster of KS
+// CTAs per group of 32 units; cooperative (guaranteed co-residency) when the
+// driver accepts it with clusters, otherwise after checking that every
+// cluster fits at once (the step counter needs every CTA resident).
+int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tmH0,
+                     const CUtensorMap &tmH1, size_t smem, cudaStream_t stream) {
+    const int H = p.H;
+    p.ks = gru_splits(H);
+    p.ka = H / p.ks / 64;
+    p.uo = kGroup / p.ks;
+    p.n_cta = gru_cta_count(H);
+    p.nq = (p.ka % 4 == 0) ? 4 : (p.ka % 3 == 0) ? 3 : (p.ka % 2 == 0) ? 2 : 1;
+    p.qk = p.ka / p.nq;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(p.ks);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeCooperative;
+    attr[1].val.cooperative = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(p.n_cta), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
+    if (e == cudaSuccess) return ISAM_OK;
+    (void)cudaGetLastError();
+    cfg.numAttrs = 1;
+    int max_clusters = 0;
+    e = cudaOccupancyMaxActiveClusters(&max_clusters, gru_recurrent_kernel, &cfg);
+    if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveClusters(gru)");
+    if (max_clusters * p.ks < p.n_cta)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "GRU recurrence: %d CTAs in clusters of %d cannot be co-resident (%d clusters fit)",
+                         p.n_cta, p.ks, max_clusters);
+    e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
+    if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel");
     return ISAM_OK;
 }
 
@@ -306,7 +432,7 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
          reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |
          reinterpret_cast<uintptr_t>(h0) | reinterpret_cast<uintptr_t>(h_out)) & 15u)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: pointers must be 16-byte aligned");
-    const int n_cta = H / kUnits;
+    const int n_cta = gru_cta_count(H);
     if (n_cta > ds.num_sms)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: %d CTAs cannot be co-resident", n_cta);
     const size_t smem = gru_smem_bytes(H);
@@ -340,30 +466,11 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
 
     // 2. Recurrence.
     CUtensorMap tmU, tmH0, tmH1;
-    {
-        const uint64_t dims[3] = {static_cast<uint64_t>(H), static_cast<uint64_t>(H), 3};
-        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, static_cast<uint64_t>(H) * H * 2};
-        const uint32_t box[3] = {64, kUnits, 3};
-        if ((rc = make_tmap_3d_bf16(&tmU, U, dims, strides, box))) return rc;
-    }
-    const int nk = H / 64;
-    const int nq = (nk % 4 == 0) ? 4 : (nk % 2 == 0) ? 2 : 1;
-    for (int i = 0; i < 2; ++i) {
-        const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(nk)};
-        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
-        const uint32_t box[3] = {64, kBatchPad, static_cast<uint32_t>(nk / nq)};
-        if ((rc = make_tmap_3d_bf16(i ? &tmH1 : &tmH0, ds.gru_hx + static_cast<size_t>(i) * kBatchPad * H,
-                                    dims, strides, box)))
-            return rc;
-    }
+    if ((rc = recurrent_maps(U, ds.gru_hx, H, &tmU, &tmH0, &tmH1))) return rc;
     GruParams p{};
     p.T = T;
     p.batch = batch;
     p.H = H;
-    p.nk = nk;
-    p.nq = nq;
-    p.qk = nk / nq;
-    p.n_cta = n_cta;
     p.gx = ds.gru_gx;
     p.b_hh = b + 3 * H;
     p.h0 = h0;
@@ -384,19 +491,7 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
         if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
         attr_set = true;
     }
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
-    cfg.gridDim = dim3(static_cast<unsigned>(n_cta), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
-    if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel");
-    return ISAM_OK;
+    return launch_recurrent(p, tmU, tmH0, tmH1, smem, stream);
 }
 
 }  // namespace isam
@@ -519,7 +614,7 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
             g_noalloc_attr = true;
         }
     }
-    const int n_cta = H / kUnits;
+    const int n_cta = gru_cta_count(H);
     const size_t smem = gru_smem_bytes(H);
     if (n_cta > nd.num_sms || smem > static_cast<size_t>(nd.smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward_noalloc: hidden too large");
@@ -541,22 +636,7 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
     if ((e = cudaMemsetAsync(err, 0, 16, stream)) != cudaSuccess)
         return cuda_error(e, "clearing the scratch error word");
     CUtensorMap tmU, tmH0, tmH1;
-    {
-        const uint64_t dims[3] = {static_cast<uint64_t>(H), static_cast<uint64_t>(H), 3};
-        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, static_cast<uint64_t>(H) * H * 2};
-        const uint32_t box[3] = {64, kUnits, 3};
-        if ((rc = make_tmap_3d_bf16(&tmU, U, dims, strides, box))) return rc;
-    }
-    const int nk = H / 64;
-    const int nq = (nk % 4 == 0) ? 4 : (nk % 2 == 0) ? 2 : 1;
-    for (int i = 0; i < 2; ++i) {
-        const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(nk)};
-        const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
-        const uint32_t box[3] = {64, kBatchPad, static_cast<uint32_t>(nk / nq)};
-        if ((rc = make_tmap_3d_bf16(i ? &tmH1 : &tmH0, hx + static_cast<size_t>(i) * kBatchPad * H,
-                                    dims, strides, box)))
-            return rc;
-    }
+    if ((rc = recurrent_maps(U, hx, H, &tmU, &tmH0, &tmH1))) return rc;
     const size_t step_elems = static_cast<size_t>(batch) * H;
     for (long long t0 = 0; t0 < T; t0 += chunk) {
         const int tc = static_cast<int>(T - t0 < chunk ? T - t0 : chunk);
@@ -574,10 +654,6 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         p.T = tc;
         p.batch = batch;
         p.H = H;
-        p.nk = nk;
-        p.nq = nq;
-        p.qk = nk / nq;
-        p.n_cta = n_cta;
         p.gx = gx;
         p.b_hh = b + 3 * H;
         p.h0 = t0 == 0 ? h0 : h_out + static_cast<size_t>(t0 - 1) * step_elems;
@@ -587,18 +663,7 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         p.skip_publish_cta = -1;
         p.timeout_ns = wait_timeout_ns();
         p.err = err;
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeCooperative;
-        attr[0].val.cooperative = 1;
-        cfg.gridDim = dim3(static_cast<unsigned>(n_cta), 1, 1);
-        cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = smem;
-        cfg.stream = stream;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
-        if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel (noalloc)");
+        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, smem, stream))) return rc;
     }
     // Report device-side timeouts of this call before returning.
     if ((e = cudaStreamSynchronize(stream)) != cudaSuccess)
