@@ -47,7 +47,8 @@ int get_encoder() {
 
 int encode(CUtensorMap *out, const uint64_t key[12], cuuint32_t rank, const void *base,
            const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box,
-           CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
+           CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+           CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
     {
         std::lock_guard<std::mutex> lk(g_tmap_mu);
         for (int i = 0; i < kTmapCache; ++i)
@@ -61,7 +62,7 @@ int encode(CUtensorMap *out, const uint64_t key[12], cuuint32_t rank, const void
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = g_encode(out, dtype, rank, const_cast<void *>(base), dims,
                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS)
         return set_error(ISAM_ERR_UNSUPPORTED, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
@@ -164,6 +165,17 @@ int make_tmap_2d_f32(CUtensorMap *out, const void *base, uint64_t inner, uint64_
     cuuint64_t strides[1] = {row_pitch_bytes};
     cuuint32_t box[2] = {box_inner, box_outer};
     return encode(out, key, 2, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+}
+
+int make_tmap_3d_bf16_plain(CUtensorMap *out, const void *base, const uint64_t dims_in[3],
+                            const uint64_t strides_bytes[2], const uint32_t box_in[3]) {
+    const uint64_t key[12] = {0x3A, reinterpret_cast<uint64_t>(base), dims_in[0], dims_in[1], dims_in[2],
+                              strides_bytes[0], strides_bytes[1], box_in[0], box_in[1], box_in[2], 0, 0};
+    cuuint64_t dims[3] = {dims_in[0], dims_in[1], dims_in[2]};
+    cuuint64_t strides[2] = {strides_bytes[0], strides_bytes[1]};
+    cuuint32_t box[3] = {box_in[0], box_in[1], box_in[2]};
+    return encode(out, key, 3, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                  CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
 int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims_in[3],

@@ -328,6 +328,343 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// ---------------------------------------------------------------- row-ring variant
+// For images no wider than 128 pixels: a tile is rt = 128 / W whole image
+// rows, each CTA walks a contiguous range of tiles, and the input rows live in
+// a shared-memory ring filled by one TMA copy per row.  Every input element
+// then leaves L2 about once per CTA, and the producers read the 3x3 taps from
+// shared memory.
+constexpr int kRingMax = 32;  // input rows resident per CTA: 2 * rt + 2 (this tile + halo + the next)
+
+enum : uint32_t { SITE_DW_RING = 0x306 };
+
+struct DwRowParams {
+    int N, H, W, Cin, Cout;
+    int rt;              // image rows per tile (rt * W <= 128)
+    int tiles_per_img;   // ceil(H / rt)
+    int tiles;           // N * tiles_per_img
+    int kb, nchunks;
+    int row_bytes;       // one input row in shared memory (W * Cin * 2, rounded to 128)
+    int ring;            // input rows resident per CTA (2 * rt + 2 <= kRingMax)
+    const uint16_t *dw;
+    float *out;
+    unsigned long long timeout_ns;
+    uint32_t *err;
+};
+
+struct DwRowLayout {
+    int off_ring, off_a, off_w, off_stage, off_dwf, off_bars, total;
+};
+
+__host__ __device__ inline DwRowLayout dw_row_layout(int W, int Cin, int Cout, int ring) {
+    DwRowLayout L;
+    const int row_bytes = (W * Cin * 2 + 127) / 128 * 128;
+    const int atoms = (Cin + 63) / 64;
+    const int nchunks = (Cout + 63) / 64;
+    L.off_ring = 0;
+    L.off_a = (ring * row_bytes + 1023) / 1024 * 1024;
+    L.off_w = L.off_a + atoms * kBM * 128;
+    L.off_stage = L.off_w + atoms * nchunks * 8192;
+    L.off_dwf = L.off_stage + 4 * 2 * 4096;
+    L.off_bars = L.off_dwf + ((9 * Cin * 4) + 1023) / 1024 * 1024;
+    L.total = L.off_bars + 8 * (kRingMax + 8) + 16 + 1024;
+    return L;
+}
+
+// First and last global input row (n * H + y) a tile reads.
+__device__ __forceinline__ void tile_rows(const DwRowParams &p, int tile, int &n, int &y0, int &y1, int &lo,
+                                          int &hi) {
+    n = tile / p.tiles_per_img;
+    y0 = (tile - n * p.tiles_per_img) * p.rt;
+    y1 = min(p.H, y0 + p.rt) - 1;
+    lo = n * p.H + max(0, y0 - 1);
+    hi = n * p.H + min(p.H - 1, y1 + 1);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    dwsep_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                      const __grid_constant__ CUtensorMap tmOut, const DwRowParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    const DwRowLayout L = dw_row_layout(p.W, p.Cin, p.Cout, p.ring);
+    const int kRing = p.ring;
+    uint8_t *ring = smem + L.off_ring;
+    uint8_t *sA = smem + L.off_a;
+    uint8_t *sW = smem + L.off_w;
+    uint8_t *sStage = smem + L.off_stage;
+    float *dwf = reinterpret_cast<float *>(smem + L.off_dwf);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L.off_bars);
+    uint64_t *ring_full = bars;           // [ring]
+    uint64_t *a_full = ring_full + kRing;
+    uint64_t *a_empty = a_full + 1;
+    uint64_t *tfull = a_empty + 1;        // [2]
+    uint64_t *tempty = tfull + 2;         // [2]
+    uint64_t *wbar = tempty + 2;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(wbar + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5;
+    const int lane = tid & 31;
+    const int Cin = p.Cin, Cout = p.Cout, W = p.W, H = p.H;
+    const int ncols = Cout <= 64 ? 64 : (Cout <= 128 ? 128 : 256);
+    const uint32_t tmem_cols = 2u * static_cast<uint32_t>(ncols);
+    // This CTA's contiguous tile range.
+    const int tb = static_cast<int>((static_cast<long long>(blockIdx.x) * p.tiles) / gridDim.x);
+    const int te = static_cast<int>((static_cast<long long>(blockIdx.x + 1) * p.tiles) / gridDim.x);
+
+    if (tid == 0) {
+        for (int i = 0; i < kRing; ++i) mbar_init(&ring_full[i], 1);
+        mbar_init(a_full, kProd);
+        mbar_init(a_empty, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        mbar_init(wbar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    for (int i = tid; i < 9 * Cin; i += kThreads)
+        dwf[i] = __uint_as_float(static_cast<uint32_t>(p.dw[i]) << 16);
+    __syncwarp();
+    if (warp == kMmaWarp) {
+        tmem_alloc(tmem_slot, tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const WaitCtx w{p.timeout_ns, p.err, abort_flag};
+
+    if (warp < kProdWarps) {
+        // ------------------------------------------------ depthwise producers
+        const int groups = Cin / 8;  // divides kProd (Cin is 16, 32, ..., 256)
+        const uint32_t row_tx = static_cast<uint32_t>(W * Cin * 2);
+        const int g = tid % groups;
+        const int pi0 = tid / groups;
+        const int pstep = kProd / groups;
+        float wreg[9][8];
+#pragma unroll
+        for (int t = 0; t < 9; ++t)
+#pragma unroll
+            for (int i = 0; i < 8; ++i) wreg[t][i] = dwf[t * Cin + g * 8 + i];
+        int first_row = 0, dummy0, dummy1, dummy2, dummy3;
+        if (tb < te) tile_rows(p, tb, dummy0, dummy1, dummy2, first_row, dummy3);
+        int next_issue = first_row;  // next global row to load (tid 0 only)
+        uint32_t a_phase = 0;
+        bool ok = true;
+        for (int tile = tb; tile < te; ++tile) {
+            int n, y0, y1, lo, hi;
+            tile_rows(p, tile, n, y0, y1, lo, hi);
+            // All producers are done with the previous tile, so rows below lo
+            // are free: load what this tile and the next one need.  The same
+            // barrier makes the decision to stop (a wait that ran out)
+            // uniform across the producers.
+            __syncwarp();
+            if (!named_bar_and(2, kProd, ok)) break;
+            if (tid == 0) {
+                int nhi = hi;
+                if (tile + 1 < te) {
+                    int n2, a2, b2, lo2, hi2;
+                    tile_rows(p, tile + 1, n2, a2, b2, lo2, hi2);
+                    nhi = hi2;
+                }
+                while (next_issue <= nhi && next_issue - kRing < lo) {
+                    const int slot = next_issue % kRing;
+                    mbar_arrive_expect_tx(&ring_full[slot], row_tx);
+                    tma_load_3d(&tmX, &ring_full[slot], ring + slot * p.row_bytes, 0, 0, next_issue);
+                    ++next_issue;
+                }
+            }
+            __syncwarp();
+            for (int r = lo; ok && r <= hi; ++r)
+                ok = bounded_wait(&ring_full[r % kRing], static_cast<uint32_t>(((r - first_row) / kRing) & 1), w,
+                                  SITE_DW_RING);
+            if (ok) ok = bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY);
+            if (!ok) continue;  // leave together at the next barrier
+            const int npix = (y1 - y0 + 1) * W;
+            const int base_row = n * H;
+            // Thread tid keeps channel group g (weights in registers) and takes
+            // pixels pi0, pi0 + pstep, ...
+            for (int pi = pi0; pi < npix; pi += pstep) {
+                const int ly = pi / W;
+                const int x = pi - ly * W;
+                const int y = y0 + ly;
+                float acc[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
+                int slot = (base_row + y - 1 + kRing) % kRing;  // row y - 1
+#pragma unroll
+                for (int di = 0; di < 3; ++di) {
+                    const int yy = y + di - 1;
+                    if (yy >= 0 && yy < H) {
+                        const uint8_t *rowp = ring + slot * p.row_bytes + g * 16;
+#pragma unroll
+                        for (int dj = 0; dj < 3; ++dj) {
+                            const int xc = x + dj - 1;
+                            if (xc < 0 || xc >= W) continue;
+                            const uint4 q = *reinterpret_cast<const uint4 *>(rowp + xc * Cin * 2);
+                            const float *wt = wreg[di * 3 + dj];
+                            acc[0] = fmaf(bf_lo(q.x), wt[0], acc[0]);
+                            acc[1] = fmaf(bf_hi(q.x), wt[1], acc[1]);
+                            acc[2] = fmaf(bf_lo(q.y), wt[2], acc[2]);
+                            acc[3] = fmaf(bf_hi(q.y), wt[3], acc[3]);
+                            acc[4] = fmaf(bf_lo(q.z), wt[4], acc[4]);
+                            acc[5] = fmaf(bf_hi(q.z), wt[5], acc[5]);
+                            acc[6] = fmaf(bf_lo(q.w), wt[6], acc[6]);
+                            acc[7] = fmaf(bf_hi(q.w), wt[7], acc[7]);
+                        }
+                    }
+                    slot = (slot + 1 == kRing) ? 0 : slot + 1;
+                }
+                uint4 o;
+                o.x = pack_bf16x2(acc[0], acc[1]);
+                o.y = pack_bf16x2(acc[2], acc[3]);
+                o.z = pack_bf16x2(acc[4], acc[5]);
+                o.w = pack_bf16x2(acc[6], acc[7]);
+                const int atom = g >> 3;
+                const int chunk = (g & 7) ^ (pi & 7);
+                *reinterpret_cast<uint4 *>(sA + atom * (kBM * 128) + pi * 128 + chunk * 16) = o;
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(a_full);
+            a_phase ^= 1u;
+        }
+        __syncwarp();
+        // Let every row copy already issued land before the CTA can exit.
+        if (tid == 0) {
+            for (int r = max(first_row, next_issue - kRing); r < next_issue; ++r) {
+                const uint32_t a = smem_u32(&ring_full[r % kRing]);
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(a, static_cast<uint32_t>(((r - first_row) / kRing) & 1)))
+                    if (globaltimer() - t0 > p.timeout_ns) break;
+            }
+        }
+        __syncwarp();
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------ weights + MMA issuer
+        if (lane == 0) {
+            bool ok = true;
+            tma_prefetch_desc(&tmW);
+            mbar_arrive_expect_tx(wbar, static_cast<uint32_t>(p.kb * p.nchunks * 8192));
+            for (int kb = 0; kb < p.kb; ++kb)
+                for (int c = 0; c < p.nchunks; ++c)
+                    tma_load_2d(&tmW, wbar, sW + (kb * p.nchunks + c) * 8192, c * 64, kb * 64);
+            ok = bounded_wait(wbar, 0, w, SITE_DW_W);
+            const uint32_t idesc = idesc_bf16_f32(kBM, Cout, false, true);
+            const int ksteps = Cin / 16;
+            int acc = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            for (int tile = tb; ok && tile < te; ++tile) {
+                if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_DW_TEMPTY)) break;
+                if (!bounded_wait(a_full, phase, w, SITE_DW_AFULL)) break;
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA);
+                const uint32_t w0 = smem_u32(sW);
+                const uint32_t d = tmem_base + static_cast<uint32_t>(acc * ncols);
+                for (int ks = 0; ks < ksteps; ++ks) {
+                    const int atom = ks >> 2, kk = ks & 3;
+                    const uint64_t ad = sdesc_sw128(a0 + atom * (kBM * 128) + kk * 32, 16, 1024);
+                    const uint64_t bd = sdesc_sw128(w0 + atom * (p.nchunks * 8192) + kk * 2048, 8192, 1024);
+                    umma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
+                }
+                umma_commit(a_empty);
+                umma_commit(&tfull[acc]);
+                phase ^= 1u;
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------ epilogue (warps 9-12)
+        const int q = warp & 3;
+        const int ew = warp - kEpiWarp0;
+        uint8_t *stg = sStage + ew * (2 * 4096);
+        int acc = 0, buf = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = tb; tile < te; ++tile) {
+            if (!__all_sync(0xffffffffu, bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL) ? 1 : 0)) break;
+            tc_fence_after();
+            int n, y0, y1, lo, hi;
+            tile_rows(p, tile, n, y0, y1, lo, hi);
+            const int npix = (y1 - y0 + 1) * W;
+            const int nv = min(32, max(0, npix - q * 32));  // valid rows of this quadrant
+            const long long row0 = (static_cast<long long>(n) * H + y0) * W + q * 32;
+            const uint32_t tb_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                     static_cast<uint32_t>(acc * ncols);
+            for (int c = 0; c < Cout && nv > 0; c += 32) {
+                uint32_t r[32];
+                if (Cout - c >= 32) {
+                    tmem_ld32(tb_addr + c, r);
+                } else {
+                    uint32_t h[16];
+                    tmem_ld16(tb_addr + c, h);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        r[i] = h[i];
+                        r[16 + i] = 0u;
+                    }
+                }
+                tmem_ld_wait();
+                if (lane == 0) bulk_wait_read<1>();
+                __syncwarp();
+                uint8_t *sb = stg + buf * 4096;
+#pragma unroll
+                for (int ch = 0; ch < 8; ++ch) {
+                    const int pos = ch ^ (lane & 7);
+                    *reinterpret_cast<uint4 *>(sb + lane * 128 + pos * 16) =
+                        make_uint4(r[4 * ch], r[4 * ch + 1], r[4 * ch + 2], r[4 * ch + 3]);
+                }
+                if (nv == 32) {
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tmOut, sb, c, static_cast<int>(row0));
+                        bulk_commit();
+                    }
+                } else {
+                    // Partial quadrant (the tile ends inside it): plain
+                    // coalesced row stores, 32 columns per row.
+                    __syncwarp();
+                    const int cols = min(32, Cout - c);
+                    for (int rr = 0; rr < nv; ++rr) {
+                        if (lane < cols) {
+                            const int pos = (lane >> 2) ^ (rr & 7);
+                            const float v = *reinterpret_cast<const float *>(sb + rr * 128 + pos * 16 + (lane & 3) * 4);
+                            p.out[(row0 + rr) * Cout + c + lane] = v;
+                        }
+                    }
+                    __syncwarp();
+                }
+                buf ^= 1;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+            __syncwarp();
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+        if (lane == 0) bulk_wait_all<0>();
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, tmem_cols);
+    }
+}
+
 }  // namespace
 
 int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
@@ -343,11 +680,59 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
     const long long M = static_cast<long long>(N) * H * W;
     if (M > (1ll << 31) - 256)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: N*H*W too large");
+    int rc;
+    // Row-ring path: rt image rows per tile, 2 * rt + 2 rows resident.
+    int rt = (W <= kBM && kProd % (Cin / 8) == 0) ? kBM / W : 0;
+    if (rt > (kRingMax - 2) / 2) rt = (kRingMax - 2) / 2;
+    while (rt > 1 && dw_row_layout(W, Cin, Cout, 2 * rt + 2).total > ds.max_smem_optin) --rt;
+    const DwRowLayout RL = dw_row_layout(W, Cin, Cout, 2 * rt + 2);
+    if (rt >= 1 && RL.total <= ds.max_smem_optin) {
+        CUtensorMap tmX, tmW, tmOut;
+        const uint64_t dims[3] = {static_cast<uint64_t>(Cin), static_cast<uint64_t>(W),
+                                  static_cast<uint64_t>(N) * H};
+        const uint64_t strides[2] = {static_cast<uint64_t>(Cin) * 2, static_cast<uint64_t>(W) * Cin * 2};
+        const uint32_t box[3] = {static_cast<uint32_t>(Cin), static_cast<uint32_t>(W), 1};
+        if ((rc = make_tmap_3d_bf16_plain(&tmX, x, dims, strides, box))) return rc;
+        if ((rc = make_tmap_2d_bf16(&tmW, pw, static_cast<uint64_t>(Cout), static_cast<uint64_t>(Cin),
+                                    static_cast<uint64_t>(Cout) * 2, 64, 64)))
+            return rc;
+        if ((rc = make_tmap_2d_f32(&tmOut, out, static_cast<uint64_t>(Cout), static_cast<uint64_t>(M),
+                                   static_cast<uint64_t>(Cout) * 4, 32, 32)))
+            return rc;
+        DwRowParams q{};
+        q.N = N;
+        q.H = H;
+        q.W = W;
+        q.Cin = Cin;
+        q.Cout = Cout;
+        q.rt = rt;
+        q.ring = 2 * rt + 2;
+        q.tiles_per_img = (H + q.rt - 1) / q.rt;
+        q.tiles = N * q.tiles_per_img;
+        q.kb = (Cin + 63) / 64;
+        q.nchunks = (Cout + 63) / 64;
+        q.row_bytes = (W * Cin * 2 + 127) / 128 * 128;
+        q.dw = dw;
+        q.out = out;
+        q.timeout_ns = wait_timeout_ns();
+        q.err = ds.err_word;
+        static bool rattr = false;
+        if (!rattr) {
+            cudaError_t e = cudaFuncSetAttribute(dwsep_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 ds.max_smem_optin);
+            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(dwsep rows)");
+            rattr = true;
+        }
+        const int grid = q.tiles < ds.num_sms ? q.tiles : ds.num_sms;
+        dwsep_rows_kernel<<<grid, kThreads, RL.total, stream>>>(tmX, tmW, tmOut, q);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_error(e, "launch dwsep_rows_kernel");
+        return ISAM_OK;
+    }
     const DwLayout L = dw_layout(Cin, Cout);
     if (L.total > ds.max_smem_optin)
         return set_error(ISAM_ERR_UNSUPPORTED,
                          "isam_dwsep_conv: Cin=%d, Cout=%d does not fit shared memory", Cin, Cout);
-    int rc;
     CUtensorMap tmW, tmOut;
     if ((rc = make_tmap_2d_bf16(&tmW, pw, static_cast<uint64_t>(Cout), static_cast<uint64_t>(Cin),
                                 static_cast<uint64_t>(Cout) * 2, 64, 64)))

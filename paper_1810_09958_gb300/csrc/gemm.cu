@@ -454,13 +454,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // tile: S sources x 128 / S rows); each owner sums the S slices
                 // it received in rank order (deterministic) and stores its rows
                 // of C.
-                if (iter > 0 &&
-                    !warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE)) {
-                    ok = false;
-                    break;
-                }
+                // A wait that runs out skips the work but still reaches the
+                // epilogue barrier below, which makes the decision to stop
+                // uniform across the four warps.
+                bool wok = true;
+                if (iter > 0)
+                    wok = warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE);
                 const int rows_per = kBM / S;
-                {
+                if (wok) {
                     const uint32_t owner = static_cast<uint32_t>(row_local / rows_per);
                     const int rr = row_local - static_cast<int>(owner) * rows_per;
                     const uint32_t dst = mapa_shared(
@@ -493,63 +494,63 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&tempty[acc]);
                 __syncwarp();
-                if (!warp_wait<true>(red_full, static_cast<uint32_t>(iter & 1), w, SITE_EPI_REDFULL)) {
+                if (wok) wok = warp_wait<true>(red_full, static_cast<uint32_t>(iter & 1), w, SITE_EPI_REDFULL);
+                if (wok) {
+                    const int g4 = BN / 4;
+                    const int groups = rows_per * g4;
+                    for (int g = ew * 32 + lane; g < groups; g += 128) {
+                        const int rr = g / g4;
+                        const int c4 = (g % g4) * 4;
+                        const int grow = mt * kBM + static_cast<int>(rank) * rows_per + rr;
+                        const int gcol = col0 + c4;
+                        if (grow >= p.M) continue;
+                        float *crow = p.C + static_cast<size_t>(grow) * p.N;
+                        const bool vec = p.n_vec4 && gcol + 3 < p.N;
+                        float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
+                        if (p.beta != 0.0f && vec) cin = *reinterpret_cast<const float4 *>(crow + gcol);
+                        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+                        for (int r = 0; r < S; ++r) {
+                            const float4 v = *reinterpret_cast<const float4 *>(
+                                ebuf + static_cast<size_t>(r * rows_per + rr) * (BN + 4) + c4);
+                            s.x += v.x;
+                            s.y += v.y;
+                            s.z += v.z;
+                            s.w += v.w;
+                        }
+                        float o[4] = {s.x, s.y, s.z, s.w};
+                        if (vec) {
+                            float4 v;
+                            float *vv = reinterpret_cast<float *>(&v);
+                            const float *ci = reinterpret_cast<const float *>(&cin);
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                float x = p.alpha * o[j] + (p.bias ? p.bias[gcol + j] : 0.0f);
+                                if (p.beta != 0.0f) x += p.beta * ci[j];
+                                vv[j] = x;
+                            }
+                            *reinterpret_cast<float4 *>(crow + gcol) = v;
+                        } else {
+                            for (int j = 0; j < 4; ++j) {
+                                if (gcol + j >= p.N) break;
+                                float x = p.alpha * o[j] + (p.bias ? p.bias[gcol + j] : 0.0f);
+                                if (p.beta != 0.0f) x += p.beta * crow[gcol + j];
+                                crow[gcol + j] = x;
+                            }
+                        }
+                    }
+                }
+                __syncwarp();
+                if (!named_bar_and(1, 128, wok)) {
                     ok = false;
                     break;
-                }
-                const int g4 = BN / 4;
-                const int groups = rows_per * g4;
-                for (int g = ew * 32 + lane; g < groups; g += 128) {
-                    const int rr = g / g4;
-                    const int c4 = (g % g4) * 4;
-                    const int grow = mt * kBM + static_cast<int>(rank) * rows_per + rr;
-                    const int gcol = col0 + c4;
-                    if (grow >= p.M) continue;
-                    float *crow = p.C + static_cast<size_t>(grow) * p.N;
-                    const bool vec = p.n_vec4 && gcol + 3 < p.N;
-                    float4 cin = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (p.beta != 0.0f && vec) cin = *reinterpret_cast<const float4 *>(crow + gcol);
-                    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
-                    for (int r = 0; r < S; ++r) {
-                        const float4 v = *reinterpret_cast<const float4 *>(
-                            ebuf + static_cast<size_t>(r * rows_per + rr) * (BN + 4) + c4);
-                        s.x += v.x;
-                        s.y += v.y;
-                        s.z += v.z;
-                        s.w += v.w;
-                    }
-                    float o[4] = {s.x, s.y, s.z, s.w};
-                    if (vec) {
-                        float4 v;
-                        float *vv = reinterpret_cast<float *>(&v);
-                        const float *ci = reinterpret_cast<const float *>(&cin);
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            float x = p.alpha * o[j] + (p.bias ? p.bias[gcol + j] : 0.0f);
-                            if (p.beta != 0.0f) x += p.beta * ci[j];
-                            vv[j] = x;
-                        }
-                        *reinterpret_cast<float4 *>(crow + gcol) = v;
-                    } else {
-                        for (int j = 0; j < 4; ++j) {
-                            if (gcol + j >= p.N) break;
-                            float x = p.alpha * o[j] + (p.bias ? p.bias[gcol + j] : 0.0f);
-                            if (p.beta != 0.0f) x += p.beta * crow[gcol + j];
-                            crow[gcol + j] = x;
-                        }
-                    }
                 }
                 // Release the slot to every pusher, unless nobody pushes again
                 // (after the cluster's last tile no remote arrive may target an
                 // exited CTA).
-                if (tile + num_clusters < num_tiles) {
-                    __syncwarp();
-                    named_bar(1, 128);
-                    if (ew == 0 && lane == 0) {
-                        for (int r = 0; r < S; ++r) mbar_arrive_remote(red_free, static_cast<uint32_t>(r));
-                    }
-                    __syncwarp();
+                if (tile + num_clusters < num_tiles && ew == 0 && lane == 0) {
+                    for (int r = 0; r < S; ++r) mbar_arrive_remote(red_free, static_cast<uint32_t>(r));
                 }
+                __syncwarp();
             }
             if (S == 1) {
                 tc_fence_before();
