@@ -485,21 +485,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                                   SITE_DW_RING);
             if (ok) ok = bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY);
             if (!ok) continue;  // leave together at the next barrier
-            const int npix = (y1 - y0 + 1) * W;
+            const int rows = y1 - y0 + 1;
             const int base_row = n * H;
             // Thread tid keeps channel group g (weights in registers) and takes
-            // pixels pi0, pi0 + pstep, ...
-            for (int pi = pi0; pi < npix; pi += pstep) {
-                const int ly = pi / W;
-                const int x = pi - ly * W;
-                const int y = y0 + ly;
-                float acc[8];
+            // vertical pixel pairs (tile rows 2ry and 2ry + 1, column x): the
+            // pair reads 4 input rows x 3 columns, 12 taps for 2 outputs.
+            const int npairs = ((rows + 1) >> 1) * W;
+            for (int pp = pi0; pp < npairs; pp += pstep) {
+                const int ry = pp / W;
+                const int x = pp - ry * W;
+                const int ya = y0 + 2 * ry;
+                const bool two = 2 * ry + 1 < rows;
+                float acc0[8], acc1[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) acc[i] = 0.0f;
-                int slot = (base_row + y - 1 + kRing) % kRing;  // row y - 1
+                for (int i = 0; i < 8; ++i) {
+                    acc0[i] = 0.0f;
+                    acc1[i] = 0.0f;
+                }
+                int slot = (base_row + ya - 1 + kRing) % kRing;  // input row ya - 1
 #pragma unroll
-                for (int di = 0; di < 3; ++di) {
-                    const int yy = y + di - 1;
+                for (int k = 0; k < 4; ++k) {
+                    const int yy = ya - 1 + k;
                     if (yy >= 0 && yy < H) {
                         const uint8_t *rowp = ring + slot * p.row_bytes + g * 16;
 #pragma unroll
@@ -507,27 +513,48 @@ __global__ void __launch_bounds__(kThreads, 1)
                             const int xc = x + dj - 1;
                             if (xc < 0 || xc >= W) continue;
                             const uint4 q = *reinterpret_cast<const uint4 *>(rowp + xc * Cin * 2);
-                            const float *wt = wreg[di * 3 + dj];
-                            acc[0] = fmaf(bf_lo(q.x), wt[0], acc[0]);
-                            acc[1] = fmaf(bf_hi(q.x), wt[1], acc[1]);
-                            acc[2] = fmaf(bf_lo(q.y), wt[2], acc[2]);
-                            acc[3] = fmaf(bf_hi(q.y), wt[3], acc[3]);
-                            acc[4] = fmaf(bf_lo(q.z), wt[4], acc[4]);
-                            acc[5] = fmaf(bf_hi(q.z), wt[5], acc[5]);
-                            acc[6] = fmaf(bf_lo(q.w), wt[6], acc[6]);
-                            acc[7] = fmaf(bf_hi(q.w), wt[7], acc[7]);
+                            float f[8];
+                            f[0] = bf_lo(q.x);
+                            f[1] = bf_hi(q.x);
+                            f[2] = bf_lo(q.y);
+                            f[3] = bf_hi(q.y);
+                            f[4] = bf_lo(q.z);
+                            f[5] = bf_hi(q.z);
+                            f[6] = bf_lo(q.w);
+                            f[7] = bf_hi(q.w);
+                            if (k <= 2) {
+                                const float *wt = wreg[k * 3 + dj];
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) acc0[i] = fmaf(f[i], wt[i], acc0[i]);
+                            }
+                            if (k >= 1) {
+                                const float *wt = wreg[(k - 1) * 3 + dj];
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) acc1[i] = fmaf(f[i], wt[i], acc1[i]);
+                            }
                         }
                     }
                     slot = (slot + 1 == kRing) ? 0 : slot + 1;
                 }
-                uint4 o;
-                o.x = pack_bf16x2(acc[0], acc[1]);
-                o.y = pack_bf16x2(acc[2], acc[3]);
-                o.z = pack_bf16x2(acc[4], acc[5]);
-                o.w = pack_bf16x2(acc[6], acc[7]);
                 const int atom = g >> 3;
-                const int chunk = (g & 7) ^ (pi & 7);
-                *reinterpret_cast<uint4 *>(sA + atom * (kBM * 128) + pi * 128 + chunk * 16) = o;
+                {
+                    const int pi = 2 * ry * W + x;
+                    uint4 o;
+                    o.x = pack_bf16x2(acc0[0], acc0[1]);
+                    o.y = pack_bf16x2(acc0[2], acc0[3]);
+                    o.z = pack_bf16x2(acc0[4], acc0[5]);
+                    o.w = pack_bf16x2(acc0[6], acc0[7]);
+                    *reinterpret_cast<uint4 *>(sA + atom * (kBM * 128) + pi * 128 + (((g & 7) ^ (pi & 7)) << 4)) = o;
+                }
+                if (two) {
+                    const int pi = (2 * ry + 1) * W + x;
+                    uint4 o;
+                    o.x = pack_bf16x2(acc1[0], acc1[1]);
+                    o.y = pack_bf16x2(acc1[2], acc1[3]);
+                    o.z = pack_bf16x2(acc1[4], acc1[5]);
+                    o.w = pack_bf16x2(acc1[6], acc1[7]);
+                    *reinterpret_cast<uint4 *>(sA + atom * (kBM * 128) + pi * 128 + (((g & 7) ^ (pi & 7)) << 4)) = o;
+                }
             }
             fence_proxy_async_smem();
             mbar_arrive(a_full);
