@@ -5,15 +5,17 @@ Timed workload (one "step"): the tall-skinny GEMM sweep of the paper's
 DeepBench-sized GEMM benchmark (Section 5.1.1): (M, K) in {(1760,1760),
 (2560,2560), (4096,4096), (7680,2560)} x N in {16, 32, 64, 128} x {NN, TN},
 bf16 operands U[-1,1], fp32 accumulate and output, beta = 0.  32 GEMMs per
-step, each on its own operands (0.74 GB of inputs per step, larger than L2,
-so no GEMM finds its operands in L2 from the step before).
+step, each on its own operands (0.78 GB per step, larger than L2, so no
+GEMM finds its operands in L2 from the step before).  A step is one
+isam_gemm_grouped call over the 32 problems (one persistent launch).
 
 value  = GEMM TFLOP/s over the sweep (all ranks' flops / max rank time).
 e2e    = the same through host buffers: pinned host -> device copies of every
-         operand, the GEMMs, device -> host copies of every result, per step.
-roofline: the sweep's kernel (gemm_tc_kernel) is HBM-bound: algorithmic bytes
-         (2MK + 2KN + 4MN per GEMM) / summed per-launch CUDA-event time, against
-         the measured copy bandwidth.
+         operand, the grouped call, device -> host copies of every result.
+roofline: the sweep's kernel (gemm_group_kernel) is HBM-bound: algorithmic
+         bytes (2MK + 2KN + 4MN per GEMM, summed) / per-launch CUDA-event time,
+         against the measured copy bandwidth.
+per_call_sweep: the same 32 GEMMs as 32 isam_gemm calls (one launch each).
 hot_path: the other rows measured in the same run (not part of value): the
          8192^3 GEMM with beta = 1 (TFLOP/s vs dense bf16), the GRU forward
          (hidden 1024, batch 32, 128 steps: timesteps/s), the fused separable
@@ -45,6 +47,10 @@ SWEEP_N = [16, 32, 64, 128]
 METRIC = "GEMM TFLOP/s (tall-skinny sweep) and GRU timesteps/s on 1 GB300; % of roofline"
 WORKLOAD = ("tall-skinny GEMM sweep: (M,K) in {(1760,1760),(2560,2560),(4096,4096),(7680,2560)} "
             "x N in {16,32,64,128} x {NN,TN}; bf16 U[-1,1]; fp32 accumulate/output; beta=0")
+# dram__bytes_read.sum + dram__bytes_write.sum of one gemm_group_kernel launch
+# over the sweep, from the ncu capture summarised in
+# profiles/gemm_group_kernel_skinny_sweep.md (None until taken for the current kernel).
+TRAFFIC_PER_STEP = None
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -60,6 +66,12 @@ def gemm_flops(M, N, K):
 
 def gemm_bytes(M, N, K, beta=False):
     return 2.0 * M * K + 2.0 * K * N + 4.0 * M * N * (2 if beta else 1)
+
+
+def whole_job_tflops(flops_per_step: float, steps: int, world: int, max_rank_ms: float) -> float:
+    """All ranks' flops over the slowest rank's time (every rank runs the full
+    step: weak scaling)."""
+    return flops_per_step * steps * world / (max_rank_ms / 1e3) / 1e12
 
 
 def dist_env():
@@ -103,7 +115,7 @@ def row_sample(M: int, stride: int):
 
 # --------------------------------------------------------------------------- clocks
 class ClockSampler:
-    """nvidia-smi sampled every 200 ms in the background."""
+    """nvidia-smi sampled every 20 ms in the background."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -119,7 +131,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
@@ -200,18 +212,56 @@ def time_sweep(isam, probs, steps, warmup):
     end = torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
+    t0 = time.time()
     start.record(stream)
     for _ in range(steps):
         graph.replay()
     end.record(stream)
     torch.cuda.synchronize()
+    t1 = time.time()
     barrier()
     isam.sync()
-    return start.elapsed_time(end), graph
+    del graph
+    return start.elapsed_time(end), (t0, t1)
+
+
+def time_grouped(isam, probs, steps, warmup):
+    """K steps of the sweep as ONE isam_gemm_grouped launch per step (the 32
+    problems share one persistent grid), replayed as a CUDA graph."""
+    import torch
+    call = isam.GroupedGemm([(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
+                             for p in probs])
+    for _ in range(warmup):
+        call()
+    isam.sync()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        call()
+    for _ in range(warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    t0 = time.time()
+    start.record(stream)
+    for _ in range(steps):
+        graph.replay()
+    end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    barrier()
+    isam.sync()
+    del graph
+    return start.elapsed_time(end), (t0, t1)
 
 
 def time_e2e(isam, probs, steps, warmup):
-    """Same sweep through host buffers: H2D of operands, GEMMs, D2H of results."""
+    """The sweep through host buffers: per step, pinned host -> device copies of
+    every operand, one isam_gemm_grouped launch, device -> host copies of every
+    result, all on the current stream."""
     import torch
     host = []
     for p in probs:
@@ -219,12 +269,15 @@ def time_e2e(isam, probs, steps, warmup):
                      "C": torch.empty(p["M"] * p["N"], dtype=torch.float32).pin_memory()})
     h2d = sum(h["A"].numel() * 2 + h["B"].numel() * 2 for h in host)
     d2h = sum(h["C"].numel() * 4 for h in host)
+    call = isam.GroupedGemm([(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
+                             for p in probs])
 
     def one():
         for p, h in zip(probs, host):
             p["A"].copy_(h["A"], non_blocking=True)
             p["B"].copy_(h["B"], non_blocking=True)
-            isam.gemm(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
+        call()
+        for p, h in zip(probs, host):
             h["C"].copy_(p["C"], non_blocking=True)
 
     for _ in range(warmup):
@@ -414,7 +467,8 @@ def reference_arm(args):
 # --------------------------------------------------------------------------- single case
 def run_case(args):
     """Times one hot-path call on its own (for profiling and sweeps):
-    gemm:M,N,K,transA,transB,beta | gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]."""
+    sweep (the 32 sweep GEMMs in one grouped call) | gemm:M,N,K,transA,transB,beta |
+    gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]."""
     import torch
     from paper_1810_09958_gb300 import build, isam, synth
     torch.cuda.set_device(0)
@@ -434,6 +488,13 @@ def run_case(args):
         fn = lambda: isam.gemm(M, N, K, tA, tB, 1.0, A, B, beta, C)
         work = {"tflops": gemm_flops(M, N, K) / 1e12, "gb": gemm_bytes(M, N, K, beta != 0) / 1e9,
                 "plan": isam.gemm_plan(M, N, K, tA, tB, beta)}
+    elif kind == "sweep":
+        probs = make_sweep(dev)
+        call = isam.GroupedGemm([(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
+                                 for p in probs])
+        fn = call
+        work = {"tflops": sum(p["flops"] for p in probs) / 1e12,
+                "gb": sum(p["bytes"] for p in probs) / 1e9}
     elif kind == "gru":
         T, batch, H = (int(v) for v in vals) if vals else (128, 32, 1024)
         s = H ** -0.5
@@ -474,13 +535,13 @@ def run_case(args):
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--steps", type=int, default=3000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["isam", "reference"], default="isam")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-hot-path", action="store_true")
     ap.add_argument("--case", default=None,
-                    help="time one call instead of the benchmark: gemm:M,N,K,tA,tB,beta | "
+                    help="time one call instead of the benchmark: sweep (grouped) | gemm:M,N,K,tA,tB,beta | "
                          "gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]")
     args = ap.parse_args(argv)
     if args.warmup < 3:
@@ -511,53 +572,65 @@ def main(argv=None):
     torch.cuda.synchronize()
     sampler = ClockSampler(dev.index).start() if rank == 0 else None
     time.sleep(0.3)
-    t0 = time.time()
-    total_ms, graph = time_sweep(isam, probs, args.steps, args.warmup)
-    t1 = time.time()
-    kern_ms = total_ms
-    total_ms = reduce_max(total_ms, dev)
     flops_step = sum(p["flops"] for p in probs)
     bytes_step = sum(p["bytes"] for p in probs)
-    value = flops_step * args.steps * world / (total_ms / 1e3) / 1e12
-    launches = args.steps * len(probs)
 
-    e2e_ms, h2d, d2h = time_e2e(isam, probs, max(3, args.steps // 20), 2)
-    e2e_ms = reduce_max(e2e_ms, dev)
+    # value: one isam_gemm_grouped launch per step over the 32 problems.
+    kern_ms, window = time_grouped(isam, probs, args.steps, args.warmup)
+    total_ms = reduce_max(kern_ms, dev)
+    value = whole_job_tflops(flops_step, args.steps, world, total_ms)
+    launches = args.steps
+
+    # The same sweep as 32 separate isam_gemm launches per step.
+    call_ms, _ = time_sweep(isam, probs, args.steps, args.warmup)
+    call_ms = reduce_max(call_ms, dev)
+    call_value = whole_job_tflops(flops_step, args.steps, world, call_ms)
+
     e2e_steps = max(3, args.steps // 20)
-    e2e_value = flops_step * e2e_steps * world / (e2e_ms / 1e3) / 1e12
+    e2e_ms, h2d, d2h = time_e2e(isam, probs, e2e_steps, args.warmup)
+    e2e_ms = reduce_max(e2e_ms, dev)
+    e2e_value = whole_job_tflops(flops_step, e2e_steps, world, e2e_ms)
 
     hot = None
     if not args.no_hot_path:
         hot = hot_path_rows(isam, dev, peaks)
     if sampler:
         sampler.stop()
-    del probs, graph
+    del probs
     torch.cuda.empty_cache()
 
     if rank == 0:
         achieved = bytes_step * args.steps / (kern_ms / 1e3) / 1e9
+        call_gbs = bytes_step * args.steps / (call_ms / 1e3) / 1e9
         line = {
             "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": WORKLOAD, "gemms_per_step": 32,
+                       "api": "isam_gemm_grouped: the 32 GEMMs of a step in one call",
                        "l2": "inputs larger than L2: each GEMM has its own operands, "
                              f"{bytes_step / 1e9:.2f} GB per step",
                        "parallelism": f"replica x{world}"},
-            "roofline": {"kernel": "gemm_tc_kernel", "bound": "hbm", "achieved": round(achieved, 1),
+            "roofline": {"kernel": "gemm_group_kernel", "bound": "hbm", "achieved": round(achieved, 1),
                          "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                         "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": None,
+                         "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": TRAFFIC_PER_STEP,
                          "peak_source": peaks_src,
-                         "algorithmic_bytes_per_step": bytes_step,
-                         "launches_per_step": 32,
-                         "timing": "the sweep is this kernel's 32 launches back to back in a CUDA "
-                                   "graph; duration = timed-region events / steps (inter-launch "
-                                   "gaps included)"},
+                         "algorithmic_bytes_per_launch": bytes_step,
+                         "launches_per_step": 1,
+                         "timing": "one launch per step, replayed from a CUDA graph; duration = "
+                                   "timed-region CUDA events on the replay stream / steps"},
             "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                    "what": "pinned host operands copied in, isam_gemm_grouped, results copied out"},
             "gpu_launches": launches,
-            "clocks": sampler.summary(t0, t1) if sampler else None,
+            "clocks": sampler.summary(*window) if sampler else None,
+            "per_call_sweep": {
+                "value": round(call_value, 3), "unit": "TFLOP/s",
+                "ms_per_step": round(call_ms / args.steps, 5), "achieved_gbs": round(call_gbs, 1),
+                "frac_hbm": round(call_gbs / peaks["hbm_gbs"], 4), "launches_per_step": 32,
+                "what": "the same 32 GEMMs as 32 isam_gemm calls per step (gemm_tc_kernel), "
+                        "graph-replayed; inter-launch gaps included"},
         }
         if hot is not None:
             line["hot_path"] = hot

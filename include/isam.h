@@ -91,6 +91,26 @@ int isam_gemm(int M, int N, int K, int transA, int transB, float alpha,
               const isam_bf16 *A, const isam_bf16 *B, float beta, float *C);
 
 /*
+ * Several independent GEMMs in one launch: problem i computes
+ * C[i] <- alpha[i] * op(A[i]) * op(B[i]) + beta[i] * C[i] exactly as isam_gemm
+ * would, with the same per-problem argument rules.
+ *
+ * The tiles of all problems are scheduled across the GPU's SMs by one
+ * persistent kernel (the paper's scheduler placing compute tiles across
+ * compute units, Sections 3.3-3.4, over a set of matrix multiplications), so
+ * the per-launch costs are paid once for the group.  Arrays M..C are HOST
+ * arrays of count entries; A[i], B[i], C[i] are device pointers.
+ *   - 1 <= count <= 64 (else ISAM_ERR_INVALID_ARG).
+ *   - The problems run concurrently: no C[i] may overlap any A[j], B[j] or
+ *     another C[j]; results are undefined otherwise.
+ *   - Tile width is min(128, N rounded up to 16) per problem; no split-K.
+ * Errors name the offending problem.
+ */
+int isam_gemm_grouped(int count, const int *M, const int *N, const int *K, const int *transA,
+                      const int *transB, const float *alpha, const isam_bf16 *const *A,
+                      const isam_bf16 *const *B, const float *beta, float *const *C);
+
+/*
  * The tile plan isam_gemm would use for this problem, chosen by the
  * library's analytic cost model (the paper's "Approach" interface for
  * tiling and device-allocation choices, Sections 3.4 and 4).  Nothing is

@@ -263,6 +263,29 @@ int isam_gemm(int M, int N, int K, int transA, int transB, float alpha, const is
     return gemm_launch(g, plan, *ds, current_stream());
 }
 
+int isam_gemm_grouped(int count, const int *M, const int *N, const int *K, const int *transA,
+                      const int *transB, const float *alpha, const isam_bf16 *const *A,
+                      const isam_bf16 *const *B, const float *beta, float *const *C) {
+    if (count < 1 || count > 64)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped: count must be in [1, 64]");
+    if (!M || !N || !K || !transA || !transB || !alpha || !A || !B || !beta || !C)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped: null array");
+    GemmDesc g[64];
+    for (int i = 0; i < count; ++i) {
+        g[i] = GemmDesc{M[i], N[i], K[i], transA[i], transB[i], alpha[i], beta[i], A[i], B[i], C[i], nullptr};
+        int rc = gemm_validate(g[i]);
+        if (rc) {
+            char msg[512];
+            snprintf(msg, sizeof msg, "isam_gemm_grouped: problem %d: %s", i, isam_last_error_string());
+            return set_error(rc, "%s", msg);
+        }
+    }
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gemm_grouped_launch(count, g, *ds, current_stream());
+}
+
 // Reports the tile plan the cost model picks for a GEMM (for benchmarks and
 // tests; nothing is launched).  out[0..5] = BN, split, stages, group_m, grid,
 // shared-memory bytes.

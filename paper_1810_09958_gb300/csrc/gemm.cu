@@ -22,6 +22,7 @@
 #include <cstring>
 #include <mutex>
 
+#include "gemm_common.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -82,24 +83,6 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
     const int local = tile - g * per_group;
     mt = first_m + local % gm;
     nt = local / gm;
-}
-
-// Waits ignoring the abort flag (used only to let copies already issued land).
-__device__ bool drain_wait(uint64_t *bar, uint32_t parity, unsigned long long timeout_ns) {
-    const uint32_t a = smem_u32(bar);
-    const unsigned long long t0 = globaltimer();
-    while (!mbar_try_wait(a, parity)) {
-        if (globaltimer() - t0 > timeout_ns) return false;
-    }
-    return true;
-}
-
-// bounded_wait by every lane of a warp, with a warp-uniform result.
-template <bool cluster_scope = false>
-__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, const WaitCtx &w,
-                                          uint32_t site) {
-    const bool ok = bounded_wait<cluster_scope>(bar, parity, w, site);
-    return __all_sync(0xffffffffu, ok) != 0;
 }
 
 template <int BN, bool A_MN, bool B_MN>

@@ -1,0 +1,437 @@
+// gemm_grouped.cu -- many independent GEMMs in one persistent tcgen05 launch.
+//
+// The tiles of every problem form one list that the persistent CTAs walk
+// round-robin (problems ordered by decreasing tile cost on the host), so the
+// SMs stream the operands of several problems at once and the per-launch costs
+// -- pipeline fill to the first data, the last tile's epilogue, the gap
+// between kernels -- are paid once for the whole group instead of once per
+// problem.  This is the paper's scheduler placing compute tiles across compute
+// units (Sections 3.3-3.4) applied across a set of matrix multiplications.
+//
+// Per CTA: warp 0 TMA producer, warp 1 single-thread tcgen05.mma issuer into a
+// double-buffered TMEM accumulator, warps 2-5 epilogue moving C through
+// swizzled shared memory with TMA (or plain stores when a row of C is not
+// 16-byte aligned).  Layout (NN/TN/NT/TT) and tile width are per problem; a
+// problem's tensor maps travel in the kernel parameters.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <numeric>
+
+#include "gemm_common.cuh"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace isam {
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+constexpr int kMaxGroup = 64;
+constexpr int kBNMax = 128;
+constexpr int kAStage = kBM * kBK * 2;      // 16 KB
+constexpr int kBStage = kBNMax * kBK * 2;   // 16 KB (either B layout at BN = 128)
+constexpr int kEpiBytes = 4 * 2 * 4096;     // per-warp 2 x 32x32 fp32 staging
+
+enum : uint32_t {
+    SITE_G_EMPTY = 0x401,
+    SITE_G_TEMPTY = 0x402,
+    SITE_G_FULL = 0x403,
+    SITE_G_TFULL = 0x404,
+    SITE_G_CLOAD = 0x405,
+    SITE_G_DONE = 0x406,
+};
+
+struct GroupProblem {
+    int M, N, K;
+    int m_tiles, n_tiles, kb_total;
+    int a_mn, b_mn, bn;
+    int tma_c;        // C rows 16-byte aligned: TMA epilogue
+    int tile_start;   // first global tile index of this problem
+    float alpha, beta;
+    float *C;
+};
+
+struct GroupParams {
+    int count, total_tiles, stages;
+    unsigned long long timeout_ns;
+    uint32_t *err;
+    GroupProblem prob[kMaxGroup];
+    CUtensorMap tmA[kMaxGroup];
+    CUtensorMap tmB[kMaxGroup];
+    CUtensorMap tmC[kMaxGroup];
+};
+
+__device__ __forceinline__ int find_problem(const GroupParams &p, int tile) {
+    int i = 0;
+    while (i + 1 < p.count && p.prob[i + 1].tile_start <= tile) ++i;
+    return i;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_constant__ GroupParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~static_cast<uintptr_t>(1023));
+    const int ST = p.stages;
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + static_cast<size_t>(ST) * kAStage;
+    uint8_t *ebuf = sB + static_cast<size_t>(ST) * kBStage;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(ebuf + kEpiBytes);
+    uint64_t *full = bars;
+    uint64_t *empty = bars + ST;
+    uint64_t *tfull = empty + ST;
+    uint64_t *tempty = tfull + 2;
+    uint64_t *cbar = tempty + 2;    // [4 warps][2]
+    uint64_t *done = cbar + 8;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    constexpr uint32_t kTmemCols = 2 * kBNMax;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < ST; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&tfull[i], 1);
+            mbar_init(&tempty[i], 4);
+        }
+        for (int i = 0; i < 8; ++i) mbar_init(&cbar[i], 1);
+        mbar_init(done, 4);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncwarp();
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const WaitCtx w{p.timeout_ns, p.err, abort_flag};
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            int stage = 0, issued = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; ok && tile < p.total_tiles; tile += gridDim.x) {
+                const int pi = find_problem(p, tile);
+                const GroupProblem &pr = p.prob[pi];
+                const int local = tile - pr.tile_start;
+                const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
+                const uint32_t bbytes = pr.b_mn ? static_cast<uint32_t>((pr.bn + 63) / 64) * 8192u
+                                                : static_cast<uint32_t>(pr.bn) * 128u;
+                for (int kb = 0; kb < pr.kb_total; ++kb) {
+                    if (!bounded_wait(&empty[stage], phase ^ 1u, w, SITE_G_EMPTY)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(kAStage) + bbytes);
+                    uint8_t *a = sA + static_cast<size_t>(stage) * kAStage;
+                    uint8_t *b = sB + static_cast<size_t>(stage) * kBStage;
+                    const int k0 = kb * kBK;
+                    if (pr.a_mn) {
+                        tma_load_2d(&p.tmA[pi], &full[stage], a, mt * kBM, k0);
+                        tma_load_2d(&p.tmA[pi], &full[stage], a + 8192, mt * kBM + 64, k0);
+                    } else {
+                        tma_load_2d(&p.tmA[pi], &full[stage], a, k0, mt * kBM);
+                    }
+                    if (pr.b_mn) {
+                        for (int c = 0; c < (pr.bn + 63) / 64; ++c)
+                            tma_load_2d(&p.tmB[pi], &full[stage], b + c * 8192, nt * pr.bn + c * 64, k0);
+                    } else {
+                        tma_load_2d(&p.tmB[pi], &full[stage], b, k0, nt * pr.bn);
+                    }
+                    ++issued;
+                    if (++stage == ST) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                const int pending = min(issued, ST);
+                int s = stage;
+                uint32_t ph = phase;
+                for (int i = 0; i < pending; ++i) {
+                    if (--s < 0) {
+                        s = ST - 1;
+                        ph ^= 1u;
+                    }
+                    drain_wait(&full[s], ph, p.timeout_ns);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            int stage = 0, acc = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            bool ok = true;
+            for (int tile = blockIdx.x; ok && tile < p.total_tiles; tile += gridDim.x) {
+                const GroupProblem &pr = p.prob[find_problem(p, tile)];
+                const uint32_t idesc = idesc_bf16_f32(kBM, pr.bn, pr.a_mn != 0, pr.b_mn != 0);
+                if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_G_TEMPTY)) break;
+                tc_fence_after();
+                const uint32_t d = tmem_base + static_cast<uint32_t>(acc * kBNMax);
+                for (int kb = 0; kb < pr.kb_total; ++kb) {
+                    if (!bounded_wait(&full[stage], phase, w, SITE_G_FULL)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(sA + static_cast<size_t>(stage) * kAStage);
+                    const uint32_t b0 = smem_u32(sB + static_cast<size_t>(stage) * kBStage);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k) {
+                        const uint64_t ad = pr.a_mn ? sdesc_sw128(a0 + k * 2048, 8192, 1024)
+                                                    : sdesc_sw128(a0 + k * 32, 16, 1024);
+                        const uint64_t bd = pr.b_mn ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
+                                                    : sdesc_sw128(b0 + k * 32, 16, 1024);
+                        umma_bf16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                    }
+                    umma_commit(&empty[stage]);
+                    if (++stage == ST) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                umma_commit(&tfull[acc]);
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_phase ^= 1u;
+                }
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------ epilogue (warps 2-5)
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        uint8_t *stg = ebuf + ew * 8192;
+        uint64_t *cb = cbar + ew * 2;
+        uint32_t cpar[2] = {0u, 0u};
+        bool cpend[2] = {false, false};
+        int gbuf = 0, acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < p.total_tiles; tile += gridDim.x) {
+            const int pi = find_problem(p, tile);
+            const GroupProblem &pr = p.prob[pi];
+            const int local = tile - pr.tile_start;
+            const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
+            const int row0 = mt * kBM + q * 32;
+            const int col0 = nt * pr.bn;
+            const bool load_c = pr.tma_c && pr.beta != 0.0f;
+            const int nch = (pr.bn + 31) / 32;
+            if (load_c) {
+                if (lane == 0) {
+                    bulk_wait_read<0>();
+                    const int b = gbuf & 1;
+                    mbar_arrive_expect_tx(&cb[b], 4096);
+                    tma_load_2d(&p.tmC[pi], &cb[b], stg + b * 4096, col0, row0);
+                }
+                cpend[gbuf & 1] = true;
+                __syncwarp();
+            }
+            if (!warp_wait(&tfull[acc], acc_phase, w, SITE_G_TFULL)) break;
+            tc_fence_after();
+            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                   static_cast<uint32_t>(acc * kBNMax);
+            bool ok = true;
+            for (int j = 0; j < nch; ++j) {
+                const int b = gbuf & 1;
+                if (load_c && j + 1 < nch) {
+                    if (lane == 0) {
+                        bulk_wait_read<0>();
+                        mbar_arrive_expect_tx(&cb[b ^ 1], 4096);
+                        tma_load_2d(&p.tmC[pi], &cb[b ^ 1], stg + (b ^ 1) * 4096, col0 + (j + 1) * 32, row0);
+                    }
+                    cpend[b ^ 1] = true;
+                }
+                if (!load_c && lane == 0) bulk_wait_read<1>();
+                uint32_t r[32];
+                if (pr.bn - j * 32 >= 32) {
+                    tmem_ld32(tbase + j * 32, r);
+                } else {
+                    uint32_t h[16];
+                    tmem_ld16(tbase + j * 32, h);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        r[i] = h[i];
+                        r[16 + i] = 0u;
+                    }
+                }
+                tmem_ld_wait();
+                if (load_c) {
+                    if (!warp_wait(&cb[b], cpar[b], w, SITE_G_CLOAD)) {
+                        ok = false;
+                        break;
+                    }
+                    cpar[b] ^= 1u;
+                    cpend[b] = false;
+                }
+                __syncwarp();
+                uint8_t *sb = stg + b * 4096;
+#pragma unroll
+                for (int ch = 0; ch < 8; ++ch) {
+                    const int pos = ch ^ (lane & 7);
+                    float4 *slot = reinterpret_cast<float4 *>(sb + lane * 128 + pos * 16);
+                    float4 v = make_float4(pr.alpha * __uint_as_float(r[4 * ch]),
+                                           pr.alpha * __uint_as_float(r[4 * ch + 1]),
+                                           pr.alpha * __uint_as_float(r[4 * ch + 2]),
+                                           pr.alpha * __uint_as_float(r[4 * ch + 3]));
+                    if (load_c) {
+                        const float4 cv = *slot;
+                        v.x += pr.beta * cv.x;
+                        v.y += pr.beta * cv.y;
+                        v.z += pr.beta * cv.z;
+                        v.w += pr.beta * cv.w;
+                    }
+                    *slot = v;
+                }
+                const int cbase = col0 + j * 32;
+                if (pr.tma_c) {
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&p.tmC[pi], sb, cbase, row0);
+                        bulk_commit();
+                    }
+                } else {
+                    // Rows of C not 16-byte aligned: plain stores, one row per
+                    // iteration, 32 consecutive columns (coalesced).
+                    __syncwarp();
+                    const int col = cbase + lane;
+                    for (int rr = 0; rr < 32; ++rr) {
+                        const int grow = row0 + rr;
+                        if (grow >= pr.M) break;
+                        if (col < pr.N && lane < pr.bn - j * 32) {
+                            const int pos = (lane >> 2) ^ (rr & 7);
+                            float v = *reinterpret_cast<const float *>(sb + rr * 128 + pos * 16 + (lane & 3) * 4);
+                            if (pr.beta != 0.0f) v += pr.beta * pr.C[static_cast<size_t>(grow) * pr.N + col];
+                            pr.C[static_cast<size_t>(grow) * pr.N + col] = v;
+                        }
+                    }
+                    __syncwarp();
+                }
+                ++gbuf;
+            }
+            if (!ok) break;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+            __syncwarp();
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+        for (int b = 0; b < 2; ++b)
+            if (cpend[b] && lane == 0) drain_wait(&cb[b], cpar[b], p.timeout_ns);
+        if (lane == 0) bulk_wait_all<0>();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(done);
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        bounded_wait(done, 0, w, SITE_G_DONE);
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+size_t group_smem_bytes(int stages) {
+    return 1024 + static_cast<size_t>(stages) * (kAStage + kBStage) + kEpiBytes + (2 * stages + 13) * 8 + 16;
+}
+
+std::mutex g_group_mu;
+bool g_group_attr = false;
+
+}  // namespace
+
+int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStream_t stream) {
+    if (count < 1 || count > kMaxGroup)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped: count must be in [1, %d]", kMaxGroup);
+    // Host-side order: problems with the costliest tiles first, so the
+    // round-robin walk over tiles ends with the cheap ones.
+    int order[kMaxGroup];
+    std::iota(order, order + count, 0);
+    std::stable_sort(order, order + count, [&](int a, int b) { return g[a].K > g[b].K; });
+
+    static GroupParams p;  // ~29 KB: built under the lock, copied into the launch
+    std::lock_guard<std::mutex> lk(g_group_mu);
+    memset(&p, 0, sizeof p);
+    p.count = count;
+    int tiles = 0;
+    for (int s = 0; s < count; ++s) {
+        const GemmDesc &d = g[order[s]];
+        GroupProblem &pr = p.prob[s];
+        pr.M = d.M;
+        pr.N = d.N;
+        pr.K = d.K;
+        pr.a_mn = d.transA;
+        pr.b_mn = d.transB == 0 ? 1 : 0;
+        pr.bn = std::min(kBNMax, (d.N + 15) / 16 * 16);
+        pr.m_tiles = (d.M + kBM - 1) / kBM;
+        pr.n_tiles = (d.N + pr.bn - 1) / pr.bn;
+        pr.kb_total = (d.K + kBK - 1) / kBK;
+        pr.tma_c = (d.N % 4 == 0) ? 1 : 0;
+        pr.tile_start = tiles;
+        pr.alpha = d.alpha;
+        pr.beta = d.beta;
+        pr.C = d.C;
+        tiles += pr.m_tiles * pr.n_tiles;
+        int rc;
+        if (pr.a_mn)
+            rc = make_tmap_2d_bf16(&p.tmA[s], d.A, d.M, d.K, static_cast<uint64_t>(d.M) * 2, 64, 64);
+        else
+            rc = make_tmap_2d_bf16(&p.tmA[s], d.A, d.K, d.M, static_cast<uint64_t>(d.K) * 2, 64, kBM);
+        if (rc) return rc;
+        if (pr.b_mn)
+            rc = make_tmap_2d_bf16(&p.tmB[s], d.B, d.N, d.K, static_cast<uint64_t>(d.N) * 2, 64, 64);
+        else
+            rc = make_tmap_2d_bf16(&p.tmB[s], d.B, d.K, d.N, static_cast<uint64_t>(d.K) * 2, 64,
+                                   static_cast<uint32_t>(pr.bn));
+        if (rc) return rc;
+        if (pr.tma_c &&
+            (rc = make_tmap_2d_f32(&p.tmC[s], d.C, d.N, d.M, static_cast<uint64_t>(d.N) * 4, 32, 32)))
+            return rc;
+    }
+    p.total_tiles = tiles;
+    int st = 8;
+    while (st > 2 && group_smem_bytes(st) > static_cast<size_t>(ds.max_smem_optin)) --st;
+    p.stages = st;
+    p.timeout_ns = wait_timeout_ns();
+    p.err = ds.err_word;
+    const size_t smem = group_smem_bytes(st);
+    if (!g_group_attr) {
+        cudaError_t e = cudaFuncSetAttribute(gemm_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             ds.max_smem_optin);
+        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(grouped gemm)");
+        g_group_attr = true;
+    }
+    const int grid = std::min(tiles, ds.num_sms);
+    gemm_group_kernel<<<grid, kThreads, smem, stream>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_error(e, "launch gemm_group_kernel");
+    return ISAM_OK;
+}
+
+}  // namespace isam

@@ -70,6 +70,9 @@ int gemm_validate(const GemmDesc &g);
 int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan);
 int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t s);
 
+// Independent GEMMs in one persistent launch (1 <= count <= 64).
+int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStream_t s);
+
 int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
                const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
                cudaStream_t s);

@@ -56,10 +56,12 @@ def load():
         lib.isam_shutdown.argtypes = []
         lib.isam_gemm.argtypes = [i, i, i, i, i, f, P, P, f, P]
         lib.isam_gemm_plan_info.argtypes = [i, i, i, i, i, f, P]
+        lib.isam_gemm_grouped.argtypes = [i, P, P, P, P, P, P, P, P, P, P]
         lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
-                     "isam_gemm_plan_info", "isam_gru_forward", "isam_dwsep_conv"):
+                     "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gru_forward",
+                     "isam_dwsep_conv"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
         return lib
@@ -115,6 +117,37 @@ def gemm(M, N, K, transA, transB, alpha, A, B, beta, C) -> None:
     _use_current_stream(lib)
     check(lib.isam_gemm(M, N, K, int(transA), int(transB), float(alpha), _ptr(A), _ptr(B),
                         float(beta), _ptr(C)))
+
+
+class GroupedGemm:
+    """Marshalled argument arrays of one isam_gemm_grouped call (build once,
+    call many times: the arrays keep the ctypes buffers alive)."""
+
+    def __init__(self, problems):
+        import torch
+        n = len(problems)
+        ia = lambda vals: (ctypes.c_int * n)(*vals)
+        fa = lambda vals: (ctypes.c_float * n)(*vals)
+        pa = lambda vals: (ctypes.c_void_p * n)(*vals)
+        for (M, N, K, tA, tB, alpha, A, B, beta, C) in problems:
+            _dev(A, torch.bfloat16, M * K, "A")
+            _dev(B, torch.bfloat16, K * N, "B")
+            _dev(C, torch.float32, M * N, "C")
+        cols = list(zip(*problems))
+        self.n = n
+        self.args = (ia(cols[0]), ia(cols[1]), ia(cols[2]), ia(cols[3]), ia(cols[4]), fa(cols[5]),
+                     pa([t.data_ptr() for t in cols[6]]), pa([t.data_ptr() for t in cols[7]]), fa(cols[8]),
+                     pa([t.data_ptr() for t in cols[9]]))
+
+    def __call__(self):
+        lib = load()
+        _use_current_stream(lib)
+        check(lib.isam_gemm_grouped(self.n, *self.args))
+
+
+def gemm_grouped(problems) -> None:
+    """isam_gemm_grouped over a list of (M, N, K, transA, transB, alpha, A, B, beta, C)."""
+    GroupedGemm(problems)()
 
 
 def gemm_plan(M, N, K, transA, transB, beta=0.0) -> dict:

@@ -58,3 +58,10 @@ def test_binding_has_no_fallback(monkeypatch, tmp_path):
     monkeypatch.setattr(isam, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(ImportError):
         isam.load()
+
+
+def test_grouped_rejects_bad_count_without_cuda(lib):
+    p = ctypes.c_void_p(16)
+    assert lib.isam_gemm_grouped(0, p, p, p, p, p, p, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gemm_grouped(65, p, p, p, p, p, p, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gemm_grouped(2, None, p, p, p, p, p, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
