@@ -217,6 +217,13 @@ int isam_sync(void) {
     uint32_t w[4] = {0, 0, 0, 0};
     if ((e = cudaMemcpy(w, ds->err_word, sizeof w, cudaMemcpyDeviceToHost)) != cudaSuccess)
         return cuda_error(e, "reading the device error word");
+    if (w[0] & DEV_ERR_LAUNCH_SHAPE) {
+        cudaMemset(ds->err_word, 0, 16);
+        return set_error(ISAM_ERR_CUDA,
+                         "a cluster kernel found clusters of %u CTAs, not the shape it was launched "
+                         "for (site 0x%x, block %u); it returned without computing",
+                         w[3], w[1], w[2]);
+    }
     if (w[0] != 0) {
         cudaMemset(ds->err_word, 0, 16);
         return set_error(ISAM_ERR_TIMEOUT,

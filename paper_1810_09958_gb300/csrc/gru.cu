@@ -125,6 +125,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     gru_recurrent_kernel(const __grid_constant__ CUtensorMap tmU,
                          const __grid_constant__ CUtensorMap tmH0,
                          const __grid_constant__ CUtensorMap tmH1, const GruParams p) {
+    if (!launch_shape_ok(p.err, static_cast<uint32_t>(p.ks), static_cast<uint32_t>(p.n_cta), 0x3F0u))
+        return;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
@@ -671,6 +673,11 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
     uint32_t w[4] = {0, 0, 0, 0};
     if ((e = cudaMemcpy(w, err, sizeof w, cudaMemcpyDeviceToHost)) != cudaSuccess)
         return cuda_error(e, "isam_gru_forward_noalloc: reading the scratch error word");
+    if (w[0] & DEV_ERR_LAUNCH_SHAPE)
+        return set_error(ISAM_ERR_CUDA,
+                         "isam_gru_forward_noalloc: the recurrent kernel found clusters of %u CTAs, "
+                         "not the shape it was launched for; h_out is undefined",
+                         w[3]);
     if (w[0] != 0)
         return set_error(ISAM_ERR_TIMEOUT,
                          "isam_gru_forward_noalloc: a bounded device wait ran out (site 0x%x, "

@@ -10,6 +10,11 @@
 
 namespace isam {
 
+// Device error word layout (uint32 x 4), written by kernels and read by
+// isam_sync: [0] flags, [1] site of the first error, [2] blockIdx.x of that
+// CTA, [3] detail (the cluster size a kernel found, for a launch-shape error).
+enum : uint32_t { DEV_ERR_TIMEOUT = 1u, DEV_ERR_LAUNCH_SHAPE = 2u };
+
 // Per-device state, created on first use with that device current.
 struct DeviceState {
     int device = -1;

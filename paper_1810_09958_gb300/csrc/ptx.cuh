@@ -9,11 +9,9 @@
 #include <cstdint>
 #include <cuda.h>
 
-namespace isam {
+#include "internal.h"
 
-// Device error word layout (uint32 x 4): [0] flags, [1] site of the first
-// timeout, [2] blockIdx.x of that CTA, [3] reserved.
-enum : uint32_t { DEV_ERR_TIMEOUT = 1u };
+namespace isam {
 
 struct WaitCtx {
     unsigned long long timeout_ns;
@@ -325,6 +323,29 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
     uint32_t r;
     asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
     return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+
+// Kernels that address peer CTAs' shared memory (mapa / st.shared::cluster)
+// call this first: when the launch did not give them clusters of `want` CTAs
+// and a grid of `grid` CTAs (a launcher or tool that dropped the cluster
+// attribute), they record a launch-shape error and return before touching any
+// barrier or peer address.  The decision is the same in every CTA.
+static __device__ __noinline__ bool launch_shape_ok(uint32_t *err, uint32_t want, uint32_t grid,
+                                                    uint32_t site) {
+    const uint32_t got = cluster_nctarank();
+    if (got == want && gridDim.x == grid) return true;
+    if (threadIdx.x == 0 && atomicOr(err, DEV_ERR_LAUNCH_SHAPE) == 0u) {
+        err[1] = site;
+        err[2] = blockIdx.x;
+        err[3] = got;
+    }
+    return false;
 }
 
 __device__ __forceinline__ void cluster_sync_all() {
