@@ -50,7 +50,7 @@ WORKLOAD = ("tall-skinny GEMM sweep: (M,K) in {(1760,1760),(2560,2560),(4096,409
 # dram__bytes_read.sum + dram__bytes_write.sum of one gemm_group_kernel launch
 # over the sweep, from the ncu capture summarised in
 # profiles/gemm_group_kernel_skinny_sweep.md (None until taken for the current kernel).
-TRAFFIC_PER_STEP = None
+TRAFFIC_PER_STEP = 749125376 + 26610176
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
