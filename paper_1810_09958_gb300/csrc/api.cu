@@ -167,17 +167,6 @@ int make_tmap_2d_f32(CUtensorMap *out, const void *base, uint64_t inner, uint64_
     return encode(out, key, 2, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
 }
 
-int make_tmap_3d_bf16_plain(CUtensorMap *out, const void *base, const uint64_t dims_in[3],
-                            const uint64_t strides_bytes[2], const uint32_t box_in[3]) {
-    const uint64_t key[12] = {0x3A, reinterpret_cast<uint64_t>(base), dims_in[0], dims_in[1], dims_in[2],
-                              strides_bytes[0], strides_bytes[1], box_in[0], box_in[1], box_in[2], 0, 0};
-    cuuint64_t dims[3] = {dims_in[0], dims_in[1], dims_in[2]};
-    cuuint64_t strides[2] = {strides_bytes[0], strides_bytes[1]};
-    cuuint32_t box[3] = {box_in[0], box_in[1], box_in[2]};
-    return encode(out, key, 3, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
-                  CU_TENSOR_MAP_SWIZZLE_NONE);
-}
-
 int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims_in[3],
                       const uint64_t strides_bytes[2], const uint32_t box_in[3]) {
     const uint64_t key[12] = {3,           reinterpret_cast<uint64_t>(base),

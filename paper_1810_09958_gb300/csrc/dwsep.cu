@@ -82,9 +82,34 @@ __device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v <<
 __device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-    const uint32_t l = __bfloat16_as_ushort(__float2bfloat16_rn(lo));
-    const uint32_t h = __bfloat16_as_ushort(__float2bfloat16_rn(hi));
-    return l | (h << 16);
+    uint32_t r;  // round-to-nearest-even of both; hi in the upper half
+    asm("cvt.rn.bf16x2.f32 %0, %2, %1;" : "=r"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+// c + a * w with a and w bf16 (the lower or upper halves of x and wp) and c
+// fp32: both bf16 operands widen exactly to fp32, and the multiply-add rounds
+// once, as fmaf on the widened values would.
+__device__ __forceinline__ float fma_bf16_lo(uint32_t x, uint32_t wp, float c) {
+    float d;
+    asm("{\n\t.reg .b16 xl, xh, wl, wh;\n\t"
+        "mov.b32 {xl, xh}, %1;\n\t"
+        "mov.b32 {wl, wh}, %2;\n\t"
+        "fma.rn.f32.bf16 %0, xl, wl, %3;\n\t}"
+        : "=f"(d)
+        : "r"(x), "r"(wp), "f"(c));
+    return d;
+}
+
+__device__ __forceinline__ float fma_bf16_hi(uint32_t x, uint32_t wp, float c) {
+    float d;
+    asm("{\n\t.reg .b16 xl, xh, wl, wh;\n\t"
+        "mov.b32 {xl, xh}, %1;\n\t"
+        "mov.b32 {wl, wh}, %2;\n\t"
+        "fma.rn.f32.bf16 %0, xh, wh, %3;\n\t}"
+        : "=f"(d)
+        : "r"(x), "r"(wp), "f"(c));
+    return d;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -344,7 +369,8 @@ struct DwRowParams {
     int tiles_per_img;   // ceil(H / rt)
     int tiles;           // N * tiles_per_img
     int kb, nchunks;
-    int row_bytes;       // one input row in shared memory (W * Cin * 2, rounded to 128)
+    const uint16_t *x;   // NHWC input: row (n * H + y) is W * Cin contiguous elements
+    int row_bytes;       // one ring slot: W * Cin * 2 bytes of pixels + >= one pixel of zeros, rounded to 128
     int ring;            // input rows resident per CTA (2 * rt + 2 <= kRingMax)
     const uint16_t *dw;
     float *out;
@@ -352,21 +378,27 @@ struct DwRowParams {
     uint32_t *err;
 };
 
+// The ring: a leading pad of dw_ring_lead bytes, then `ring` slots of
+// dw_ring_row_bytes each.  A slot holds one input row (W pixels, written by
+// TMA) followed by at least one pixel of zeros, so the left neighbour of
+// pixel 0 (the previous slot's tail, or the leading pad) and the right
+// neighbour of pixel W - 1 read as zero: the taps need no bounds test along x.
+__host__ __device__ inline int dw_ring_lead(int Cin) { return (Cin * 2 + 127) / 128 * 128; }
+__host__ __device__ inline int dw_ring_row_bytes(int W, int Cin) { return (W * Cin * 2 + Cin * 2 + 127) / 128 * 128; }
+
 struct DwRowLayout {
-    int off_ring, off_a, off_w, off_stage, off_dwf, off_bars, total;
+    int off_ring, off_a, off_w, off_stage, off_bars, total;
 };
 
 __host__ __device__ inline DwRowLayout dw_row_layout(int W, int Cin, int Cout, int ring) {
     DwRowLayout L;
-    const int row_bytes = (W * Cin * 2 + 127) / 128 * 128;
     const int atoms = (Cin + 63) / 64;
     const int nchunks = (Cout + 63) / 64;
     L.off_ring = 0;
-    L.off_a = (ring * row_bytes + 1023) / 1024 * 1024;
+    L.off_a = (dw_ring_lead(Cin) + ring * dw_ring_row_bytes(W, Cin) + 1023) / 1024 * 1024;
     L.off_w = L.off_a + atoms * kBM * 128;
     L.off_stage = L.off_w + atoms * nchunks * 8192;
-    L.off_dwf = L.off_stage + 4 * 2 * 4096;
-    L.off_bars = L.off_dwf + ((9 * Cin * 4) + 1023) / 1024 * 1024;
+    L.off_bars = L.off_stage + 4 * 2 * 4096;
     L.total = L.off_bars + 8 * (kRingMax + 8) + 16 + 1024;
     return L;
 }
@@ -381,19 +413,63 @@ __device__ __forceinline__ void tile_rows(const DwRowParams &p, int tile, int &n
     hi = n * p.H + min(p.H - 1, y1 + 1);
 }
 
+// The 3x3 depthwise sums of one vertical pixel pair (rows ya and ya + 1,
+// column x) for the 4 channels whose bf16 weights are in wb: acc0 for row ya,
+// acc1 for row ya + 1.  Input row ya - 1 + k is ring slot (slot0 + k) mod
+// kRing; pixels x - 1 and x + 1 may be the zero pad.  kCheckRows skips input
+// rows outside the image; tiles with no such row run the straight-line form.
+template <bool kCheckRows>
+__device__ __forceinline__ void dw_pair(const uint8_t *ring, int row_bytes, int kRing, int slot0, int ya,
+                                        int H, int x, int Cin2, int g, const uint32_t (&wb)[9][2],
+                                        float (&acc0)[4], float (&acc1)[4]) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        acc0[i] = 0.0f;
+        acc1[i] = 0.0f;
+    }
+    int slot = slot0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int yy = ya - 1 + k;
+        if (!kCheckRows || (yy >= 0 && yy < H)) {
+            const uint8_t *rp = ring + slot * row_bytes + x * Cin2 + g * 8;
+#pragma unroll
+            for (int dj = 0; dj < 3; ++dj) {
+                const uint2 q = *reinterpret_cast<const uint2 *>(rp + (dj - 1) * Cin2);
+                if (k <= 2) {
+                    const uint32_t *wt = wb[k * 3 + dj];
+                    acc0[0] = fma_bf16_lo(q.x, wt[0], acc0[0]);
+                    acc0[1] = fma_bf16_hi(q.x, wt[0], acc0[1]);
+                    acc0[2] = fma_bf16_lo(q.y, wt[1], acc0[2]);
+                    acc0[3] = fma_bf16_hi(q.y, wt[1], acc0[3]);
+                }
+                if (k >= 1) {
+                    const uint32_t *wt = wb[(k - 1) * 3 + dj];
+                    acc1[0] = fma_bf16_lo(q.x, wt[0], acc1[0]);
+                    acc1[1] = fma_bf16_hi(q.x, wt[0], acc1[1]);
+                    acc1[2] = fma_bf16_lo(q.y, wt[1], acc1[2]);
+                    acc1[3] = fma_bf16_hi(q.y, wt[1], acc1[3]);
+                }
+            }
+        }
+        slot = (slot + 1 == kRing) ? 0 : slot + 1;
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-    dwsep_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                      const __grid_constant__ CUtensorMap tmOut, const DwRowParams p) {
+    dwsep_rows_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmOut,
+                      const __grid_constant__ CUtensorMap tmOut16, const __grid_constant__ CUtensorMap tmOut8,
+                      const DwRowParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
     const DwRowLayout L = dw_row_layout(p.W, p.Cin, p.Cout, p.ring);
     const int kRing = p.ring;
-    uint8_t *ring = smem + L.off_ring;
+    const int lead = dw_ring_lead(p.Cin);
+    uint8_t *ring = smem + L.off_ring + lead;  // slot s starts at ring + s * row_bytes
     uint8_t *sA = smem + L.off_a;
     uint8_t *sW = smem + L.off_w;
     uint8_t *sStage = smem + L.off_stage;
-    float *dwf = reinterpret_cast<float *>(smem + L.off_dwf);
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L.off_bars);
     uint64_t *ring_full = bars;           // [ring]
     uint64_t *a_full = ring_full + kRing;
@@ -416,7 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (tid == 0) {
         for (int i = 0; i < kRing; ++i) mbar_init(&ring_full[i], 1);
-        mbar_init(a_full, kProd);
+        mbar_init(a_full, kProdWarps);
         mbar_init(a_empty, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
@@ -426,8 +502,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         *abort_flag = 0;
         fence_mbar_init();
     }
-    for (int i = tid; i < 9 * Cin; i += kThreads)
-        dwf[i] = __uint_as_float(static_cast<uint32_t>(p.dw[i]) << 16);
+    {
+        // Zero the leading pad and every slot's tail (TMA never writes them).
+        const int tail = p.row_bytes - W * Cin * 2;  // multiple of 16
+        const int units = (lead + kRing * tail) / 16;
+        for (int i = tid; i < units; i += kThreads) {
+            const int off = i * 16;
+            int at;
+            if (off < lead) {
+                at = off;
+            } else {
+                const int s = (off - lead) / tail;
+                at = lead + s * p.row_bytes + W * Cin * 2 + (off - lead - s * tail);
+            }
+            *reinterpret_cast<uint4 *>(smem + L.off_ring + at) = make_uint4(0u, 0u, 0u, 0u);
+        }
+    }
     __syncwarp();
     if (warp == kMmaWarp) {
         tmem_alloc(tmem_slot, tmem_cols);
@@ -441,24 +531,60 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp < kProdWarps) {
         // ------------------------------------------------ depthwise producers
-        const int groups = Cin / 8;  // divides kProd (Cin is 16, 32, ..., 256)
+        // Thread tid owns 4 channels (group g, weights in registers); with
+        // Cin = 128 the 32 lanes of a warp cover one pixel's channels, so
+        // the image-edge decisions below are the same for the whole warp.
+        // Tile, row and ring-slot positions advance incrementally: an integer
+        // division by a run-time value costs hundreds of cycles of latency,
+        // and here it would sit on the critical path of every tile.
+        const int groups = Cin / 4;  // divides kProd (Cin is 16, 32, ..., 256)
         const uint32_t row_tx = static_cast<uint32_t>(W * Cin * 2);
         const int g = tid % groups;
         const int pi0 = tid / groups;
         const int pstep = kProd / groups;
-        float wreg[9][8];
+        uint32_t wb[9][2];  // bf16 weights of channels 4g..4g+3, two per word
 #pragma unroll
-        for (int t = 0; t < 9; ++t)
-#pragma unroll
-            for (int i = 0; i < 8; ++i) wreg[t][i] = dwf[t * Cin + g * 8 + i];
-        int first_row = 0, dummy0, dummy1, dummy2, dummy3;
-        if (tb < te) tile_rows(p, tb, dummy0, dummy1, dummy2, first_row, dummy3);
-        int next_issue = first_row;  // next global row to load (tid 0 only)
+        for (int t = 0; t < 9; ++t) {
+            const uint2 wv = *reinterpret_cast<const uint2 *>(p.dw + t * Cin + g * 4);
+            wb[t][0] = wv.x;
+            wb[t][1] = wv.y;
+        }
+        // Channels 4g..4g+3 in the A tile: K atom g / 16, 16-byte chunk
+        // (g % 16) / 2 (swizzled by the pixel row), half g % 2 of the chunk.
+        const int atom = g >> 4;
+        const int chunk = (g & 15) >> 1;
+        const int half = (g & 1) * 8;
+        // Global input row r lives in ring slot (r - first_row) mod kRing;
+        // its barrier completes phase (r - first_row) / kRing.
+        int n = 0, yt = 0, first_row = 0;
+        if (tb < te) {
+            n = tb / p.tiles_per_img;
+            yt = tb - n * p.tiles_per_img;
+            first_row = n * H + max(0, yt * p.rt - 1);
+        }
+        int lo_prev = first_row, lo_slot = 0;  // slot and round of this tile's first row
+        uint32_t lo_round = 0;
+        int next_issue = first_row, is_slot = 0;  // next row to load (tid 0)
+        uint32_t is_round = 0;
         uint32_t a_phase = 0;
         bool ok = true;
         for (int tile = tb; tile < te; ++tile) {
-            int n, y0, y1, lo, hi;
-            tile_rows(p, tile, n, y0, y1, lo, hi);
+            const int y0 = yt * p.rt;
+            const int y1 = min(H, y0 + p.rt) - 1;
+            const int base_row = n * H;
+            const int lo = base_row + max(0, y0 - 1);
+            const int hi = base_row + min(H - 1, y1 + 1);
+            for (int d = lo - lo_prev; d > 0; --d)
+                if (++lo_slot == kRing) {
+                    lo_slot = 0;
+                    ++lo_round;
+                }
+            lo_prev = lo;
+            int n2 = n, yt2 = yt + 1;
+            if (yt2 == p.tiles_per_img) {
+                yt2 = 0;
+                ++n2;
+            }
             // All producers are done with the previous tile, so rows below lo
             // are free: load what this tile and the next one need.  The same
             // barrier makes the decision to stop (a wait that ran out)
@@ -466,107 +592,108 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (!named_bar_and(2, kProd, ok)) break;
             if (tid == 0) {
-                int nhi = hi;
-                if (tile + 1 < te) {
-                    int n2, a2, b2, lo2, hi2;
-                    tile_rows(p, tile + 1, n2, a2, b2, lo2, hi2);
-                    nhi = hi2;
-                }
+                const int nhi = tile + 1 < te ? n2 * H + min(H - 1, min(H, yt2 * p.rt + p.rt)) : hi;
                 while (next_issue <= nhi && next_issue - kRing < lo) {
-                    const int slot = next_issue % kRing;
-                    mbar_arrive_expect_tx(&ring_full[slot], row_tx);
-                    tma_load_3d(&tmX, &ring_full[slot], ring + slot * p.row_bytes, 0, 0, next_issue);
+                    mbar_arrive_expect_tx(&ring_full[is_slot], row_tx);
+                    bulk_load(ring + is_slot * p.row_bytes,
+                              p.x + static_cast<size_t>(next_issue) * W * Cin, row_tx, &ring_full[is_slot]);
                     ++next_issue;
+                    if (++is_slot == kRing) {
+                        is_slot = 0;
+                        ++is_round;
+                    }
                 }
             }
+            // One lane per warp polls the barriers; the barrier after it
+            // combines the answers and joins the producers again.  (Without
+            // it a warp whose lane 0 took the branch alone stayed split for
+            // the whole first round of the tile: measured 3x slower.)
             __syncwarp();
-            for (int r = lo; ok && r <= hi; ++r)
-                ok = bounded_wait(&ring_full[r % kRing], static_cast<uint32_t>(((r - first_row) / kRing) & 1), w,
-                                  SITE_DW_RING);
-            if (ok) ok = bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY);
+            bool wok = true;
+            if (lane == 0) {
+                int sl = lo_slot;
+                uint32_t rnd = lo_round;
+                for (int r = lo; wok && r <= hi; ++r) {
+                    wok = bounded_wait(&ring_full[sl], rnd & 1u, w, SITE_DW_RING);
+                    if (++sl == kRing) {
+                        sl = 0;
+                        ++rnd;
+                    }
+                }
+                if (wok) wok = bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY);
+            }
+            __syncwarp();
+            ok = named_bar_and(2, kProd, wok);
             if (!ok) continue;  // leave together at the next barrier
             const int rows = y1 - y0 + 1;
-            const int base_row = n * H;
-            // Thread tid keeps channel group g (weights in registers) and takes
-            // vertical pixel pairs (tile rows 2ry and 2ry + 1, column x): the
-            // pair reads 4 input rows x 3 columns, 12 taps for 2 outputs.
+            // Ring slot of input row y0 - 1 (any slot when y0 == 0: that row is
+            // outside the image and never used).
+            int s_top = lo_slot + (base_row + y0 - 1 - lo);
+            if (s_top < 0) s_top += kRing;
+            // Each thread takes vertical pixel pairs (tile rows 2ry and
+            // 2ry + 1, column x): the pair reads 4 input rows x 3 columns,
+            // 12 taps for 2 outputs.  Every lane of a warp runs the same
+            // number of rounds and the __syncwarp at the end of a round
+            // rejoins the lanes.  Interior tiles run the tap loop without a
+            // branch, so all 12 loads can be in flight at once.
             const int npairs = ((rows + 1) >> 1) * W;
-            for (int pp = pi0; pp < npairs; pp += pstep) {
-                const int ry = pp / W;
-                const int x = pp - ry * W;
+            // Every input row the tile reads lies inside the image.
+            const bool interior = y0 >= 1 && y1 + 1 <= H - 1;
+            int ry = 0, x = pi0;
+            while (x >= W) {
+                x -= W;
+                ++ry;
+            }
+            for (int pp0 = 0; pp0 < npairs; pp0 += pstep) {
+                const bool act = pp0 + pi0 < npairs;
                 const int ya = y0 + 2 * ry;
-                const bool two = 2 * ry + 1 < rows;
-                float acc0[8], acc1[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    acc0[i] = 0.0f;
-                    acc1[i] = 0.0f;
-                }
-                int slot = (base_row + ya - 1 + kRing) % kRing;  // input row ya - 1
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const int yy = ya - 1 + k;
-                    if (yy >= 0 && yy < H) {
-                        const uint8_t *rowp = ring + slot * p.row_bytes + g * 16;
-#pragma unroll
-                        for (int dj = 0; dj < 3; ++dj) {
-                            const int xc = x + dj - 1;
-                            if (xc < 0 || xc >= W) continue;
-                            const uint4 q = *reinterpret_cast<const uint4 *>(rowp + xc * Cin * 2);
-                            float f[8];
-                            f[0] = bf_lo(q.x);
-                            f[1] = bf_hi(q.x);
-                            f[2] = bf_lo(q.y);
-                            f[3] = bf_hi(q.y);
-                            f[4] = bf_lo(q.z);
-                            f[5] = bf_hi(q.z);
-                            f[6] = bf_lo(q.w);
-                            f[7] = bf_hi(q.w);
-                            if (k <= 2) {
-                                const float *wt = wreg[k * 3 + dj];
-#pragma unroll
-                                for (int i = 0; i < 8; ++i) acc0[i] = fmaf(f[i], wt[i], acc0[i]);
-                            }
-                            if (k >= 1) {
-                                const float *wt = wreg[(k - 1) * 3 + dj];
-#pragma unroll
-                                for (int i = 0; i < 8; ++i) acc1[i] = fmaf(f[i], wt[i], acc1[i]);
-                            }
-                        }
-                    }
-                    slot = (slot + 1 == kRing) ? 0 : slot + 1;
-                }
-                const int atom = g >> 3;
-                {
+                const bool two = act && (2 * ry + 1 < rows);
+                int slot = s_top + 2 * ry;  // input row ya - 1
+                while (slot >= kRing) slot -= kRing;
+                float acc0[4], acc1[4];
+                if (interior)
+                    dw_pair<false>(ring, p.row_bytes, kRing, slot, ya, H, x, Cin * 2, g, wb, acc0, acc1);
+                else
+                    dw_pair<true>(ring, p.row_bytes, kRing, slot, ya, H, x, Cin * 2, g, wb, acc0, acc1);
+                if (act) {
                     const int pi = 2 * ry * W + x;
-                    uint4 o;
-                    o.x = pack_bf16x2(acc0[0], acc0[1]);
-                    o.y = pack_bf16x2(acc0[2], acc0[3]);
-                    o.z = pack_bf16x2(acc0[4], acc0[5]);
-                    o.w = pack_bf16x2(acc0[6], acc0[7]);
-                    *reinterpret_cast<uint4 *>(sA + atom * (kBM * 128) + pi * 128 + (((g & 7) ^ (pi & 7)) << 4)) = o;
+                    const uint2 o = make_uint2(pack_bf16x2(acc0[0], acc0[1]), pack_bf16x2(acc0[2], acc0[3]));
+                    *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) + half) = o;
                 }
                 if (two) {
                     const int pi = (2 * ry + 1) * W + x;
-                    uint4 o;
-                    o.x = pack_bf16x2(acc1[0], acc1[1]);
-                    o.y = pack_bf16x2(acc1[2], acc1[3]);
-                    o.z = pack_bf16x2(acc1[4], acc1[5]);
-                    o.w = pack_bf16x2(acc1[6], acc1[7]);
-                    *reinterpret_cast<uint4 *>(sA + atom * (kBM * 128) + pi * 128 + (((g & 7) ^ (pi & 7)) << 4)) = o;
+                    const uint2 o = make_uint2(pack_bf16x2(acc1[0], acc1[1]), pack_bf16x2(acc1[2], acc1[3]));
+                    *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) + half) = o;
+                }
+                __syncwarp();
+                x += pstep;
+                while (x >= W) {
+                    x -= W;
+                    ++ry;
                 }
             }
             fence_proxy_async_smem();
-            mbar_arrive(a_full);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(a_full);
             a_phase ^= 1u;
+            n = n2;
+            yt = yt2;
         }
         __syncwarp();
         // Let every row copy already issued land before the CTA can exit.
         if (tid == 0) {
-            for (int r = max(first_row, next_issue - kRing); r < next_issue; ++r) {
-                const uint32_t a = smem_u32(&ring_full[r % kRing]);
+            int sl = is_slot;
+            uint32_t rnd = is_round;
+            for (int i = 0; i < kRing && next_issue - 1 - i >= first_row; ++i) {
+                if (sl == 0) {
+                    sl = kRing - 1;
+                    --rnd;
+                } else {
+                    --sl;
+                }
+                const uint32_t a = smem_u32(&ring_full[sl]);
                 const unsigned long long t0 = globaltimer();
-                while (!mbar_try_wait(a, static_cast<uint32_t>(((r - first_row) / kRing) & 1)))
+                while (!mbar_try_wait(a, rnd & 1u))
                     if (globaltimer() - t0 > p.timeout_ns) break;
             }
         }
@@ -616,7 +743,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         int acc = 0, buf = 0;
         uint32_t acc_phase = 0;
         for (int tile = tb; tile < te; ++tile) {
-            if (!__all_sync(0xffffffffu, bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL) ? 1 : 0)) break;
+            bool tok = true;
+            if (lane == 0) tok = bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL);
+            __syncwarp();
+            // The 4 epilogue warps decide together and leave the wait joined.
+            if (!named_bar_and(3, 128, tok)) break;
             tc_fence_after();
             int n, y0, y1, lo, hi;
             tile_rows(p, tile, n, y0, y1, lo, hi);
@@ -656,11 +787,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                         bulk_commit();
                     }
                 } else {
-                    // Partial quadrant (the tile ends inside it): plain
-                    // coalesced row stores, 32 columns per row.
+                    // Partial quadrant (the tile ends inside it): its first
+                    // 16 and/or 8 rows by TMA (boxes of 16 and 8 rows), the
+                    // rest (fewer than 8) by plain coalesced row stores.
+                    const int r16 = nv >= 16 ? 16 : 0;
+                    const int r8 = nv - r16 >= 8 ? 8 : 0;
+                    if (r16 + r8 > 0) {
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            if (r16) tma_store_2d(&tmOut16, sb, c, static_cast<int>(row0));
+                            if (r8) tma_store_2d(&tmOut8, sb + r16 * 128, c, static_cast<int>(row0) + r16);
+                            bulk_commit();
+                        }
+                    }
                     __syncwarp();
                     const int cols = min(32, Cout - c);
-                    for (int rr = 0; rr < nv; ++rr) {
+                    for (int rr = r16 + r8; rr < nv; ++rr) {
                         if (lane < cols) {
                             const int pos = (lane >> 2) ^ (rr & 7);
                             const float v = *reinterpret_cast<const float *>(sb + rr * 128 + pos * 16 + (lane & 3) * 4);
@@ -670,6 +813,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
                 buf ^= 1;
+                __syncwarp();  // joined again before the next aligned tcgen05.ld
             }
             tc_fence_before();
             __syncwarp();
@@ -709,23 +853,21 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: N*H*W too large");
     int rc;
     // Row-ring path: rt image rows per tile, 2 * rt + 2 rows resident.
-    int rt = (W <= kBM && kProd % (Cin / 8) == 0) ? kBM / W : 0;
+    int rt = (W <= kBM && kProd % (Cin / 4) == 0) ? kBM / W : 0;
     if (rt > (kRingMax - 2) / 2) rt = (kRingMax - 2) / 2;
     while (rt > 1 && dw_row_layout(W, Cin, Cout, 2 * rt + 2).total > ds.max_smem_optin) --rt;
     const DwRowLayout RL = dw_row_layout(W, Cin, Cout, 2 * rt + 2);
     if (rt >= 1 && RL.total <= ds.max_smem_optin) {
-        CUtensorMap tmX, tmW, tmOut;
-        const uint64_t dims[3] = {static_cast<uint64_t>(Cin), static_cast<uint64_t>(W),
-                                  static_cast<uint64_t>(N) * H};
-        const uint64_t strides[2] = {static_cast<uint64_t>(Cin) * 2, static_cast<uint64_t>(W) * Cin * 2};
-        const uint32_t box[3] = {static_cast<uint32_t>(Cin), static_cast<uint32_t>(W), 1};
-        if ((rc = make_tmap_3d_bf16_plain(&tmX, x, dims, strides, box))) return rc;
+        CUtensorMap tmW, tmOut, tmOut16, tmOut8;
         if ((rc = make_tmap_2d_bf16(&tmW, pw, static_cast<uint64_t>(Cout), static_cast<uint64_t>(Cin),
                                     static_cast<uint64_t>(Cout) * 2, 64, 64)))
             return rc;
-        if ((rc = make_tmap_2d_f32(&tmOut, out, static_cast<uint64_t>(Cout), static_cast<uint64_t>(M),
-                                   static_cast<uint64_t>(Cout) * 4, 32, 32)))
-            return rc;
+        // Output boxes of 32 columns x 32, 16 and 8 rows.
+        CUtensorMap *outs[3] = {&tmOut, &tmOut16, &tmOut8};
+        for (int i = 0; i < 3; ++i)
+            if ((rc = make_tmap_2d_f32(outs[i], out, static_cast<uint64_t>(Cout), static_cast<uint64_t>(M),
+                                       static_cast<uint64_t>(Cout) * 4, 32, 32u >> i)))
+                return rc;
         DwRowParams q{};
         q.N = N;
         q.H = H;
@@ -738,7 +880,8 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
         q.tiles = N * q.tiles_per_img;
         q.kb = (Cin + 63) / 64;
         q.nchunks = (Cout + 63) / 64;
-        q.row_bytes = (W * Cin * 2 + 127) / 128 * 128;
+        q.row_bytes = dw_ring_row_bytes(W, Cin);
+        q.x = x;
         q.dw = dw;
         q.out = out;
         q.timeout_ns = wait_timeout_ns();
@@ -751,7 +894,7 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
             rattr = true;
         }
         const int grid = q.tiles < ds.num_sms ? q.tiles : ds.num_sms;
-        dwsep_rows_kernel<<<grid, kThreads, RL.total, stream>>>(tmX, tmW, tmOut, q);
+        dwsep_rows_kernel<<<grid, kThreads, RL.total, stream>>>(tmW, tmOut, tmOut16, tmOut8, q);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_error(e, "launch dwsep_rows_kernel");
         return ISAM_OK;

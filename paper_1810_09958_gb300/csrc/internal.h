@@ -42,9 +42,6 @@ int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64
                       uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
 int make_tmap_2d_f32(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
                      uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
-// Same without swizzling (rows land packed in shared memory).
-int make_tmap_3d_bf16_plain(CUtensorMap *out, const void *base, const uint64_t dims[3],
-                            const uint64_t strides_bytes[2], const uint32_t box[3]);
 int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims[3],
                       const uint64_t strides_bytes[2], const uint32_t box[3]);
 

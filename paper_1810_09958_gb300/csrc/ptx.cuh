@@ -142,6 +142,16 @@ __device__ __forceinline__ void tma_load_3d(const void *map, uint64_t *bar, void
         : "memory");
 }
 
+// Contiguous copy of `bytes` (a multiple of 16) from global to shared memory,
+// both 16-byte aligned; completion is counted on the mbarrier.
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
 // 3-D tensor box multicast to every CTA of the cluster in cta_mask: the data
 // lands at the same shared offset in each, and each CTA's mbarrier at the same
 // offset receives the complete_tx.
