@@ -359,6 +359,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 // a shared-memory ring filled by one TMA copy per row.  Every input element
 // then leaves L2 about once per CTA, and the producers read the 3x3 taps from
 // shared memory.
+constexpr int kRProdWarps = 12;               // depthwise producer warps 0-11
+constexpr int kRProd = kRProdWarps * 32;
+constexpr int kRMmaWarp = kRProdWarps;         // warp 12: ring loader + MMA issuer
+constexpr int kREpiWarp0 = kRProdWarps + 1;    // warps 13-16: epilogue
+constexpr int kRThreads = (kRProdWarps + 5) * 32;
 constexpr int kRingMax = 32;  // input rows resident per CTA: 2 * rt + 2 (this tile + halo + the next)
 
 enum : uint32_t { SITE_DW_RING = 0x306 };
@@ -413,6 +418,32 @@ __device__ __forceinline__ void tile_rows(const DwRowParams &p, int tile, int &n
     hi = n * p.H + min(p.H - 1, y1 + 1);
 }
 
+// A tile of the row-ring kernel: image n, tile row yt (image rows
+// yt * rt .. yt * rt + rt - 1); it reads global input rows dw_lo .. dw_hi.
+struct DwTilePos {
+    int n, yt;
+};
+
+__device__ __forceinline__ DwTilePos dw_pos(const DwRowParams &p, int tile) {
+    const int n = tile / p.tiles_per_img;
+    return DwTilePos{n, tile - n * p.tiles_per_img};
+}
+
+__device__ __forceinline__ void dw_advance(const DwRowParams &p, DwTilePos &t) {
+    if (++t.yt == p.tiles_per_img) {
+        t.yt = 0;
+        ++t.n;
+    }
+}
+
+__device__ __forceinline__ int dw_lo(const DwRowParams &p, DwTilePos t) {
+    return t.n * p.H + max(0, t.yt * p.rt - 1);
+}
+
+__device__ __forceinline__ int dw_hi(const DwRowParams &p, DwTilePos t) {
+    return t.n * p.H + min(p.H - 1, min(p.H, t.yt * p.rt + p.rt));
+}
+
 // The 3x3 depthwise sums of one vertical pixel pair (rows ya and ya + 1,
 // column x) for the 4 channels whose bf16 weights are in wb: acc0 for row ya,
 // acc1 for row ya + 1.  Input row ya - 1 + k is ring slot (slot0 + k) mod
@@ -456,7 +487,7 @@ __device__ __forceinline__ void dw_pair(const uint8_t *ring, int row_bytes, int 
     }
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kRThreads, 1)
     dwsep_rows_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmOut,
                       const __grid_constant__ CUtensorMap tmOut16, const __grid_constant__ CUtensorMap tmOut8,
                       const DwRowParams p) {
@@ -492,7 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (tid == 0) {
         for (int i = 0; i < kRing; ++i) mbar_init(&ring_full[i], 1);
-        mbar_init(a_full, kProdWarps);
+        mbar_init(a_full, kRProdWarps);
         mbar_init(a_empty, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
@@ -506,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Zero the leading pad and every slot's tail (TMA never writes them).
         const int tail = p.row_bytes - W * Cin * 2;  // multiple of 16
         const int units = (lead + kRing * tail) / 16;
-        for (int i = tid; i < units; i += kThreads) {
+        for (int i = tid; i < units; i += kRThreads) {
             const int off = i * 16;
             int at;
             if (off < lead) {
@@ -519,7 +550,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
     __syncwarp();
-    if (warp == kMmaWarp) {
+    if (warp == kRMmaWarp) {
         tmem_alloc(tmem_slot, tmem_cols);
         tmem_relinquish();
     }
@@ -529,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
     const WaitCtx w{p.timeout_ns, p.err, abort_flag};
 
-    if (warp < kProdWarps) {
+    if (warp < kRProdWarps) {
         // ------------------------------------------------ depthwise producers
         // Thread tid owns 4 channels (group g, weights in registers); with
         // Cin = 128 the 32 lanes of a warp cover one pixel's channels, so
@@ -537,11 +568,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Tile, row and ring-slot positions advance incrementally: an integer
         // division by a run-time value costs hundreds of cycles of latency,
         // and here it would sit on the critical path of every tile.
-        const int groups = Cin / 4;  // divides kProd (Cin is 16, 32, ..., 256)
-        const uint32_t row_tx = static_cast<uint32_t>(W * Cin * 2);
+        const int groups = Cin / 4;  // divides kRProd (Cin is 16, 32, ..., 256)
         const int g = tid % groups;
         const int pi0 = tid / groups;
-        const int pstep = kProd / groups;
+        const int pstep = kRProd / groups;
         uint32_t wb[9][2];  // bf16 weights of channels 4g..4g+3, two per word
 #pragma unroll
         for (int t = 0; t < 9; ++t) {
@@ -555,76 +585,48 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int chunk = (g & 15) >> 1;
         const int half = (g & 1) * 8;
         // Global input row r lives in ring slot (r - first_row) mod kRing;
-        // its barrier completes phase (r - first_row) / kRing.
-        int n = 0, yt = 0, first_row = 0;
-        if (tb < te) {
-            n = tb / p.tiles_per_img;
-            yt = tb - n * p.tiles_per_img;
-            first_row = n * H + max(0, yt * p.rt - 1);
-        }
+        // its barrier completes phase (r - first_row) / kRing.  The MMA
+        // thread loads the rows; the producers only wait for them.
+        DwTilePos pos = dw_pos(p, tb);
+        const int first_row = tb < te ? dw_lo(p, pos) : 0;
         int lo_prev = first_row, lo_slot = 0;  // slot and round of this tile's first row
         uint32_t lo_round = 0;
-        int next_issue = first_row, is_slot = 0;  // next row to load (tid 0)
-        uint32_t is_round = 0;
         uint32_t a_phase = 0;
-        bool ok = true;
+        bool ok = true, a_ok = true;
         for (int tile = tb; tile < te; ++tile) {
-            const int y0 = yt * p.rt;
+            const int n = pos.n;
+            const int y0 = pos.yt * p.rt;
             const int y1 = min(H, y0 + p.rt) - 1;
             const int base_row = n * H;
-            const int lo = base_row + max(0, y0 - 1);
-            const int hi = base_row + min(H - 1, y1 + 1);
+            const int lo = dw_lo(p, pos);
+            const int hi = dw_hi(p, pos);
             for (int d = lo - lo_prev; d > 0; --d)
                 if (++lo_slot == kRing) {
                     lo_slot = 0;
                     ++lo_round;
                 }
             lo_prev = lo;
-            int n2 = n, yt2 = yt + 1;
-            if (yt2 == p.tiles_per_img) {
-                yt2 = 0;
-                ++n2;
-            }
-            // All producers are done with the previous tile, so rows below lo
-            // are free: load what this tile and the next one need.  The same
-            // barrier makes the decision to stop (a wait that ran out)
-            // uniform across the producers.
+            // Lane k of each warp polls the barrier of the tile's k-th input
+            // row, all at once (one after another they cost a barrier round
+            // trip each); the barrier after it combines the answers (and a
+            // failed A-stage wait of the previous tile) and joins the
+            // producers again.  (Without it a warp whose lanes took different
+            // branches stayed split for the whole first round of the tile:
+            // measured 3x slower.)
             __syncwarp();
-            if (!named_bar_and(2, kProd, ok)) break;
-            if (tid == 0) {
-                const int nhi = tile + 1 < te ? n2 * H + min(H - 1, min(H, yt2 * p.rt + p.rt)) : hi;
-                while (next_issue <= nhi && next_issue - kRing < lo) {
-                    mbar_arrive_expect_tx(&ring_full[is_slot], row_tx);
-                    bulk_load(ring + is_slot * p.row_bytes,
-                              p.x + static_cast<size_t>(next_issue) * W * Cin, row_tx, &ring_full[is_slot]);
-                    ++next_issue;
-                    if (++is_slot == kRing) {
-                        is_slot = 0;
-                        ++is_round;
-                    }
-                }
-            }
-            // One lane per warp polls the barriers; the barrier after it
-            // combines the answers and joins the producers again.  (Without
-            // it a warp whose lane 0 took the branch alone stayed split for
-            // the whole first round of the tile: measured 3x slower.)
-            __syncwarp();
-            bool wok = true;
-            if (lane == 0) {
-                int sl = lo_slot;
+            bool wok = a_ok;
+            if (lane <= hi - lo) {
+                int sl = lo_slot + lane;
                 uint32_t rnd = lo_round;
-                for (int r = lo; wok && r <= hi; ++r) {
-                    wok = bounded_wait(&ring_full[sl], rnd & 1u, w, SITE_DW_RING);
-                    if (++sl == kRing) {
-                        sl = 0;
-                        ++rnd;
-                    }
+                if (sl >= kRing) {
+                    sl -= kRing;
+                    ++rnd;
                 }
-                if (wok) wok = bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY);
+                wok = wok && bounded_wait(&ring_full[sl], rnd & 1u, w, SITE_DW_RING);
             }
             __syncwarp();
-            ok = named_bar_and(2, kProd, wok);
-            if (!ok) continue;  // leave together at the next barrier
+            ok = named_bar_and(2, kRProd, wok);
+            if (!ok) break;  // the same decision in every producer
             const int rows = y1 - y0 + 1;
             // Ring slot of input row y0 - 1 (any slot when y0 == 0: that row is
             // outside the image and never used).
@@ -655,12 +657,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     dw_pair<false>(ring, p.row_bytes, kRing, slot, ya, H, x, Cin * 2, g, wb, acc0, acc1);
                 else
                     dw_pair<true>(ring, p.row_bytes, kRing, slot, ya, H, x, Cin * 2, g, wb, acc0, acc1);
-                if (act) {
+                if (pp0 == 0) {
+                    // The A stage is free once the MMA of the previous tile is
+                    // done; the first round's taps are computed meanwhile.
+                    a_ok = __all_sync(0xffffffffu, bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY));
+                }
+                if (act && a_ok) {
                     const int pi = 2 * ry * W + x;
                     const uint2 o = make_uint2(pack_bf16x2(acc0[0], acc0[1]), pack_bf16x2(acc0[2], acc0[3]));
                     *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) + half) = o;
                 }
-                if (two) {
+                if (two && a_ok) {
                     const int pi = (2 * ry + 1) * W + x;
                     const uint2 o = make_uint2(pack_bf16x2(acc1[0], acc1[1]), pack_bf16x2(acc1[2], acc1[3]));
                     *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) + half) = o;
@@ -676,31 +683,38 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(a_full);
             a_phase ^= 1u;
-            n = n2;
-            yt = yt2;
+            dw_advance(p, pos);
         }
         __syncwarp();
-        // Let every row copy already issued land before the CTA can exit.
-        if (tid == 0) {
-            int sl = is_slot;
-            uint32_t rnd = is_round;
-            for (int i = 0; i < kRing && next_issue - 1 - i >= first_row; ++i) {
-                if (sl == 0) {
-                    sl = kRing - 1;
-                    --rnd;
-                } else {
-                    --sl;
-                }
-                const uint32_t a = smem_u32(&ring_full[sl]);
-                const unsigned long long t0 = globaltimer();
-                while (!mbar_try_wait(a, rnd & 1u))
-                    if (globaltimer() - t0 > p.timeout_ns) break;
-            }
-        }
-        __syncwarp();
-    } else if (warp == kMmaWarp) {
+    } else if (warp == kRMmaWarp) {
         // ------------------------------------------------ weights + MMA issuer
         if (lane == 0) {
+            // Ring loader: rows go in order from the first tile's first row,
+            // row r to slot (r - first_row) mod kRing.  Once the producers
+            // are done with tile j, the rows below tile j + 1's first row are
+            // free, and the rows tile j + 2 needs are loaded.
+            const uint32_t row_tx = static_cast<uint32_t>(W * Cin * 2);
+            DwTilePos cur = dw_pos(p, tb);
+            const int first_row = tb < te ? dw_lo(p, cur) : 0;
+            int next_issue = first_row, is_slot = 0;
+            uint32_t is_round = 0;
+            auto load_rows = [&](int last, int free_below) {
+                while (next_issue <= last && next_issue - kRing < free_below) {
+                    mbar_arrive_expect_tx(&ring_full[is_slot], row_tx);
+                    bulk_load(ring + is_slot * p.row_bytes, p.x + static_cast<size_t>(next_issue) * W * Cin,
+                              row_tx, &ring_full[is_slot]);
+                    ++next_issue;
+                    if (++is_slot == kRing) {
+                        is_slot = 0;
+                        ++is_round;
+                    }
+                }
+            };
+            if (tb < te) {
+                DwTilePos nx = cur;
+                dw_advance(p, nx);
+                load_rows(tb + 1 < te ? dw_hi(p, nx) : dw_hi(p, cur), dw_lo(p, cur));
+            }
             bool ok = true;
             tma_prefetch_desc(&tmW);
             mbar_arrive_expect_tx(wbar, static_cast<uint32_t>(p.kb * p.nchunks * 8192));
@@ -732,13 +746,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                     acc = 0;
                     acc_phase ^= 1u;
                 }
+                if (tile + 1 < te) {
+                    DwTilePos n1 = cur;
+                    dw_advance(p, n1);
+                    DwTilePos n2 = n1;
+                    dw_advance(p, n2);
+                    load_rows(tile + 2 < te ? dw_hi(p, n2) : dw_hi(p, n1), dw_lo(p, n1));
+                }
+                dw_advance(p, cur);
+            }
+            // Let every row copy already issued land before the CTA can exit.
+            int sl = is_slot;
+            uint32_t rnd = is_round;
+            for (int i = 0; i < kRing && next_issue - 1 - i >= first_row; ++i) {
+                if (sl == 0) {
+                    sl = kRing - 1;
+                    --rnd;
+                } else {
+                    --sl;
+                }
+                const uint32_t a = smem_u32(&ring_full[sl]);
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(a, rnd & 1u))
+                    if (globaltimer() - t0 > p.timeout_ns) break;
             }
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------ epilogue (warps 9-12)
+        // ------------------------------------------------ epilogue (warps 13-16)
         const int q = warp & 3;
-        const int ew = warp - kEpiWarp0;
+        const int ew = warp - kREpiWarp0;
         uint8_t *stg = sStage + ew * (2 * 4096);
         int acc = 0, buf = 0;
         uint32_t acc_phase = 0;
@@ -756,20 +793,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             const long long row0 = (static_cast<long long>(n) * H + y0) * W + q * 32;
             const uint32_t tb_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                      static_cast<uint32_t>(acc * ncols);
+            // The TMEM load of chunk c + 32 is issued as soon as chunk c sits
+            // in the staging buffer, so its latency overlaps the store of c.
+            uint32_t r[32];
+            if (nv > 0) {
+                if (Cout >= 32)
+                    tmem_ld32(tb_addr, r);
+                else
+                    tmem_ld16(tb_addr, *reinterpret_cast<uint32_t (*)[16]>(&r[0]));
+            }
             for (int c = 0; c < Cout && nv > 0; c += 32) {
-                uint32_t r[32];
-                if (Cout - c >= 32) {
-                    tmem_ld32(tb_addr + c, r);
-                } else {
-                    uint32_t h[16];
-                    tmem_ld16(tb_addr + c, h);
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        r[i] = h[i];
-                        r[16 + i] = 0u;
-                    }
-                }
-                tmem_ld_wait();
+                tmem_ld_wait(r);
                 if (lane == 0) bulk_wait_read<1>();
                 __syncwarp();
                 uint8_t *sb = stg + buf * 4096;
@@ -778,6 +812,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int pos = ch ^ (lane & 7);
                     *reinterpret_cast<uint4 *>(sb + lane * 128 + pos * 16) =
                         make_uint4(r[4 * ch], r[4 * ch + 1], r[4 * ch + 2], r[4 * ch + 3]);
+                }
+                if (c + 32 < Cout) {
+                    if (Cout - c - 32 >= 32)
+                        tmem_ld32(tb_addr + c + 32, r);
+                    else
+                        tmem_ld16(tb_addr + c + 32, *reinterpret_cast<uint32_t (*)[16]>(&r[0]));
                 }
                 if (nv == 32) {
                     fence_proxy_async_smem();
@@ -830,7 +870,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     tc_fence_before();
     __syncthreads();
-    if (warp == kMmaWarp) {
+    if (warp == kRMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tmem_base, tmem_cols);
     }
@@ -853,7 +893,7 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: N*H*W too large");
     int rc;
     // Row-ring path: rt image rows per tile, 2 * rt + 2 rows resident.
-    int rt = (W <= kBM && kProd % (Cin / 4) == 0) ? kBM / W : 0;
+    int rt = (W <= kBM && kRProd % (Cin / 4) == 0) ? kBM / W : 0;
     if (rt > (kRingMax - 2) / 2) rt = (kRingMax - 2) / 2;
     while (rt > 1 && dw_row_layout(W, Cin, Cout, 2 * rt + 2).total > ds.max_smem_optin) --rt;
     const DwRowLayout RL = dw_row_layout(W, Cin, Cout, 2 * rt + 2);
@@ -894,7 +934,7 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
             rattr = true;
         }
         const int grid = q.tiles < ds.num_sms ? q.tiles : ds.num_sms;
-        dwsep_rows_kernel<<<grid, kThreads, RL.total, stream>>>(tmW, tmOut, tmOut16, tmOut8, q);
+        dwsep_rows_kernel<<<grid, kRThreads, RL.total, stream>>>(tmW, tmOut, tmOut16, tmOut8, q);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_error(e, "launch dwsep_rows_kernel");
         return ISAM_OK;
