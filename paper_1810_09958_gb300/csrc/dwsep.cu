@@ -18,6 +18,7 @@
 #include <cuda_bf16.h>
 
 #include <cstdio>
+#include <type_traits>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -444,49 +445,6 @@ __device__ __forceinline__ int dw_hi(const DwRowParams &p, DwTilePos t) {
     return t.n * p.H + min(p.H - 1, min(p.H, t.yt * p.rt + p.rt));
 }
 
-// The 3x3 depthwise sums of one vertical pixel pair (rows ya and ya + 1,
-// column x) for the 4 channels whose bf16 weights are in wb: acc0 for row ya,
-// acc1 for row ya + 1.  Input row ya - 1 + k is ring slot (slot0 + k) mod
-// kRing; pixels x - 1 and x + 1 may be the zero pad.  kCheckRows skips input
-// rows outside the image; tiles with no such row run the straight-line form.
-template <bool kCheckRows>
-__device__ __forceinline__ void dw_pair(const uint8_t *ring, int row_bytes, int kRing, int slot0, int ya,
-                                        int H, int x, int Cin2, int g, const uint32_t (&wb)[9][2],
-                                        float (&acc0)[4], float (&acc1)[4]) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        acc0[i] = 0.0f;
-        acc1[i] = 0.0f;
-    }
-    int slot = slot0;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int yy = ya - 1 + k;
-        if (!kCheckRows || (yy >= 0 && yy < H)) {
-            const uint8_t *rp = ring + slot * row_bytes + x * Cin2 + g * 8;
-#pragma unroll
-            for (int dj = 0; dj < 3; ++dj) {
-                const uint2 q = *reinterpret_cast<const uint2 *>(rp + (dj - 1) * Cin2);
-                if (k <= 2) {
-                    const uint32_t *wt = wb[k * 3 + dj];
-                    acc0[0] = fma_bf16_lo(q.x, wt[0], acc0[0]);
-                    acc0[1] = fma_bf16_hi(q.x, wt[0], acc0[1]);
-                    acc0[2] = fma_bf16_lo(q.y, wt[1], acc0[2]);
-                    acc0[3] = fma_bf16_hi(q.y, wt[1], acc0[3]);
-                }
-                if (k >= 1) {
-                    const uint32_t *wt = wb[(k - 1) * 3 + dj];
-                    acc1[0] = fma_bf16_lo(q.x, wt[0], acc1[0]);
-                    acc1[1] = fma_bf16_hi(q.x, wt[0], acc1[1]);
-                    acc1[2] = fma_bf16_lo(q.y, wt[1], acc1[2]);
-                    acc1[3] = fma_bf16_hi(q.y, wt[1], acc1[3]);
-                }
-            }
-        }
-        slot = (slot + 1 == kRing) ? 0 : slot + 1;
-    }
-}
-
 __global__ void __launch_bounds__(kRThreads, 1)
     dwsep_rows_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmOut,
                       const __grid_constant__ CUtensorMap tmOut16, const __grid_constant__ CUtensorMap tmOut8,
@@ -570,8 +528,13 @@ __global__ void __launch_bounds__(kRThreads, 1)
         // and here it would sit on the critical path of every tile.
         const int groups = Cin / 4;  // divides kRProd (Cin is 16, 32, ..., 256)
         const int g = tid % groups;
-        const int pi0 = tid / groups;
-        const int pstep = kRProd / groups;
+        // Column segment of this thread: the kRProd / groups segments split
+        // the W columns evenly (lengths differ by at most one).
+        const int nseg = kRProd / groups;
+        const int seg = tid / groups;
+        const int xs = (seg * W) / nseg;
+        const int xe = ((seg + 1) * W) / nseg;
+        const int seg_max = (W + nseg - 1) / nseg;
         uint32_t wb[9][2];  // bf16 weights of channels 4g..4g+3, two per word
 #pragma unroll
         for (int t = 0; t < 9; ++t) {
@@ -632,53 +595,99 @@ __global__ void __launch_bounds__(kRThreads, 1)
             // outside the image and never used).
             int s_top = lo_slot + (base_row + y0 - 1 - lo);
             if (s_top < 0) s_top += kRing;
-            // Each thread takes vertical pixel pairs (tile rows 2ry and
-            // 2ry + 1, column x): the pair reads 4 input rows x 3 columns,
-            // 12 taps for 2 outputs.  Every lane of a warp runs the same
-            // number of rounds and the __syncwarp at the end of a round
-            // rejoins the lanes.  Interior tiles run the tap loop without a
-            // branch, so all 12 loads can be in flight at once.
-            const int npairs = ((rows + 1) >> 1) * W;
-            // Every input row the tile reads lies inside the image.
+            // Each thread walks its column segment [xs, xe) of every pair of
+            // tile rows (2rp, 2rp + 1), keeping a 4-row x 3-column window of
+            // taps in registers: one new column (4 loads) per output pair.
+            // Every thread runs the same number of steps (the longest
+            // segment), so the lanes of a warp stay together; steps past the
+            // segment read a valid column and store nothing.  Interior tiles
+            // (every input row inside the image) run without row tests.
             const bool interior = y0 >= 1 && y1 + 1 <= H - 1;
-            int ry = 0, x = pi0;
-            while (x >= W) {
-                x -= W;
-                ++ry;
-            }
-            for (int pp0 = 0; pp0 < npairs; pp0 += pstep) {
-                const bool act = pp0 + pi0 < npairs;
-                const int ya = y0 + 2 * ry;
-                const bool two = act && (2 * ry + 1 < rows);
-                int slot = s_top + 2 * ry;  // input row ya - 1
-                while (slot >= kRing) slot -= kRing;
-                float acc0[4], acc1[4];
-                if (interior)
-                    dw_pair<false>(ring, p.row_bytes, kRing, slot, ya, H, x, Cin * 2, g, wb, acc0, acc1);
-                else
-                    dw_pair<true>(ring, p.row_bytes, kRing, slot, ya, H, x, Cin * 2, g, wb, acc0, acc1);
-                if (pp0 == 0) {
-                    // The A stage is free once the MMA of the previous tile is
-                    // done; the first round's taps are computed meanwhile.
-                    a_ok = __all_sync(0xffffffffu, bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY));
+            const int nrp = (rows + 1) >> 1;
+            auto run = [&](auto check_rows) {
+                constexpr bool kCheckRows = decltype(check_rows)::value;
+                for (int rp = 0; rp < nrp; ++rp) {
+                    const int ya = y0 + 2 * rp;
+                    const bool two = 2 * rp + 1 < rows;
+                    int sl = s_top + 2 * rp;  // input row ya - 1
+                    while (sl >= kRing) sl -= kRing;
+                    const uint8_t *rowp[4];
+                    bool rv[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        rowp[k] = ring + sl * p.row_bytes + g * 8;
+                        rv[k] = !kCheckRows || (ya - 1 + k >= 0 && ya - 1 + k < H);
+                        sl = (sl + 1 == kRing) ? 0 : sl + 1;
+                    }
+                    auto col = [&](int k, int xc) {
+                        uint2 q = *reinterpret_cast<const uint2 *>(rowp[k] + xc * (Cin * 2));
+                        if (kCheckRows && !rv[k]) q = make_uint2(0u, 0u);
+                        return q;
+                    };
+                    uint2 c0[4], c1[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        c0[k] = col(k, xs - 1);  // x = -1 reads the zero pad
+                        c1[k] = col(k, xs);
+                    }
+                    for (int st = 0; st < seg_max; ++st) {
+                        const int x = xs + st;
+                        const bool act = x < xe;
+                        uint2 c2[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) c2[k] = col(k, min(x + 1, W));  // x + 1 == W: zero pad
+                        float acc0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, acc1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+#pragma unroll
+                            for (int dj = 0; dj < 3; ++dj) {
+                                const uint2 q = dj == 0 ? c0[k] : (dj == 1 ? c1[k] : c2[k]);
+                                if (k <= 2) {
+                                    const uint32_t *wt = wb[k * 3 + dj];
+                                    acc0[0] = fma_bf16_lo(q.x, wt[0], acc0[0]);
+                                    acc0[1] = fma_bf16_hi(q.x, wt[0], acc0[1]);
+                                    acc0[2] = fma_bf16_lo(q.y, wt[1], acc0[2]);
+                                    acc0[3] = fma_bf16_hi(q.y, wt[1], acc0[3]);
+                                }
+                                if (k >= 1) {
+                                    const uint32_t *wt = wb[(k - 1) * 3 + dj];
+                                    acc1[0] = fma_bf16_lo(q.x, wt[0], acc1[0]);
+                                    acc1[1] = fma_bf16_hi(q.x, wt[0], acc1[1]);
+                                    acc1[2] = fma_bf16_lo(q.y, wt[1], acc1[2]);
+                                    acc1[3] = fma_bf16_hi(q.y, wt[1], acc1[3]);
+                                }
+                            }
+                        }
+                        if (rp == 0 && st == 0) {
+                            // The A stage is free once the MMA of the previous
+                            // tile is done; the first step is computed meanwhile.
+                            a_ok = __all_sync(0xffffffffu, bounded_wait(a_empty, a_phase ^ 1u, w, SITE_DW_AEMPTY));
+                        }
+                        if (act && a_ok) {
+                            const int pi = 2 * rp * W + x;
+                            const uint2 o = make_uint2(pack_bf16x2(acc0[0], acc0[1]), pack_bf16x2(acc0[2], acc0[3]));
+                            *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) +
+                                                       half) = o;
+                            if (two) {
+                                const int pj = pi + W;
+                                const uint2 o1 = make_uint2(pack_bf16x2(acc1[0], acc1[1]), pack_bf16x2(acc1[2], acc1[3]));
+                                *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pj * 128 + ((chunk ^ (pj & 7)) << 4) +
+                                                           half) = o1;
+                            }
+                        }
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            c0[k] = c1[k];
+                            c1[k] = c2[k];
+                        }
+                    }
+                    __syncwarp();
                 }
-                if (act && a_ok) {
-                    const int pi = 2 * ry * W + x;
-                    const uint2 o = make_uint2(pack_bf16x2(acc0[0], acc0[1]), pack_bf16x2(acc0[2], acc0[3]));
-                    *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) + half) = o;
-                }
-                if (two && a_ok) {
-                    const int pi = (2 * ry + 1) * W + x;
-                    const uint2 o = make_uint2(pack_bf16x2(acc1[0], acc1[1]), pack_bf16x2(acc1[2], acc1[3]));
-                    *reinterpret_cast<uint2 *>(sA + atom * (kBM * 128) + pi * 128 + ((chunk ^ (pi & 7)) << 4) + half) = o;
-                }
-                __syncwarp();
-                x += pstep;
-                while (x >= W) {
-                    x -= W;
-                    ++ry;
-                }
-            }
+            };
+            if (interior)
+                run(std::false_type{});
+            else
+                run(std::true_type{});
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(a_full);
