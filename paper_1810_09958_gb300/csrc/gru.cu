@@ -44,7 +44,10 @@ constexpr int kThreads = 128;
 constexpr int kAtomU = kRowsG * 128;     // one 64-wide K atom of the U slice (12 KB)
 constexpr int kAtomH = kBatchPad * 128;  // one K atom of h (4 KB)
 constexpr int kUPad = 32 * 128;          // the M = 128 MMA reads 32 rows past an atom
-constexpr int kRecvBytes = kRowsG * kBatchPad * 4;  // partial rows received per step (12 KB)
+// Partial rows received per step: 96 rows of 32 batch values, each row padded
+// to 36 floats so the 8 units a warp reads fall into different banks.
+constexpr int kRecvStride = kBatchPad + 4;
+constexpr int kRecvBytes = kRowsG * kRecvStride * 4;
 constexpr int kMaxPieces = 4;
 
 enum : uint32_t {
@@ -83,7 +86,12 @@ __device__ __forceinline__ void red_release_gpu_add(uint32_t *p, uint32_t v) {
     asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
-__device__ __forceinline__ float sigmoidf_fast(float v) { return 1.0f / (1.0f + __expf(-v)); }
+// Branch-free gate nonlinearities (a data-dependent branch in the gate code
+// would split warps for the rest of the step): __expf and the approximate
+// __fdividef, exact in the limits (exp overflow gives 0 and +-1).
+__device__ __forceinline__ float sigmoidf_fast(float v) { return __fdividef(1.0f, 1.0f + __expf(-v)); }
+// tanh(v) = 1 - 2 / (1 + e^{2v})
+__device__ __forceinline__ float tanhf_fast(float v) { return 1.0f - __fdividef(2.0f, 1.0f + __expf(2.0f * v)); }
 
 __device__ __forceinline__ uint16_t f32_to_bf16_rne(float f) {
     return __bfloat16_as_ushort(__float2bfloat16_rn(f));
@@ -159,7 +167,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(ubar, 1);
         for (int q = 0; q < kMaxPieces; ++q) mbar_init(&hbar[q], 1);
         mbar_init(mma_done, 1);
-        mbar_init(red_full, kRowsG);
+        mbar_init(red_full, 1);  // armed with the bytes of a step's partial rows
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -173,6 +181,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (KS > 1) cluster_sync_all();  // peers' barriers exist before any remote arrive
     tc_fence_after();
     const uint32_t tmem_d = *tmem_slot;
+    // Partial rows of one step for my units: KS sources x 3 gates x UO x 32.
+    const uint32_t recv_bytes = static_cast<uint32_t>(KS * 3 * UO * kBatchPad * 4);
+    if (tid == 0) mbar_arrive_expect_tx(red_full, recv_bytes);
 
     // ---- priming iteration: persistent weights and initial state.
     if (tid == 0) {
@@ -208,6 +219,25 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const uint32_t idesc = idesc_bf16_f32(128, kBatchPad, false, false);
     int issued_phase = -1;  // last step whose h loads were issued (for the drain)
+    // Input projection of a step (independent of h), loaded one step ahead so
+    // its memory latency is off the recurrence's critical path.
+    float gxr[kMaxPairs], gxz[kMaxPairs], gxn[kMaxPairs];
+    auto load_gx = [&](int tt) {
+#pragma unroll
+        for (int k = 0; k < kMaxPairs; ++k) {
+            const int b = tid / UO + k * bstep;
+            if (k < np && b < p.batch && tt < p.T) {
+                const float *g = p.gx + (static_cast<size_t>(tt) * p.batch + b) * G + j;
+                gxr[k] = __ldg(g);
+                gxz[k] = __ldg(g + H);
+                gxn[k] = __ldg(g + 2 * H);
+            } else {
+                gxr[k] = gxz[k] = gxn[k] = 0.0f;
+            }
+        }
+    };
+    load_gx(0);
+    int last_t = -1;  // step whose h (in hprev) still has to go to h_out
 
     // ---- recursive iteration, T times.
     for (int t = 0; t < p.T; ++t) {
@@ -224,20 +254,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         __syncwarp();
-        // Input projection of this step (independent of h): prefetch.
-        float gxr[kMaxPairs], gxz[kMaxPairs], gxn[kMaxPairs];
+        // Off thread 0's path to the next counter poll: h_{t-1} to h_out and
+        // this step's input projection (still ahead of its use in the gates).
+        if (last_t >= 0) {
 #pragma unroll
-        for (int k = 0; k < kMaxPairs; ++k) {
-            const int b = tid / UO + k * bstep;
-            if (k < np && b < p.batch) {
-                const float *g = p.gx + (static_cast<size_t>(t) * p.batch + b) * G + j;
-                gxr[k] = g[0];
-                gxz[k] = g[H];
-                gxn[k] = g[2 * H];
-            } else {
-                gxr[k] = gxz[k] = gxn[k] = 0.0f;
+            for (int k = 0; k < kMaxPairs; ++k) {
+                const int b = tid / UO + k * bstep;
+                if (k < np && b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
             }
+            last_t = -1;
         }
+        if (t > 0) load_gx(t);
         if (tid == 32 && ok) {
             for (int q = 0; q < p.nq && ok; ++q) {
                 if (!bounded_wait(&hbar[q], par, w, SITE_GRU_H)) {
@@ -270,13 +297,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t owner = static_cast<uint32_t>(lane / UO);
             const int oui = lane % UO;
             const uint32_t dst = mapa_shared(
-                smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kBatchPad), owner);
+                smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kRecvStride), owner);
+            const uint32_t rbar = mapa_shared(smem_u32(red_full), owner);
+            // Asynchronous remote stores: each counts its bytes on the owner's
+            // barrier, so nothing here waits for them to land.
 #pragma unroll
             for (int c = 0; c < 8; ++c)
-                st_dsmem_f4(dst + c * 16, make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
-                                                      __uint_as_float(r[4 * c + 2]),
-                                                      __uint_as_float(r[4 * c + 3])));
-            mbar_arrive_remote(red_full, owner);
+                st_async_f4(dst + c * 16,
+                            make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
+                                        __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
+                            rbar);
         }
         tc_fence_before();
         __syncwarp();
@@ -287,32 +317,42 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int b = tid / UO + k * bstep;
             if (k >= np || b >= p.batch) continue;
             float ghr = bh_r, ghz = bh_z, ghn = bh_n;
-            for (int s = 0; s < KS; ++s) {
-                const float *rs = recv + (s * 3 * UO + ui) * kBatchPad + b;
-                ghr += rs[0];
-                ghz += rs[UO * kBatchPad];
-                ghn += rs[2 * UO * kBatchPad];
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {  // KS <= 4 sources, summed in rank order
+                if (s < KS) {
+                    const float *rs = recv + (s * 3 * UO + ui) * kRecvStride + b;
+                    ghr += rs[0];
+                    ghz += rs[UO * kRecvStride];
+                    ghn += rs[2 * UO * kRecvStride];
+                }
             }
             const float rg = sigmoidf_fast(gxr[k] + ghr);
             const float zg = sigmoidf_fast(gxz[k] + ghz);
-            const float ng = tanhf(gxn[k] + rg * ghn);
+            const float ng = tanhf_fast(gxn[k] + rg * ghn);
             const float hn = (1.0f - zg) * ng + zg * hprev[k];
             hprev[k] = hn;
             hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
         }
+        last_t = t;  // hprev holds h_t, not yet in h_out
         // Publish first (the release then waits only for the exchange-buffer
         // stores), then write this step's h_t to h_out.
         fence_proxy_async_global();
         __syncthreads();
         if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
             red_release_gpu_add(p.counter, 1u);
+        // recv is consumed: arm the barrier for the next step's partial rows
+        // (bytes that land before this are counted all the same).
+        if (tid == 0) mbar_arrive_expect_tx(red_full, recv_bytes);
         __syncwarp();
+        tc_fence_after();
+    }
+    // h_T of the last step reached (or the step the loop left at).
+    if (last_t >= 0) {
 #pragma unroll
         for (int k = 0; k < kMaxPairs; ++k) {
             const int b = tid / UO + k * bstep;
-            if (k < np && b < p.batch) p.h_out[(static_cast<size_t>(t) * p.batch + b) * H + j] = hprev[k];
+            if (k < np && b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
         }
-        tc_fence_after();
     }
 
     // ---- teardown: let issued copies land, release TMEM.
@@ -327,6 +367,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
     tc_fence_before();
     __syncthreads();
+    // No CTA leaves while a cluster peer may still write into its shared
+    // memory (a peer that gave up on a wait can be behind by a step); every
+    // wait above is bounded, so every CTA gets here.
+    if (KS > 1) cluster_sync_all();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tmem_d, 32);
