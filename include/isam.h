@@ -146,9 +146,12 @@ int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta,
  * (h itself is carried in fp32).  Gates are evaluated in fp32.
  *
  * Supported: T >= 1, 1 <= batch <= 32, hidden a multiple of 64 in
- * [64, 1024] (hidden / 16 cooperating CTAs, launched cooperatively so they
- * are co-resident); all pointers 16-byte aligned.  Otherwise
- * ISAM_ERR_UNSUPPORTED.
+ * [64, 1024] except 960; all pointers 16-byte aligned.  Otherwise
+ * ISAM_ERR_UNSUPPORTED.  The recurrence runs on hidden / 32 clusters of 4, 2
+ * or 1 CTAs (4 when hidden is a multiple of 256, 2 for the other multiples of
+ * 128, else 1), launched cooperatively so they are co-resident; each CTA keeps
+ * a 96-row slice of U in shared memory, which for hidden = 960 (one CTA per
+ * cluster, 15 K atoms) does not fit.
  */
 int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
                      const isam_bf16 *W, const isam_bf16 *U, const float *b,
@@ -163,7 +166,8 @@ int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
  * because they can synchronise the whole device.
  *
  * Same arguments, layouts, equations and support limits as isam_gru_forward
- * (1 <= batch <= 32, hidden a multiple of 64 in [64, 1024], any T >= 1).  The
+ * (1 <= batch <= 32, hidden a multiple of 64 in [64, 1024] except 960, any
+ * T >= 1).  The
  * caller still passes every input and h_out.  The workspaces live in one
  * static 8 MiB device array inside libisam.so, which every GPU that loads the
  * library holds until the process exits; the input projection is computed in

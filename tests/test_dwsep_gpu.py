@@ -45,7 +45,12 @@ def test_dwsep_benchmark_layer_full_oracle():
 
 @pytest.mark.parametrize("shape", [(1, 1, 1, 16, 32), (1, 5, 7, 16, 16), (2, 9, 8, 32, 48),
                                    (3, 4, 33, 64, 96), (2, 13, 11, 128, 256), (1, 3, 130, 48, 16),
-                                   (1, 7, 19, 256, 64), (4, 2, 3, 80, 144)])
+                                   (1, 7, 19, 256, 64), (4, 2, 3, 80, 144),
+                                   # one-row tiles (65 <= W <= 128), exactly 128 pixels, full
+                                   # 2 x 64 tiles, many small images (tiles of several images
+                                   # per CTA), a 48-channel input (12 lanes per pixel)
+                                   (2, 6, 100, 32, 32), (1, 4, 128, 64, 128), (2, 10, 64, 128, 256),
+                                   (200, 3, 40, 64, 64), (3, 8, 24, 48, 80)])
 def test_dwsep_shapes(shape):
     N, H, W, Cin, Cout = shape
     x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=sum(shape) * 31 + Cin)

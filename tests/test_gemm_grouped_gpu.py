@@ -55,6 +55,21 @@ def test_grouped_integer_bit_exact_mixed_layouts():
         assert np.array_equal(got.astype(np.float64), ref), spec
 
 
+def test_grouped_64_problems_mixed():
+    """The largest group: 64 problems of varied shape, layout, alpha and beta."""
+    specs = []
+    for i in range(64):
+        M = 64 + 40 * (i % 7) + (i % 3)
+        N = 8 * (1 + i % 20)
+        K = 16 * (1 + (i * 5) % 23)
+        tA, tB = i % 2, (i // 2) % 2
+        if tA and M % 8:
+            M += 8 - M % 8
+        specs.append((M, N, K, tA, tB, 1.0 + 0.25 * (i % 3), 0.5 * (i % 2)))
+    for (got, ref), spec in zip(run_group(specs, seed0=900), specs):
+        assert nmax_err(got, ref) <= TOL, spec
+
+
 def test_grouped_single_problem_and_beta():
     specs = [(512, 96, 512, 1, 0, 1.5, -0.5)]
     (got, ref), = run_group(specs)

@@ -53,7 +53,9 @@ def test_gru_benchmark_shape_full_oracle():
 
 
 @pytest.mark.parametrize("T,batch,H", [(1, 1, 64), (5, 3, 64), (7, 17, 192), (9, 32, 128),
-                                       (20, 32, 512), (3, 31, 320), (16, 8, 1024)])
+                                       (20, 32, 512), (3, 31, 320), (16, 8, 1024),
+                                       # 3, 7 and 13 K atoms per CTA (4, 2 and 1 K splits)
+                                       (6, 32, 768), (4, 5, 896), (3, 2, 832)])
 def test_gru_shapes_with_initial_state(T, batch, H):
     x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 1000 + batch * 10 + H)
     h0 = synth.f32_uniform(T + batch + H, (batch, H))
@@ -109,6 +111,8 @@ def test_gru_unsupported_shapes_rejected():
     p = lambda t: ctypes.c_void_p(t.data_ptr())
     assert lib.isam_gru_forward(1, 33, 64, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
     assert lib.isam_gru_forward(1, 1, 96, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    # hidden 960: one CTA per cluster would need 15 K atoms of U (does not fit).
+    assert lib.isam_gru_forward(1, 1, 960, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
 
 
 def test_gru_missing_participant_times_out_cleanly():
