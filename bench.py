@@ -332,6 +332,30 @@ def hot_path_rows(isam, dev, peaks):
                               "frac_bf16_sustained": round(tf / peaks["bf16_tflops_sustained"], 4),
                               "plan": isam.gemm_plan(n, n, n, 0, 0, 1.0)}
     del A, B, C
+    # The skinny sweep's 16 (M, K) x N shapes on E4M3 operands (K-major A and
+    # B), one isam_gemm_fp8 launch each, replayed as a CUDA graph.
+    f8 = []
+    for (M, K) in SWEEP_MK:
+        for N_ in SWEEP_N:
+            seed = synth.stream_seed(synth.BASE_SEED, 7, M, K, N_)
+            f8.append((M, N_, K, synth.e4m3_uniform_torch(synth.stream_seed(seed, 1), M * K, dev),
+                       synth.e4m3_uniform_torch(synth.stream_seed(seed, 2), N_ * K, dev),
+                       torch.empty(M * N_, dtype=torch.float32, device=dev)))
+    run_f8 = lambda: [isam.gemm_fp8(M, N_, K, 1.0, A_, B_, 0.0, C_) for (M, N_, K, A_, B_, C_) in f8]
+    for _ in range(3):
+        run_f8()
+    isam.sync()
+    g8 = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g8):
+        run_f8()
+    ms = time_call(g8.replay, reps=50, warmup=3) / 1.0
+    fl = sum(gemm_flops(M, N_, K) for (M, N_, K, *_r) in f8)
+    by = sum(M * K + N_ * K + 4 * M * N_ for (M, N_, K, *_r) in f8)
+    out["gemm_fp8_sweep_16"] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
+                                "gbs": round(by / ms / 1e6, 1), "frac_hbm": round(by / ms / 1e6 / peaks["hbm_gbs"], 4),
+                                "what": "16 skinny shapes, E4M3 A (M x K) and B (N x K), fp32 C; "
+                                        "one isam_gemm_fp8 launch each (graph replay)"}
+    del f8, g8
     # GRU: hidden = input = 1024, batch 32, T = 128.
     T, batch, H = 128, 32, 1024
     s = 1.0 / 32.0

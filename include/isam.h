@@ -91,6 +91,24 @@ int isam_gemm(int M, int N, int K, int transA, int transB, float alpha,
               const isam_bf16 *A, const isam_bf16 *B, float beta, float *C);
 
 /*
+ * GEMM on 8-bit float operands: C <- alpha * A * B^T + beta * C with A (M x K)
+ * and B (N x K) stored row-major as OCP FP8 E4M3 bytes (1 sign bit, 4
+ * exponent bits with bias 7, 3 mantissa bits; 0x7F and 0xFF are NaN, no
+ * infinities, largest finite 448), C fp32 M x N row-major.  Products are
+ * exact and accumulate in fp32, as in isam_gemm; half the operand bytes of
+ * the bf16 call, for the bandwidth-bound skinny shapes.  The paper's
+ * instruction selection (Section 2.4) chooses among instructions a program
+ * maps onto; this is the same matrix multiplication on the tensor cores'
+ * 8-bit operand kind.
+ *   - Both operands K-major (the only layout); K a multiple of 16 (16-byte
+ *     rows); A, B, C 16-byte aligned.  Otherwise ISAM_ERR_UNSUPPORTED.
+ *   - Sizes < 1 or null pointers: ISAM_ERR_INVALID_ARG.
+ * Asynchronous on the stream set by isam_set_stream; beta = 0 does not read C.
+ */
+int isam_gemm_fp8(int M, int N, int K, float alpha, const uint8_t *A, const uint8_t *B, float beta,
+                  float *C);
+
+/*
  * Several independent GEMMs in one launch: problem i computes
  * C[i] <- alpha[i] * op(A[i]) * op(B[i]) + beta[i] * C[i] exactly as isam_gemm
  * would, with the same per-problem argument rules.

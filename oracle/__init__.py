@@ -52,6 +52,10 @@ def _load():
             lib.oracle_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
             lib.oracle_dwsep.argtypes = [i, i, i, i, i, P, P, P, P]
             lib.oracle_num_threads.argtypes = []
+            lib.oracle_e4m3.argtypes = [ctypes.c_uint8]
+            lib.oracle_e4m3.restype = ctypes.c_double
+            lib.oracle_gemm_fp8.argtypes = [i, i, i, d, P, P, d, P, P]
+            lib.oracle_gemm_fp8.restype = ctypes.c_int
             for f in (lib.oracle_gemm_rows, lib.oracle_gemm, lib.oracle_gru_forward,
                       lib.oracle_dwsep, lib.oracle_num_threads):
                 f.restype = ctypes.c_int
@@ -92,6 +96,27 @@ def gemm(M, N, K, transA, transB, alpha, A, B, beta=0.0, C_in=None, rows=None):
                                  _p(A), _p(B), float(beta), _p(C_in), _p(out))
     if rc != 0:
         raise ValueError("oracle_gemm: invalid argument")
+    return out
+
+
+def e4m3(byte: int) -> float:
+    """The value of one E4M3 byte (exact)."""
+    return _load().oracle_e4m3(int(byte) & 0xFF)
+
+
+def gemm_fp8(M, N, K, alpha, A, B, beta=0.0, C_in=None):
+    """C = alpha * A @ B^T + beta * C_in, A (M x K) and B (N x K) E4M3 bytes;
+    returns [M, N] float64."""
+    A = np.ascontiguousarray(A, dtype=np.uint8)
+    B = np.ascontiguousarray(B, dtype=np.uint8)
+    assert A.size == M * K and B.size == N * K
+    if C_in is not None:
+        C_in = np.ascontiguousarray(C_in, dtype=np.float32)
+        assert C_in.size == M * N
+    out = np.empty((M, N), dtype=np.float64)
+    rc = _load().oracle_gemm_fp8(M, N, K, float(alpha), _p(A), _p(B), float(beta), _p(C_in), _p(out))
+    if rc != 0:
+        raise ValueError("oracle_gemm_fp8: invalid argument")
     return out
 
 

@@ -94,6 +94,46 @@ int oracle_gemm_rows(int M, int N, int K, int transA, int transB, double alpha,
     return 0;
 }
 
+/*
+ * OCP FP8 E4M3 byte -> double, exactly: sign s, 4 exponent bits e (bias 7), 3
+ * mantissa bits m.  e > 0: (-1)^s 2^(e-7) (1 + m/8); e == 0: (-1)^s 2^-6 (m/8);
+ * e == 15 with m == 7 is NaN (the format has no infinities).
+ */
+double oracle_e4m3(uint8_t byte) {
+    const int s = byte >> 7, e = (byte >> 3) & 15, m = byte & 7;
+    double v;
+    if (e == 15 && m == 7)
+        v = NAN;
+    else if (e == 0)
+        v = ldexp((double)m / 8.0, -6);
+    else
+        v = ldexp(1.0 + (double)m / 8.0, e - 7);
+    return s ? -v : v;
+}
+
+/*
+ * C_out = alpha * A B^T + beta * C_in with A (M x K) and B (N x K) stored as
+ * E4M3 bytes, row-major: the GEMM of Listing 1 on 8-bit operands, each dot
+ * product summed in increasing k in double precision.
+ */
+int oracle_gemm_fp8(int M, int N, int K, double alpha, const uint8_t *A, const uint8_t *B, double beta,
+                    const float *C_in, double *C_out) {
+    if (M < 1 || N < 1 || K < 1 || !A || !B || !C_out) return 1;
+    if (beta != 0.0 && !C_in) return 1;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int i = 0; i < M; ++i) {
+        for (int j = 0; j < N; ++j) {
+            double acc = 0.0;
+            for (int k = 0; k < K; ++k)
+                acc += oracle_e4m3(A[(size_t)i * K + k]) * oracle_e4m3(B[(size_t)j * K + k]);
+            double v = alpha * acc;
+            if (beta != 0.0) v += beta * (double)C_in[(size_t)i * N + j];
+            C_out[(size_t)i * N + j] = v;
+        }
+    }
+    return 0;
+}
+
 int oracle_gemm(int M, int N, int K, int transA, int transB, double alpha,
                 const uint16_t *A, const uint16_t *B, double beta,
                 const float *C_in, double *C_out) {

@@ -157,6 +157,16 @@ int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64
     return encode(out, key, 2, base, dims, strides, box);
 }
 
+int make_tmap_2d_u8(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
+                    uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer) {
+    const uint64_t key[12] = {0x8, reinterpret_cast<uint64_t>(base), inner, outer, row_pitch_bytes,
+                              box_inner, box_outer, 0, 0, 0, 0, 0};
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_pitch_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    return encode(out, key, 2, base, dims, strides, box, CU_TENSOR_MAP_DATA_TYPE_UINT8);
+}
+
 int make_tmap_2d_f32(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
                      uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer) {
     const uint64_t key[12] = {0xF32, reinterpret_cast<uint64_t>(base), inner, outer,
@@ -250,6 +260,18 @@ int isam_shutdown(void) {
 int isam_gemm(int M, int N, int K, int transA, int transB, float alpha, const isam_bf16 *A,
               const isam_bf16 *B, float beta, float *C) {
     GemmDesc g{M, N, K, transA, transB, alpha, beta, A, B, C, nullptr};
+    int rc = gemm_validate(g);
+    if (rc) return rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    GemmPlan plan;
+    if ((rc = gemm_plan(g, *ds, &plan))) return rc;
+    return gemm_launch(g, plan, *ds, current_stream());
+}
+
+int isam_gemm_fp8(int M, int N, int K, float alpha, const uint8_t *A, const uint8_t *B, float beta, float *C) {
+    GemmDesc g{M, N, K, 0, 1, alpha, beta, reinterpret_cast<const uint16_t *>(A),
+               reinterpret_cast<const uint16_t *>(B), C, nullptr, 1};
     int rc = gemm_validate(g);
     if (rc) return rc;
     DeviceState *ds = device_state(&rc);

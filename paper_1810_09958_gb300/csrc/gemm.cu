@@ -85,7 +85,10 @@ __device__ __forceinline__ void tile_coords(int tile, int m_tiles, int n_tiles, 
     nt = local / gm;
 }
 
-template <int BN, bool A_MN, bool B_MN>
+// F8: E4M3 operands (K-major A and B only): a 128-byte K atom holds 128
+// elements instead of 64; everything else -- tiles, stages, swizzle, epilogue
+// -- is byte-for-byte the bf16 kernel.
+template <int BN, bool A_MN, bool B_MN, bool F8 = false>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const GemmParams p) {
@@ -166,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kg_pf = min(kg_end, kg_begin + ST);
         for (int kg = kg_begin; kg < kg_pf; ++kg)
             for (int at = 0; at < KA; ++at) {
-                const int k0 = (kg * KA + at) * kBK;
+                const int k0 = (kg * KA + at) * (F8 ? 2 * kBK : kBK);  // in elements
                 if (A_MN) {
                     tma_prefetch_l2_2d(&tmA, mt * kBM, k0);
                     tma_prefetch_l2_2d(&tmA, mt * kBM + 64, k0);
@@ -202,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     uint8_t *a = sA + static_cast<size_t>(stage) * a_stage;
                     uint8_t *b = sB + static_cast<size_t>(stage) * b_stage;
                     for (int at = 0; at < KA; ++at) {
-                        const int k0 = (kg * KA + at) * kBK;
+                        const int k0 = (kg * KA + at) * (F8 ? 2 * kBK : kBK);  // in elements
                         uint8_t *aa = a + at * kABytes;
                         uint8_t *bb = b + at * C::kBAtom;
                         if (A_MN) {
@@ -244,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
-            const uint32_t idesc = idesc_bf16_f32(kBM, BN, A_MN, B_MN);
+            const uint32_t idesc = F8 ? idesc_e4m3_f32(kBM, BN) : idesc_bf16_f32(kBM, BN, A_MN, B_MN);
             int stage = 0;
             uint32_t phase = 0;
             int acc = 0;
@@ -271,7 +274,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                      : sdesc_sw128(aa + k * 32, 16, 1024);
                             const uint64_t bd = B_MN ? sdesc_sw128(bb + k * 2048, 8192, 1024)
                                                      : sdesc_sw128(bb + k * 32, 16, 1024);
-                            umma_bf16(d, ad, bd, idesc, (kg > kg_begin || at > 0 || k > 0) ? 1u : 0u);
+                            if constexpr (F8)
+                                umma_f8(d, ad, bd, idesc, (kg > kg_begin || at > 0 || k > 0) ? 1u : 0u);
+                            else
+                                umma_bf16(d, ad, bd, idesc, (kg > kg_begin || at > 0 || k > 0) ? 1u : 0u);
                         }
                     }
                     umma_commit(&empty[stage]);
@@ -579,6 +585,17 @@ KernelFn pick3(bool a_mn, bool b_mn) {
     return b_mn ? gemm_tc_kernel<BN, false, true> : gemm_tc_kernel<BN, false, false>;
 }
 
+KernelFn pick_kernel_f8(int BN) {
+    switch (BN) {
+        case 16: return gemm_tc_kernel<16, false, false, true>;
+        case 32: return gemm_tc_kernel<32, false, false, true>;
+        case 64: return gemm_tc_kernel<64, false, false, true>;
+        case 128: return gemm_tc_kernel<128, false, false, true>;
+        case 256: return gemm_tc_kernel<256, false, false, true>;
+        default: return nullptr;
+    }
+}
+
 KernelFn pick_kernel(int BN, bool a_mn, bool b_mn) {
     switch (BN) {
         case 16: return pick3<16>(a_mn, b_mn);
@@ -624,7 +641,8 @@ double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out)
     const int m_tiles = ceil_div(g.M, kBM);
     const int n_tiles = ceil_div(g.N, BN);
     const long long tiles = static_cast<long long>(m_tiles) * n_tiles;
-    const int kb = ceil_div(g.K, kBK);
+    const int eb = g.fp8 ? 1 : 2;                  // bytes per operand element
+    const int kb = ceil_div(g.K, kBK * 2 / eb);     // 128-byte K atoms
     const int kb_per = ceil_div(kb, S);
     const int clusters_max = std::max(1, num_sms / S);
     const int clusters = static_cast<int>(std::min<long long>(tiles, clusters_max));
@@ -639,9 +657,9 @@ double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out)
     const double t_unit = std::max(t_mma, t_load) + kTileOverheadUs;
     const double t_steady = tiles_per_cluster * t_unit;
     const double out_bytes = 4.0 * g.M * g.N * (g.beta != 0.0f ? 2.0 : 1.0);
-    const double uniq = 2.0 * g.M * g.K + 2.0 * g.K * g.N + out_bytes;
+    const double uniq = eb * (static_cast<double>(g.M) * g.K + static_cast<double>(g.K) * g.N) + out_bytes;
     const double t_hbm = uniq / kHbmBw * 1e6;
-    const double t_flops = 2.0 * g.M * g.N * g.K / kPeakFlops * 1e6;
+    const double t_flops = 2.0 * g.M * g.N * g.K / (kPeakFlops * (g.fp8 ? 2.0 : 1.0)) * 1e6;
     const double tail = (S > 1 ? kSplitTailUs : 0.0) + kBM * BN * 4.0 / S / kSmStoreBw * 1e6;
     return kFirstDataUs + std::max({t_steady, t_hbm, t_flops}) + tail + kLaunchGapUs;
 }
@@ -687,6 +705,14 @@ int gemm_validate(const GemmDesc &g) {
     if ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B) |
          reinterpret_cast<uintptr_t>(g.C)) & 15u)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: A, B and C must be 16-byte aligned");
+    if (g.fp8) {
+        if (g.transA != 0 || g.transB != 1)
+            return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm_fp8: A and B must both be K-major");
+        if (g.K % 16 != 0)
+            return set_error(ISAM_ERR_UNSUPPORTED,
+                             "isam_gemm_fp8: K (%d) must be a multiple of 16 (16-byte rows)", g.K);
+        return ISAM_OK;
+    }
     const int a_pitch = g.transA ? g.M : g.K;
     const int b_pitch = g.transB ? g.K : g.N;
     if (a_pitch % 8 != 0 || b_pitch % 8 != 0)
@@ -700,7 +726,7 @@ int gemm_validate(const GemmDesc &g) {
 int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
     const bool b_mn = g.transB == 0;
     const int nsm = ds.num_sms;
-    const int kb = ceil_div(g.K, kBK);
+    const int kb = ceil_div(g.K, g.fp8 ? 2 * kBK : kBK);
     double best = 1e300;
     GemmPlan bp{};
     const int bns[] = {16, 32, 64, 128, 256};
@@ -753,17 +779,25 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
     CUtensorMap ta, tb, tc;
     memset(&tc, 0, sizeof tc);
     int rc;
-    if (a_mn)
-        rc = make_tmap_2d_bf16(&ta, g.A, g.M, g.K, static_cast<uint64_t>(g.M) * 2, 64, 64);
-    else
-        rc = make_tmap_2d_bf16(&ta, g.A, g.K, g.M, static_cast<uint64_t>(g.K) * 2, 64, kBM);
-    if (rc) return rc;
-    if (b_mn)
-        rc = make_tmap_2d_bf16(&tb, g.B, g.N, g.K, static_cast<uint64_t>(g.N) * 2, 64, 64);
-    else
-        rc = make_tmap_2d_bf16(&tb, g.B, g.K, g.N, static_cast<uint64_t>(g.K) * 2, 64,
-                               static_cast<uint32_t>(plan.BN));
-    if (rc) return rc;
+    if (g.fp8) {
+        // 128-element (128-byte) K atoms of both K-major operands.
+        if ((rc = make_tmap_2d_u8(&ta, g.A, g.K, g.M, static_cast<uint64_t>(g.K), 128, kBM))) return rc;
+        if ((rc = make_tmap_2d_u8(&tb, g.B, g.K, g.N, static_cast<uint64_t>(g.K), 128,
+                                  static_cast<uint32_t>(plan.BN))))
+            return rc;
+    } else {
+        if (a_mn)
+            rc = make_tmap_2d_bf16(&ta, g.A, g.M, g.K, static_cast<uint64_t>(g.M) * 2, 64, 64);
+        else
+            rc = make_tmap_2d_bf16(&ta, g.A, g.K, g.M, static_cast<uint64_t>(g.K) * 2, 64, kBM);
+        if (rc) return rc;
+        if (b_mn)
+            rc = make_tmap_2d_bf16(&tb, g.B, g.N, g.K, static_cast<uint64_t>(g.N) * 2, 64, 64);
+        else
+            rc = make_tmap_2d_bf16(&tb, g.B, g.K, g.N, static_cast<uint64_t>(g.K) * 2, 64,
+                                   static_cast<uint32_t>(plan.BN));
+        if (rc) return rc;
+    }
     // The epilogue moves C with TMA when rows are 16-byte aligned (N % 4 == 0)
     // and the tile is at least one 32-column chunk wide.
     const int tma_c = (g.N % 4 == 0 && plan.BN >= 32 && plan.split == 1) ? 1 : 0;
@@ -776,7 +810,7 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
     p.K = g.K;
     p.m_tiles = ceil_div(g.M, kBM);
     p.n_tiles = ceil_div(g.N, plan.BN);
-    p.kb_total = ceil_div(g.K, kBK);
+    p.kb_total = ceil_div(g.K, g.fp8 ? 2 * kBK : kBK);
     p.ka = plan.ka;
     p.kg_total = ceil_div(p.kb_total, plan.ka);
     p.tma_c = tma_c;
@@ -791,7 +825,7 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
     p.timeout_ns = wait_timeout_ns();
     p.err = ds.err_word;
 
-    KernelFn fn = pick_kernel(plan.BN, a_mn, b_mn);
+    KernelFn fn = g.fp8 ? pick_kernel_f8(plan.BN) : pick_kernel(plan.BN, a_mn, b_mn);
     if (!fn) return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: no kernel for BN=%d", plan.BN);
     if ((rc = ensure_smem_attr(fn, plan.smem))) return rc;
 

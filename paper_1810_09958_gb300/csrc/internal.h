@@ -42,6 +42,9 @@ int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64
                       uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
 int make_tmap_2d_f32(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
                      uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
+// Same for 8-bit elements (E4M3 operands), 128-byte swizzle.
+int make_tmap_2d_u8(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,
+                    uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
 int make_tmap_3d_bf16(CUtensorMap *out, const void *base, const uint64_t dims[3],
                       const uint64_t strides_bytes[2], const uint32_t box[3]);
 
@@ -54,6 +57,7 @@ struct GemmDesc {
     const uint16_t *B;
     float *C;
     const float *bias_n;
+    int fp8 = 0;  // A and B are E4M3 bytes (A: M x K, B: N x K, both K-major)
 };
 
 // Tile plan chosen by the cost model (or forced through ISAM_FORCE_TILE).

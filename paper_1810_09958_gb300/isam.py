@@ -57,10 +57,11 @@ def load():
         lib.isam_gemm.argtypes = [i, i, i, i, i, f, P, P, f, P]
         lib.isam_gemm_plan_info.argtypes = [i, i, i, i, i, f, P]
         lib.isam_gemm_grouped.argtypes = [i, P, P, P, P, P, P, P, P, P, P]
+        lib.isam_gemm_fp8.argtypes = [i, i, i, f, P, P, f, P]
         lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
-                     "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gru_forward",
+                     "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gru_forward",
                      "isam_dwsep_conv"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
@@ -117,6 +118,20 @@ def gemm(M, N, K, transA, transB, alpha, A, B, beta, C) -> None:
     _use_current_stream(lib)
     check(lib.isam_gemm(M, N, K, int(transA), int(transB), float(alpha), _ptr(A), _ptr(B),
                         float(beta), _ptr(C)))
+
+
+def gemm_fp8(M, N, K, alpha, A, B, beta, C) -> None:
+    """isam_gemm_fp8: C = alpha A B^T + beta C (A: M x K, B: N x K, E4M3 bytes as
+    torch.uint8 or torch.float8_e4m3fn; C fp32)."""
+    import torch
+    lib = load()
+    for t, n, name in ((A, M * K, "A"), (B, N * K, "B")):
+        if t.dtype not in (torch.uint8, getattr(torch, "float8_e4m3fn", torch.uint8)):
+            raise ValueError(f"{name} must hold E4M3 bytes (uint8 or float8_e4m3fn), got {t.dtype}")
+        _dev(t, t.dtype, n, name)
+    _dev(C, torch.float32, M * N, "C")
+    _use_current_stream(lib)
+    check(lib.isam_gemm_fp8(M, N, K, float(alpha), _ptr(A), _ptr(B), float(beta), _ptr(C)))
 
 
 class GroupedGemm:

@@ -106,6 +106,58 @@ def as_torch_bf16(bits: np.ndarray):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
 
 
+def _e4m3_positive():
+    """Positive finite OCP E4M3 codes 0x00..0x7E and their values, ascending."""
+    codes = np.arange(0x7F, dtype=np.int64)
+    e, m = codes >> 3, codes & 7
+    vals = np.where(e == 0, (m / 8.0) * 2.0 ** -6, (1.0 + m / 8.0) * np.exp2(e - 7.0))
+    return codes, vals
+
+
+_E4M3_CODES, _E4M3_VALS = _e4m3_positive()
+
+
+def to_e4m3_bits(x: np.ndarray) -> np.ndarray:
+    """float -> E4M3 byte, round to nearest (ties to the even code), magnitudes
+    above 448 saturate to 448; zero encodes as 0x00."""
+    x = np.asarray(x, dtype=np.float64)
+    a = np.minimum(np.abs(x), 448.0)
+    idx = np.clip(np.searchsorted(_E4M3_VALS, a), 1, len(_E4M3_VALS) - 1)
+    lo, hi = _E4M3_VALS[idx - 1], _E4M3_VALS[idx]
+    up = (a - lo > hi - a) | ((a - lo == hi - a) & ((_E4M3_CODES[idx] & 1) == 0))
+    code = np.where(up, _E4M3_CODES[idx], _E4M3_CODES[idx - 1])
+    code = np.where(a == 0.0, 0, code)
+    sign = np.where(np.signbit(x) & (code != 0), 0x80, 0)
+    return (code | sign).astype(np.uint8)
+
+
+def e4m3_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """E4M3 byte -> float64 (finite codes; NaN codes give NaN)."""
+    b = np.asarray(bits, dtype=np.int64)
+    mag = _E4M3_VALS[np.minimum(b & 0x7F, 0x7E)]
+    mag = np.where((b & 0x7F) == 0x7F, np.nan, mag)
+    return np.where(b & 0x80, -mag, mag)
+
+
+def e4m3_uniform(seed: int, shape, lo=-1.0, hi=1.0) -> np.ndarray:
+    n = int(np.prod(shape))
+    return to_e4m3_bits(uniform(seed, n, lo, hi)).reshape(shape)
+
+
+def e4m3_integers(seed: int, shape, lo: int, hi: int) -> np.ndarray:
+    """Integers in [lo, hi] (exact in E4M3 for |v| <= 16)."""
+    n = int(np.prod(shape))
+    return to_e4m3_bits(integers(seed, n, lo, hi).astype(np.float64)).reshape(shape)
+
+
+def e4m3_uniform_torch(seed: int, n: int, device, lo=-1.0, hi=1.0):
+    """Device-side E4M3 bytes (torch.uint8) for large benchmark operands: the
+    same uniform stream rounded to E4M3 by torch's float8 cast."""
+    import torch
+    f = f32_uniform_torch(seed, n, device, lo, hi)
+    return f.to(torch.float8_e4m3fn).view(torch.uint8)
+
+
 def bf16_uniform(seed: int, shape, lo=-1.0, hi=1.0) -> np.ndarray:
     n = int(np.prod(shape))
     return to_bf16_bits(uniform(seed, n, lo, hi)).reshape(shape)

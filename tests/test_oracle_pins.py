@@ -311,3 +311,53 @@ def test_uniform_at_matches_stream():
     full = synth.uniform(seed, 5000)
     idx = np.array([[0, 4999, 17], [2500, 3, 3]])
     assert np.array_equal(synth.uniform_at(seed, idx), full[idx])
+
+
+# --------------------------------------------------------------------------- E4M3 (8-bit) GEMM
+
+def test_e4m3_decode_known_values(oracle_lib):
+    """Values fixed by the OCP E4M3 definition (bias 7, 3 mantissa bits, no
+    infinities, S.1111.111 is NaN)."""
+    known = {0x00: 0.0, 0x01: 2.0 ** -9, 0x07: 7 * 2.0 ** -9, 0x08: 2.0 ** -6, 0x38: 1.0, 0x3C: 1.5,
+             0x40: 2.0, 0x7E: 448.0, 0xB8: -1.0, 0xFE: -448.0, 0x30: 0.5, 0x48: 4.0, 0x59: 18.0}
+    for byte, v in known.items():
+        assert oracle_lib.e4m3(byte) == v, hex(byte)
+    assert math.isnan(oracle_lib.e4m3(0x7F)) and math.isnan(oracle_lib.e4m3(0xFF))
+
+
+def test_e4m3_decode_matches_float32_construction(oracle_lib):
+    """Every normal code equals the float32 with the same sign, exponent
+    (rebiased 7 -> 127) and mantissa (shifted to the top); subnormals m * 2^-9."""
+    import struct
+    for byte in range(256):
+        s, e, m = byte >> 7, (byte >> 3) & 15, byte & 7
+        if e == 15 and m == 7:
+            continue
+        if e == 0:
+            v = m * 2.0 ** -9
+        else:
+            v = struct.unpack("<f", struct.pack("<I", (e - 7 + 127) << 23 | m << 20))[0]
+        assert oracle_lib.e4m3(byte) == (-v if s else v), hex(byte)
+
+
+def test_e4m3_gemm_integer_exact_and_alpha_beta(oracle_lib):
+    """Integer inputs (exact in E4M3) against int64 matmul, with alpha = 2,
+    beta = -1: every product and partial sum is an exact integer."""
+    rng = np.random.default_rng(8)
+    M, N, K = 9, 7, 48
+    Ai = rng.integers(-4, 5, (M, K))
+    Bi = rng.integers(-4, 5, (N, K))
+    Ci = rng.integers(-8, 9, (M, N)).astype(np.float32)
+    A8, B8 = synth.to_e4m3_bits(Ai.astype(float)), synth.to_e4m3_bits(Bi.astype(float))
+    got = oracle_lib.gemm_fp8(M, N, K, 2.0, A8, B8, -1.0, Ci)
+    assert np.array_equal(got, 2.0 * (Ai @ Bi.T) - Ci)
+
+
+def test_e4m3_rounding_of_inputs(oracle_lib):
+    """The input generator rounds to nearest with ties to the even code and
+    saturates at 448; every finite code round-trips."""
+    assert list(synth.to_e4m3_bits(np.array([1.0625, 1.1875, 1000.0, -1.0, 2.0 ** -10]))) == [
+        0x38, 0x3A, 0x7E, 0xB8, 0x00]
+    codes = np.array([c for c in range(256) if (c & 0x7F) != 0x7F and c != 0x80], dtype=np.uint8)
+    vals = np.array([oracle_lib.e4m3(c) for c in codes])
+    assert np.array_equal(synth.to_e4m3_bits(vals), codes)
