@@ -355,7 +355,20 @@ def hot_path_rows(isam, dev, peaks):
                                 "gbs": round(by / ms / 1e6, 1), "frac_hbm": round(by / ms / 1e6 / peaks["hbm_gbs"], 4),
                                 "what": "16 skinny shapes, E4M3 A (M x K) and B (N x K), fp32 C; "
                                         "one isam_gemm_fp8 launch each (graph replay)"}
-    del f8, g8
+    # The same 16 problems as one isam_gemm_grouped_fp8 launch.
+    gcall = isam.GroupedGemmFp8([(M, N_, K, 1.0, A_, B_, 0.0, C_) for (M, N_, K, A_, B_, C_) in f8])
+    for _ in range(3):
+        gcall()
+    isam.sync()
+    gg = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gg):
+        gcall()
+    ms = time_call(gg.replay, reps=50, warmup=3)
+    out["gemm_fp8_grouped_16"] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
+                                  "gbs": round(by / ms / 1e6, 1),
+                                  "frac_hbm": round(by / ms / 1e6 / peaks["hbm_gbs"], 4),
+                                  "what": "the same 16 E4M3 problems in one isam_gemm_grouped_fp8 launch"}
+    del f8, g8, gg, gcall
     # GRU: hidden = input = 1024, batch 32, T = 128.
     T, batch, H = 128, 32, 1024
     s = 1.0 / 32.0

@@ -129,6 +129,17 @@ int isam_gemm_grouped(int count, const int *M, const int *N, const int *K, const
                       const isam_bf16 *const *B, const float *beta, float *const *C);
 
 /*
+ * isam_gemm_grouped for E4M3 problems: problem i computes
+ * C[i] <- alpha[i] * A[i] * B[i]^T + beta[i] * C[i] exactly as isam_gemm_fp8
+ * would (A[i]: M[i] x K[i], B[i]: N[i] x K[i], E4M3 bytes, K-major), with the
+ * same argument rules per problem and the same group rules as
+ * isam_gemm_grouped (1 <= count <= 64, host arrays, no overlapping C).
+ */
+int isam_gemm_grouped_fp8(int count, const int *M, const int *N, const int *K, const float *alpha,
+                          const uint8_t *const *A, const uint8_t *const *B, const float *beta,
+                          float *const *C);
+
+/*
  * The tile plan isam_gemm would use for this problem, chosen by the
  * library's analytic cost model (the paper's "Approach" interface for
  * tiling and device-allocation choices, Sections 3.4 and 4).  Nothing is

@@ -304,6 +304,29 @@ int isam_gemm_grouped(int count, const int *M, const int *N, const int *K, const
     return gemm_grouped_launch(count, g, *ds, current_stream());
 }
 
+int isam_gemm_grouped_fp8(int count, const int *M, const int *N, const int *K, const float *alpha,
+                          const uint8_t *const *A, const uint8_t *const *B, const float *beta, float *const *C) {
+    if (count < 1 || count > 64)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped_fp8: count must be in [1, 64]");
+    if (!M || !N || !K || !alpha || !A || !B || !beta || !C)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped_fp8: null array");
+    GemmDesc g[64];
+    for (int i = 0; i < count; ++i) {
+        g[i] = GemmDesc{M[i], N[i], K[i], 0, 1, alpha[i], beta[i], reinterpret_cast<const uint16_t *>(A[i]),
+                        reinterpret_cast<const uint16_t *>(B[i]), C[i], nullptr, 1};
+        int rc = gemm_validate(g[i]);
+        if (rc) {
+            char msg[512];
+            snprintf(msg, sizeof msg, "isam_gemm_grouped_fp8: problem %d: %s", i, isam_last_error_string());
+            return set_error(rc, "%s", msg);
+        }
+    }
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gemm_grouped_launch(count, g, *ds, current_stream());
+}
+
 // Reports the tile plan the cost model picks for a GEMM (for benchmarks and
 // tests; nothing is launched).  out[0..5] = BN, split, stages, group_m, grid,
 // shared-memory bytes.

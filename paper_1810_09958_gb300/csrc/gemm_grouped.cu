@@ -49,6 +49,7 @@ struct GroupProblem {
     int M, N, K;
     int m_tiles, n_tiles, kb_total;
     int a_mn, b_mn, bn;
+    int fp8;          // E4M3 operands (both K-major): 128-element K atoms
     int tma_c;        // C rows 16-byte aligned: TMA epilogue
     int tile_start;   // first global tile index of this problem
     float alpha, beta;
@@ -139,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                     mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(kAStage) + bbytes);
                     uint8_t *a = sA + static_cast<size_t>(stage) * kAStage;
                     uint8_t *b = sB + static_cast<size_t>(stage) * kBStage;
-                    const int k0 = kb * kBK;
+                    const int k0 = kb * (pr.fp8 ? 2 * kBK : kBK);  // in elements
                     if (pr.a_mn) {
                         tma_load_2d(&p.tmA[pi], &full[stage], a, mt * kBM, k0);
                         tma_load_2d(&p.tmA[pi], &full[stage], a + 8192, mt * kBM + 64, k0);
@@ -181,7 +182,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < p.total_tiles; tile += gridDim.x) {
                 const GroupProblem &pr = p.prob[find_problem(p, tile)];
-                const uint32_t idesc = idesc_bf16_f32(kBM, pr.bn, pr.a_mn != 0, pr.b_mn != 0);
+                const bool f8 = pr.fp8 != 0;
+                const uint32_t idesc =
+                    f8 ? idesc_e4m3_f32(kBM, pr.bn) : idesc_bf16_f32(kBM, pr.bn, pr.a_mn != 0, pr.b_mn != 0);
                 if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_G_TEMPTY)) break;
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(acc * kBNMax);
@@ -199,7 +202,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                                                     : sdesc_sw128(a0 + k * 32, 16, 1024);
                         const uint64_t bd = pr.b_mn ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
                                                     : sdesc_sw128(b0 + k * 32, 16, 1024);
-                        umma_bf16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                        if (f8)
+                            umma_f8(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                        else
+                            umma_bf16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
                     }
                     umma_commit(&empty[stage]);
                     if (++stage == ST) {
@@ -373,7 +379,8 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
     // round-robin walk over tiles ends with the cheap ones.
     int order[kMaxGroup];
     std::iota(order, order + count, 0);
-    std::stable_sort(order, order + count, [&](int a, int b) { return g[a].K > g[b].K; });
+    auto atoms = [&](int i) { return (g[i].K + (g[i].fp8 ? 2 * kBK : kBK) - 1) / (g[i].fp8 ? 2 * kBK : kBK); };
+    std::stable_sort(order, order + count, [&](int a, int b) { return atoms(a) > atoms(b); });
 
     static GroupParams p;  // ~29 KB: built under the lock, copied into the launch
     std::lock_guard<std::mutex> lk(g_group_mu);
@@ -386,12 +393,13 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
         pr.M = d.M;
         pr.N = d.N;
         pr.K = d.K;
-        pr.a_mn = d.transA;
-        pr.b_mn = d.transB == 0 ? 1 : 0;
+        pr.fp8 = d.fp8;
+        pr.a_mn = d.fp8 ? 0 : d.transA;
+        pr.b_mn = (d.fp8 || d.transB == 1) ? 0 : 1;
         pr.bn = std::min(kBNMax, (d.N + 15) / 16 * 16);
         pr.m_tiles = (d.M + kBM - 1) / kBM;
         pr.n_tiles = (d.N + pr.bn - 1) / pr.bn;
-        pr.kb_total = (d.K + kBK - 1) / kBK;
+        pr.kb_total = atoms(order[s]);
         pr.tma_c = (d.N % 4 == 0) ? 1 : 0;
         pr.tile_start = tiles;
         pr.alpha = d.alpha;
@@ -399,17 +407,25 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
         pr.C = d.C;
         tiles += pr.m_tiles * pr.n_tiles;
         int rc;
-        if (pr.a_mn)
-            rc = make_tmap_2d_bf16(&p.tmA[s], d.A, d.M, d.K, static_cast<uint64_t>(d.M) * 2, 64, 64);
-        else
-            rc = make_tmap_2d_bf16(&p.tmA[s], d.A, d.K, d.M, static_cast<uint64_t>(d.K) * 2, 64, kBM);
-        if (rc) return rc;
-        if (pr.b_mn)
-            rc = make_tmap_2d_bf16(&p.tmB[s], d.B, d.N, d.K, static_cast<uint64_t>(d.N) * 2, 64, 64);
-        else
-            rc = make_tmap_2d_bf16(&p.tmB[s], d.B, d.K, d.N, static_cast<uint64_t>(d.K) * 2, 64,
-                                   static_cast<uint32_t>(pr.bn));
-        if (rc) return rc;
+        if (pr.fp8) {
+            // 128-element (128-byte) K atoms of both K-major E4M3 operands.
+            if ((rc = make_tmap_2d_u8(&p.tmA[s], d.A, d.K, d.M, static_cast<uint64_t>(d.K), 128, kBM))) return rc;
+            if ((rc = make_tmap_2d_u8(&p.tmB[s], d.B, d.K, d.N, static_cast<uint64_t>(d.K), 128,
+                                      static_cast<uint32_t>(pr.bn))))
+                return rc;
+        } else {
+            if (pr.a_mn)
+                rc = make_tmap_2d_bf16(&p.tmA[s], d.A, d.M, d.K, static_cast<uint64_t>(d.M) * 2, 64, 64);
+            else
+                rc = make_tmap_2d_bf16(&p.tmA[s], d.A, d.K, d.M, static_cast<uint64_t>(d.K) * 2, 64, kBM);
+            if (rc) return rc;
+            if (pr.b_mn)
+                rc = make_tmap_2d_bf16(&p.tmB[s], d.B, d.N, d.K, static_cast<uint64_t>(d.N) * 2, 64, 64);
+            else
+                rc = make_tmap_2d_bf16(&p.tmB[s], d.B, d.K, d.N, static_cast<uint64_t>(d.K) * 2, 64,
+                                       static_cast<uint32_t>(pr.bn));
+            if (rc) return rc;
+        }
         if (pr.tma_c &&
             (rc = make_tmap_2d_f32(&p.tmC[s], d.C, d.N, d.M, static_cast<uint64_t>(d.N) * 4, 32, 32)))
             return rc;

@@ -58,10 +58,12 @@ def load():
         lib.isam_gemm_plan_info.argtypes = [i, i, i, i, i, f, P]
         lib.isam_gemm_grouped.argtypes = [i, P, P, P, P, P, P, P, P, P, P]
         lib.isam_gemm_fp8.argtypes = [i, i, i, f, P, P, f, P]
+        lib.isam_gemm_grouped_fp8.argtypes = [i, P, P, P, P, P, P, P, P]
         lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
-                     "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gru_forward",
+                     "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
+                     "isam_gru_forward",
                      "isam_dwsep_conv"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
@@ -158,6 +160,31 @@ class GroupedGemm:
         lib = load()
         _use_current_stream(lib)
         check(lib.isam_gemm_grouped(self.n, *self.args))
+
+
+class GroupedGemmFp8:
+    """Marshalled arguments of one isam_gemm_grouped_fp8 call over a list of
+    (M, N, K, alpha, A, B, beta, C); A, B E4M3 bytes (uint8 / float8_e4m3fn)."""
+
+    def __init__(self, problems):
+        import torch
+        n = len(problems)
+        ia = lambda vals: (ctypes.c_int * n)(*vals)
+        fa = lambda vals: (ctypes.c_float * n)(*vals)
+        pa = lambda vals: (ctypes.c_void_p * n)(*vals)
+        for (M, N, K, alpha, A, B, beta, C) in problems:
+            _dev(A, A.dtype, M * K, "A")
+            _dev(B, B.dtype, N * K, "B")
+            _dev(C, torch.float32, M * N, "C")
+        cols = list(zip(*problems))
+        self.n = n
+        self.args = (ia(cols[0]), ia(cols[1]), ia(cols[2]), fa(cols[3]), pa([t.data_ptr() for t in cols[4]]),
+                     pa([t.data_ptr() for t in cols[5]]), fa(cols[6]), pa([t.data_ptr() for t in cols[7]]))
+
+    def __call__(self):
+        lib = load()
+        _use_current_stream(lib)
+        check(lib.isam_gemm_grouped_fp8(self.n, *self.args))
 
 
 def gemm_grouped(problems) -> None:

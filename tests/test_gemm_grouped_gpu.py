@@ -86,3 +86,46 @@ def test_grouped_names_the_bad_problem():
                            (8, 8, 12, 0, 0, 1.0, z, z, 0.0, c[:64])])
     assert e.value.code == isam.ISAM_ERR_UNSUPPORTED
     assert "problem 1" in str(e.value)
+
+
+def dev_u8(bits):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(bits).reshape(-1)).to("cuda")
+
+
+def run_group_fp8(specs, dist="uniform", seed0=700):
+    """specs: (M, N, K, alpha, beta); E4M3 A (M x K) and B (N x K)."""
+    probs, keep = [], []
+    for i, (M, N, K, alpha, beta) in enumerate(specs):
+        if dist == "int":
+            A = synth.e4m3_integers(seed0 + 3 * i, (M, K), -4, 4)
+            B = synth.e4m3_integers(seed0 + 3 * i + 1, (N, K), -4, 4)
+            C0 = synth.integers(seed0 + 3 * i + 2, M * N, -8, 8).astype(np.float32).reshape(M, N)
+        else:
+            A = synth.e4m3_uniform(seed0 + 3 * i, (M, K))
+            B = synth.e4m3_uniform(seed0 + 3 * i + 1, (N, K))
+            C0 = synth.f32_uniform(seed0 + 3 * i + 2, (M, N))
+        out = Guarded(M * N, init=C0)
+        probs.append((M, N, K, alpha, dev_u8(A), dev_u8(B), beta, out.t))
+        keep.append((A, B, C0, out))
+    isam.GroupedGemmFp8(probs)()
+    isam.sync()
+    res = []
+    for (M, N, K, alpha, beta), (A, B, C0, out) in zip(specs, keep):
+        assert out.guards_intact()
+        res.append((out.numpy().reshape(M, N), oracle.gemm_fp8(M, N, K, alpha, A, B, beta, C0)))
+    return res
+
+
+def test_grouped_fp8_skinny_shapes():
+    specs = [(M, N, K, 1.0, 0.0) for (M, K) in [(1760, 1760), (2560, 2560), (4096, 4096), (7680, 2560)]
+             for N in (16, 32, 64, 128)]
+    for (got, ref), spec in zip(run_group_fp8(specs), specs):
+        assert nmax_err(got, ref) <= TOL, spec
+
+
+def test_grouped_fp8_integer_bit_exact_ragged():
+    specs = [(328, 200, 1168, 2.0, -1.0), (200, 13, 144, 1.0, 0.5), (136, 48, 80, 1.0, 0.0),
+             (1, 8, 16, 1.0, 0.0), (257, 129, 1008, 1.0, -2.0)]
+    for (got, ref), spec in zip(run_group_fp8(specs, dist="int"), specs):
+        assert np.array_equal(got.astype(np.float64), ref), spec
