@@ -55,6 +55,8 @@ def _load():
             lib.oracle_e4m3.argtypes = [ctypes.c_uint8]
             lib.oracle_e4m3.restype = ctypes.c_double
             lib.oracle_gemm_fp8.argtypes = [i, i, i, d, P, P, d, P, P]
+            lib.oracle_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
+            lib.oracle_gru_forward_reset_before.restype = ctypes.c_int
             lib.oracle_gemm_fp8.restype = ctypes.c_int
             for f in (lib.oracle_gemm_rows, lib.oracle_gemm, lib.oracle_gru_forward,
                       lib.oracle_dwsep, lib.oracle_num_threads):
@@ -120,8 +122,9 @@ def gemm_fp8(M, N, K, alpha, A, B, beta=0.0, C_in=None):
     return out
 
 
-def gru_forward(x, W, U, b, h0=None):
-    """All T hidden states [T, batch, H] float64 of the GRU (r, z, n gate order)."""
+def gru_forward(x, W, U, b, h0=None, reset_before=False):
+    """All T hidden states [T, batch, H] float64 of the GRU (r, z, n gate order);
+    reset_before: the candidate's recurrent input is U_n (r * h)."""
     x, W, U = _u16(x), _u16(W), _u16(U)
     T, batch, H = x.shape
     assert W.shape == (3 * H, H) and U.shape == (3 * H, H)
@@ -131,7 +134,8 @@ def gru_forward(x, W, U, b, h0=None):
         h0 = np.ascontiguousarray(h0, dtype=np.float32)
         assert h0.size == batch * H
     out = np.empty((T, batch, H), dtype=np.float64)
-    rc = _load().oracle_gru_forward(T, batch, H, _p(x), _p(W), _p(U), _p(b), _p(h0), _p(out))
+    fn = _load().oracle_gru_forward_reset_before if reset_before else _load().oracle_gru_forward
+    rc = fn(T, batch, H, _p(x), _p(W), _p(U), _p(b), _p(h0), _p(out))
     if rc != 0:
         raise ValueError("oracle_gru_forward: invalid argument")
     return out

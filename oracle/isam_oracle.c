@@ -203,6 +203,66 @@ int oracle_gru_forward(int T, int batch, int H, const uint16_t *x, const uint16_
 }
 
 /*
+ * The GRU with the reset gate applied before the candidate's recurrent
+ * product (the cell's original form): the candidate sees U_n (r * h_{t-1}),
+ * so r must be known for every unit before that product:
+ *
+ *   r  = sigmoid(W_r x_t + b_ir + U_r h_{t-1} + b_hr)
+ *   z  = sigmoid(W_z x_t + b_iz + U_z h_{t-1} + b_hz)
+ *   n  = tanh(W_n x_t + b_in + U_n (r * h_{t-1}) + b_hn)
+ *   h_t = (1 - z) * n + z * h_{t-1}
+ *
+ * Same arguments and layouts as oracle_gru_forward.
+ */
+int oracle_gru_forward_reset_before(int T, int batch, int H, const uint16_t *x, const uint16_t *W,
+                                    const uint16_t *U, const float *b, const float *h0, double *h_out) {
+    if (T < 1 || batch < 1 || H < 1 || !x || !W || !U || !b || !h_out) return 1;
+    const int G = 3 * H;
+#pragma omp parallel
+    {
+        double *h = (double *)malloc(sizeof(double) * (size_t)H);
+        double *rh = (double *)malloc(sizeof(double) * (size_t)H);
+        double *z = (double *)malloc(sizeof(double) * (size_t)H);
+        double *gx = (double *)malloc(sizeof(double) * (size_t)G);
+#pragma omp for schedule(dynamic, 1)
+        for (int s = 0; s < batch; ++s) {
+            for (int j = 0; j < H; ++j) h[j] = h0 ? (double)h0[(size_t)s * H + j] : 0.0;
+            for (int t = 0; t < T; ++t) {
+                const uint16_t *xt = x + ((size_t)t * batch + s) * H;
+                for (int g = 0; g < G; ++g) {
+                    double ax = 0.0;
+                    const uint16_t *wr = W + (size_t)g * H;
+                    for (int k = 0; k < H; ++k) ax += bf(wr[k]) * bf(xt[k]);
+                    gx[g] = ax + (double)b[g];
+                }
+                for (int j = 0; j < H; ++j) {  /* r and z from h_{t-1} */
+                    double ar = 0.0, az = 0.0;
+                    const uint16_t *ur = U + (size_t)j * H, *uz = U + (size_t)(H + j) * H;
+                    for (int k = 0; k < H; ++k) {
+                        ar += bf(ur[k]) * h[k];
+                        az += bf(uz[k]) * h[k];
+                    }
+                    const double r = sigmoid(gx[j] + ar + (double)b[G + j]);
+                    z[j] = sigmoid(gx[H + j] + az + (double)b[G + H + j]);
+                    rh[j] = r * h[j];
+                }
+                double *ho = h_out + ((size_t)t * batch + s) * H;
+                for (int j = 0; j < H; ++j) {  /* candidate from r * h_{t-1} */
+                    double an = 0.0;
+                    const uint16_t *un = U + (size_t)(2 * H + j) * H;
+                    for (int k = 0; k < H; ++k) an += bf(un[k]) * rh[k];
+                    const double n = tanh(gx[2 * H + j] + an + (double)b[G + 2 * H + j]);
+                    ho[j] = (1.0 - z[j]) * n + z[j] * h[j];
+                }
+                for (int j = 0; j < H; ++j) h[j] = ho[j];
+            }
+        }
+        free(h); free(rh); free(z); free(gx);
+    }
+    return 0;
+}
+
+/*
  * Separable depthwise convolution, Listing 3, with stride s = 1, channel
  * multiplier c = 1 (so r = 0 and P is indexed P[q][k]) and a zero border of
  * one pixel (input row i + di - 1, column j + dj - 1), taken in the factored

@@ -361,3 +361,71 @@ def test_e4m3_rounding_of_inputs(oracle_lib):
     codes = np.array([c for c in range(256) if (c & 0x7F) != 0x7F and c != 0x80], dtype=np.uint8)
     vals = np.array([oracle_lib.e4m3(c) for c in codes])
     assert np.array_equal(synth.to_e4m3_bits(vals), codes)
+
+
+# --------------------------------------------------------------------------- GRU, reset before the product
+
+def _gru_rb_python(x, W, U, b, h0):
+    """The reset-before equations in plain Python floats (tiny shapes)."""
+    T, B, H = x.shape
+    out = np.zeros((T, B, H))
+    for s in range(B):
+        h = [float(v) for v in h0[s]]
+        for t in range(T):
+            xt = x[t, s]
+            gx = [sum(W[g, k] * xt[k] for k in range(H)) + b[g] for g in range(3 * H)]
+            sig = lambda v: 1.0 / (1.0 + math.exp(-v))
+            r = [sig(gx[j] + sum(U[j, k] * h[k] for k in range(H)) + b[3 * H + j]) for j in range(H)]
+            z = [sig(gx[H + j] + sum(U[H + j, k] * h[k] for k in range(H)) + b[4 * H + j]) for j in range(H)]
+            rh = [r[k] * h[k] for k in range(H)]
+            n = [math.tanh(gx[2 * H + j] + sum(U[2 * H + j, k] * rh[k] for k in range(H)) + b[5 * H + j])
+                 for j in range(H)]
+            h = [(1 - z[j]) * n[j] + z[j] * h[j] for j in range(H)]
+            out[t, s] = h
+    return out
+
+
+def test_gru_reset_before_matches_python_loops(oracle_lib):
+    T, B, H = 3, 2, 4
+    x, W, U, b, _ = synth.gru_operands(T, B, H, seed=41)
+    h0 = synth.f32_uniform(42, (B, H))
+    got = oracle_lib.gru_forward(x, W, U, b, h0, reset_before=True)
+    ref = _gru_rb_python(f64(x), f64(W), f64(U), b.astype(np.float64), h0.astype(np.float64))
+    assert np.max(np.abs(got - ref)) < 1e-12
+
+
+def test_gru_reset_before_zero_weights_closed_form(oracle_lib):
+    """W = U = 0: constant gates, n = tanh(b_in + b_hn), h_t = n (1 - z^t) + z^t h0."""
+    T, B, H = 6, 3, 8
+    x = synth.bf16_normal(43, (T, B, H))
+    Z = np.zeros((3 * H, H), dtype=np.uint16)
+    b = synth.f32_uniform(44, 6 * H, -0.5, 0.5).astype(np.float32)
+    h0 = synth.f32_uniform(45, (B, H))
+    got = oracle_lib.gru_forward(x, Z, Z, b, h0, reset_before=True)
+    bb = b.astype(np.float64)
+    z = 1 / (1 + np.exp(-(bb[H:2 * H] + bb[4 * H:5 * H])))
+    n = np.tanh(bb[2 * H:3 * H] + bb[5 * H:])
+    for t in range(T):
+        assert np.max(np.abs(got[t] - (n * (1 - z ** (t + 1)) + z ** (t + 1) * h0))) < 1e-12
+
+
+def test_gru_reset_before_saturated_reset_gate(oracle_lib):
+    """r = 1 (b_ir = +30): U_n (r h) = r (U_n h), so both GRU forms agree; r = 0
+    (b_ir = -30) with b_hn = 0: U_n no longer matters, and the form equals the
+    reset-after one with the n rows of U zeroed."""
+    T, B, H = 4, 3, 16
+    x, W, U, b, _ = synth.gru_operands(T, B, H, seed=46)
+    h0 = synth.f32_uniform(47, (B, H))
+    b1 = b.copy()
+    b1[:H] = 30.0
+    a = oracle_lib.gru_forward(x, W, U, b1, h0, reset_before=True)
+    c = oracle_lib.gru_forward(x, W, U, b1, h0)
+    assert np.max(np.abs(a - c)) < 1e-10
+    b0 = b.copy()
+    b0[:H] = -30.0
+    b0[5 * H:] = 0.0
+    U0 = U.copy()
+    U0[2 * H:] = 0
+    a = oracle_lib.gru_forward(x, W, U, b0, h0, reset_before=True)
+    c = oracle_lib.gru_forward(x, W, U0, b0, h0)
+    assert np.max(np.abs(a - c)) < 1e-10
