@@ -385,6 +385,15 @@ def hot_path_rows(isam, dev, peaks):
     out["gru_h1024_b32_t128"] = {"ms": round(ms, 4), "timesteps_per_s": round(T / (ms / 1e3), 1),
                                  "us_per_step": round(ms * 1e3 / T, 3), "tflops": round(tf, 2),
                                  "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4)}
+    # The same GRU with the reset gate applied before the candidate's product
+    # (two exchange rounds per step).
+    ms = time_call(lambda: isam.gru_forward(T, batch, H, x, W, U, b, h0, hout, reset_before=True),
+                   reps=10, warmup=3, flush=flush)
+    tf = gflop / ms
+    out["gru_reset_before_h1024_b32_t128"] = {
+        "ms": round(ms, 4), "timesteps_per_s": round(T / (ms / 1e3), 1),
+        "us_per_step": round(ms * 1e3 / T, 3), "tflops": round(tf, 2),
+        "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4)}
     del x, W, U, b, h0, hout
     # Separable depthwise layer.
     N, Hh, Ww, Cin, Cout = 32, 56, 56, 128, 256
@@ -505,7 +514,8 @@ def reference_arm(args):
 def run_case(args):
     """Times one hot-path call on its own (for profiling and sweeps):
     sweep (the 32 sweep GEMMs in one grouped call) | gemm:M,N,K,transA,transB,beta |
-    gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]."""
+    gru[:T,batch,hidden] | gru_rb[:T,batch,hidden] (reset gate before the candidate's
+    product) | dwsep[:N,H,W,Cin,Cout]."""
     import torch
     from paper_1810_09958_gb300 import build, isam, synth
     torch.cuda.set_device(0)
@@ -532,7 +542,7 @@ def run_case(args):
         fn = call
         work = {"tflops": sum(p["flops"] for p in probs) / 1e12,
                 "gb": sum(p["bytes"] for p in probs) / 1e9}
-    elif kind == "gru":
+    elif kind in ("gru", "gru_rb"):
         T, batch, H = (int(v) for v in vals) if vals else (128, 32, 1024)
         s = H ** -0.5
         x = synth.bf16_normal_torch(21, T * batch * H, dev)
@@ -540,7 +550,8 @@ def run_case(args):
         U = synth.bf16_uniform_torch(23, 3 * H * H, dev, -s, s)
         b = synth.f32_uniform_torch(24, 6 * H, dev, -0.1, 0.1)
         hout = torch.empty(T * batch * H, dtype=torch.float32, device=dev)
-        fn = lambda: isam.gru_forward(T, batch, H, x, W, U, b, None, hout)
+        rb = kind == "gru_rb"
+        fn = lambda: isam.gru_forward(T, batch, H, x, W, U, b, None, hout, reset_before=rb)
         work = {"tflops": 2.0 * T * batch * 3 * H * 2 * H / 1e12, "timesteps": T}
     elif kind == "dwsep":
         N, H, W, Cin, Cout = (int(v) for v in vals) if vals else (32, 56, 56, 128, 256)
@@ -579,7 +590,7 @@ def main(argv=None):
     ap.add_argument("--no-hot-path", action="store_true")
     ap.add_argument("--case", default=None,
                     help="time one call instead of the benchmark: sweep (grouped) | gemm:M,N,K,tA,tB,beta | "
-                         "gru[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]")
+                         "gru[:T,batch,hidden] | gru_rb[:T,batch,hidden] | dwsep[:N,H,W,Cin,Cout]")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3

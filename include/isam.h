@@ -187,6 +187,24 @@ int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
                      const float *h0, float *h_out);
 
 /*
+ * GRU forward with the reset gate applied before the candidate's recurrent
+ * product (the cell's original form):
+ *
+ *   r = sigmoid(gx_r + U_r h_{t-1} + b_hr),  z = sigmoid(gx_z + U_z h_{t-1} + b_hz)
+ *   n = tanh(gx_n + U_n (r * h_{t-1}) + b_hn),  h_t = (1 - z) * n + z * h_{t-1}
+ *
+ * (gx = W x_t + b_ih as in isam_gru_forward.)  Same arguments, layouts and
+ * support limits as isam_gru_forward.  The recurrent product is no longer one
+ * fused 3H-wide product per step: U_n needs r of every unit first, so each
+ * step of the persistent kernel runs two rounds (r and z from h_{t-1}, a
+ * grid-wide exchange of bf16(r * h_{t-1}), then the n rows), the recurrent
+ * scheduling of Section 3.6 with an intra-step dependency.
+ */
+int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 *x,
+                                  const isam_bf16 *W, const isam_bf16 *U, const float *b,
+                                  const float *h0, float *h_out);
+
+/*
  * GRU forward that allocates nothing.  The paper has no counterpart: this is a
  * deployment variant of isam_gru_forward for callers that cannot let a library
  * call cudaMalloc -- a process whose device memory is all reserved up front by

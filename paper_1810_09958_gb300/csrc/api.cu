@@ -361,6 +361,18 @@ int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x, const isa
     return gru_launch(T, batch, hidden, x, W, U, b, h0, h_out, *ds, current_stream());
 }
 
+int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 *x, const isam_bf16 *W,
+                                  const isam_bf16 *U, const float *b, const float *h0, float *h_out) {
+    if (T < 1 || batch < 1 || hidden < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_reset_before: sizes must be >= 1");
+    if (!x || !W || !U || !b || !h_out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_reset_before: null pointer");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gru_launch(T, batch, hidden, x, W, U, b, h0, h_out, *ds, current_stream(), 1);
+}
+
 int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
                     const isam_bf16 *dw_w, const isam_bf16 *pw_w, float *out) {
     if (N < 1 || H < 1 || W < 1 || Cin < 1 || Cout < 1)

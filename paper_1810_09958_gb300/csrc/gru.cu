@@ -69,7 +69,9 @@ struct GruParams {
     const float *b_hh;         // [3H]
     const float *h0;           // [batch][H] or null
     float *h_out;              // [T][batch][H]
-    uint16_t *hx;              // [2][32][H] bf16 exchange
+    uint16_t *hx;              // [2][32][H] bf16 exchange of h
+    uint16_t *rhx;             // [2][32][H] bf16 exchange of r * h (reset_before)
+    int reset_before;          // candidate's recurrent input U_n (r * h): two rounds per step
     uint32_t *counter;         // step counter (zeroed before launch)
     int skip_publish_cta;      // debug: this CTA never publishes (-1: none)
     unsigned long long timeout_ns;
@@ -132,7 +134,9 @@ constexpr int kMaxPairs = 8;  // (unit, batch) pairs per thread when one CTA own
 __global__ void __launch_bounds__(kThreads, 1)
     gru_recurrent_kernel(const __grid_constant__ CUtensorMap tmU,
                          const __grid_constant__ CUtensorMap tmH0,
-                         const __grid_constant__ CUtensorMap tmH1, const GruParams p) {
+                         const __grid_constant__ CUtensorMap tmH1,
+                         const __grid_constant__ CUtensorMap tmR0,
+                         const __grid_constant__ CUtensorMap tmR1, const GruParams p) {
     if (!launch_shape_ok(p.err, static_cast<uint32_t>(p.ks), static_cast<uint32_t>(p.n_cta), 0x3F0u))
         return;
     extern __shared__ uint8_t smem_raw[];
@@ -181,15 +185,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (KS > 1) cluster_sync_all();  // peers' barriers exist before any remote arrive
     tc_fence_after();
     const uint32_t tmem_d = *tmem_slot;
-    // Partial rows of one step for my units: KS sources x 3 gates x UO x 32.
-    const uint32_t recv_bytes = static_cast<uint32_t>(KS * 3 * UO * kBatchPad * 4);
-    if (tid == 0) mbar_arrive_expect_tx(red_full, recv_bytes);
+    // A step is one round (all three gates' rows from h_{t-1}) or, with the
+    // reset gate before the product, two: round 0 takes the r and z rows from
+    // h_{t-1} and publishes r * h_{t-1}; round 1 takes the n rows from it.
+    // Partial rows of a round for my units: KS sources x gates x UO x 32.
+    const bool RB = p.reset_before != 0;
+    const int nph = RB ? 2 : 1;
+    auto round_bytes = [&](int ph) {
+        return static_cast<uint32_t>(KS * (RB ? (ph == 0 ? 2 : 1) : 3) * UO * kBatchPad * 4);
+    };
+    if (tid == 0) mbar_arrive_expect_tx(red_full, round_bytes(0));
 
     // ---- priming iteration: persistent weights and initial state.
     if (tid == 0) {
         tma_prefetch_desc(&tmU);
         tma_prefetch_desc(&tmH0);
         tma_prefetch_desc(&tmH1);
+        if (RB) {
+            tma_prefetch_desc(&tmR0);
+            tma_prefetch_desc(&tmR1);
+        }
         mbar_arrive_expect_tx(ubar, static_cast<uint32_t>(p.ka * kAtomU));
         for (int a = 0; a < p.ka; ++a)
             tma_load_3d(&tmU, ubar, sU + a * kAtomU, (atom0 + a) * 64, unit0, 0);
@@ -218,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
 
     const uint32_t idesc = idesc_bf16_f32(128, kBatchPad, false, false);
-    int issued_phase = -1;  // last step whose h loads were issued (for the drain)
+    int issued_phase = -1;  // last round whose h loads were issued (for the drain)
     // Input projection of a step (independent of h), loaded one step ahead so
     // its memory latency is off the recurrence's critical path.
     float gxr[kMaxPairs], gxz[kMaxPairs], gxn[kMaxPairs];
@@ -239,112 +254,144 @@ __global__ void __launch_bounds__(kThreads, 1)
     load_gx(0);
     int last_t = -1;  // step whose h (in hprev) still has to go to h_out
 
-    // ---- recursive iteration, T times.
-    for (int t = 0; t < p.T; ++t) {
-        const uint32_t par = static_cast<uint32_t>(t & 1);
-        if (tid == 0 && !*abort_flag) {
-            if (wait_counter(p.counter, static_cast<uint32_t>((t + 1) * p.n_cta), w)) {
-                fence_proxy_async_global();
-                const CUtensorMap *m = (t & 1) ? &tmH1 : &tmH0;
-                for (int q = 0; q < p.nq; ++q) {
-                    mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(p.qk * kAtomH));
-                    tma_load_3d(m, &hbar[q], sH + q * p.qk * kAtomH, 0, 0, atom0 + q * p.qk);
+    // ---- recursive iteration, T times (in nph rounds each).
+    float zsave[kMaxPairs];  // update gate between the two rounds of a step
+    bool alive = true;
+    for (int t = 0; t < p.T && alive; ++t) {
+        for (int ph = 0; ph < nph; ++ph) {
+            const int round = t * nph + ph;
+            const uint32_t par = static_cast<uint32_t>(round & 1);
+            if (tid == 0 && !*abort_flag) {
+                if (wait_counter(p.counter, static_cast<uint32_t>((round + 1) * p.n_cta), w)) {
+                    fence_proxy_async_global();
+                    const CUtensorMap *m = ph == 0 ? ((t & 1) ? &tmH1 : &tmH0) : ((t & 1) ? &tmR1 : &tmR0);
+                    for (int q = 0; q < p.nq; ++q) {
+                        mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(p.qk * kAtomH));
+                        tma_load_3d(m, &hbar[q], sH + q * p.qk * kAtomH, 0, 0, atom0 + q * p.qk);
+                    }
+                    issued_phase = round;
                 }
-                issued_phase = t;
             }
-        }
-        __syncwarp();
-        // Off thread 0's path to the next counter poll: h_{t-1} to h_out and
-        // this step's input projection (still ahead of its use in the gates).
-        if (last_t >= 0) {
+            __syncwarp();
+            if (ph == 0) {
+                // Off thread 0's path to the next counter poll: h_{t-1} to
+                // h_out and this step's input projection (still ahead of its
+                // use in the gates).
+                if (last_t >= 0) {
+#pragma unroll
+                    for (int k = 0; k < kMaxPairs; ++k) {
+                        const int b = tid / UO + k * bstep;
+                        if (k < np && b < p.batch)
+                            p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
+                    }
+                    last_t = -1;
+                }
+                if (t > 0) load_gx(t);
+            }
+            if (tid == 32 && ok) {
+                for (int q = 0; q < p.nq && ok; ++q) {
+                    if (!bounded_wait(&hbar[q], par, w, SITE_GRU_H)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int a = q * p.qk; a < (q + 1) * p.qk; ++a) {
+                        const uint32_t ua = smem_u32(sU + a * kAtomU);
+                        const uint32_t ha = smem_u32(sH + a * kAtomH);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k)
+                            umma_bf16(tmem_d, sdesc_sw128(ua + k * 32, 16, 1024),
+                                      sdesc_sw128(ha + k * 32, 16, 1024), idesc,
+                                      (a > 0 || k > 0) ? 1u : 0u);
+                    }
+                }
+                if (ok) umma_commit(mma_done);
+            }
+            __syncwarp();
+            // Block-uniform decision: every thread leaves at the same round.
+            if (!__syncthreads_and(bounded_wait(mma_done, par, w, SITE_GRU_MMA) ? 1 : 0)) {
+                alive = false;
+                break;
+            }
+            tc_fence_after();
+            // Push: row gate*32 + u of the partial product (TMEM lane = row)
+            // goes to the cluster CTA that owns unit u, into its slot for this
+            // source rank.  Round 0 of a reset-before step sends the r and z
+            // rows, round 1 the n rows.
+            const bool pushes = RB ? (ph == 0 ? warp < 2 : warp == 2) : warp < 3;
+            if (pushes) {
+                uint32_t r[32];
+                tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
+                tmem_ld_wait();
+                const uint32_t owner = static_cast<uint32_t>(lane / UO);
+                const int oui = lane % UO;
+                const uint32_t dst = mapa_shared(
+                    smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kRecvStride), owner);
+                const uint32_t rbar = mapa_shared(smem_u32(red_full), owner);
+                // Asynchronous remote stores: each counts its bytes on the
+                // owner's barrier, so nothing here waits for them to land.
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    st_async_f4(dst + c * 16,
+                                make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
+                                            __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
+                                rbar);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (!__syncthreads_and(bounded_wait<true>(red_full, par, w, SITE_GRU_RED) ? 1 : 0)) {
+                alive = false;
+                break;
+            }
+            uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
+            uint16_t *rhx_t = p.rhx + static_cast<size_t>(t & 1) * kBatchPad * H;
 #pragma unroll
             for (int k = 0; k < kMaxPairs; ++k) {
                 const int b = tid / UO + k * bstep;
-                if (k < np && b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
-            }
-            last_t = -1;
-        }
-        if (t > 0) load_gx(t);
-        if (tid == 32 && ok) {
-            for (int q = 0; q < p.nq && ok; ++q) {
-                if (!bounded_wait(&hbar[q], par, w, SITE_GRU_H)) {
-                    ok = false;
-                    break;
+                if (k >= np || b >= p.batch) continue;
+                float ghr = bh_r, ghz = bh_z, ghn = bh_n;
+#pragma unroll
+                for (int s = 0; s < 4; ++s) {  // KS <= 4 sources, summed in rank order
+                    if (s < KS) {
+                        const float *rs = recv + (s * 3 * UO + ui) * kRecvStride + b;
+                        if (!RB || ph == 0) {
+                            ghr += rs[0];
+                            ghz += rs[UO * kRecvStride];
+                        }
+                        if (!RB || ph == 1) ghn += rs[2 * UO * kRecvStride];
+                    }
                 }
-                tc_fence_after();
-                for (int a = q * p.qk; a < (q + 1) * p.qk; ++a) {
-                    const uint32_t ua = smem_u32(sU + a * kAtomU);
-                    const uint32_t ha = smem_u32(sH + a * kAtomH);
-#pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        umma_bf16(tmem_d, sdesc_sw128(ua + k * 32, 16, 1024),
-                                  sdesc_sw128(ha + k * 32, 16, 1024), idesc,
-                                  (a > 0 || k > 0) ? 1u : 0u);
-                }
-            }
-            if (ok) umma_commit(mma_done);
-        }
-        __syncwarp();
-        // Block-uniform decision: every thread leaves the loop at the same step.
-        if (!__syncthreads_and(bounded_wait(mma_done, par, w, SITE_GRU_MMA) ? 1 : 0)) break;
-        tc_fence_after();
-        // Push: row gate*32 + u of the partial product (TMEM lane = row) goes to
-        // the cluster CTA that owns unit u, into its slot for this source rank.
-        if (warp < 3) {
-            uint32_t r[32];
-            tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
-            tmem_ld_wait();
-            const uint32_t owner = static_cast<uint32_t>(lane / UO);
-            const int oui = lane % UO;
-            const uint32_t dst = mapa_shared(
-                smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kRecvStride), owner);
-            const uint32_t rbar = mapa_shared(smem_u32(red_full), owner);
-            // Asynchronous remote stores: each counts its bytes on the owner's
-            // barrier, so nothing here waits for them to land.
-#pragma unroll
-            for (int c = 0; c < 8; ++c)
-                st_async_f4(dst + c * 16,
-                            make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
-                                        __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
-                            rbar);
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (!__syncthreads_and(bounded_wait<true>(red_full, par, w, SITE_GRU_RED) ? 1 : 0)) break;
-        uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
-#pragma unroll
-        for (int k = 0; k < kMaxPairs; ++k) {
-            const int b = tid / UO + k * bstep;
-            if (k >= np || b >= p.batch) continue;
-            float ghr = bh_r, ghz = bh_z, ghn = bh_n;
-#pragma unroll
-            for (int s = 0; s < 4; ++s) {  // KS <= 4 sources, summed in rank order
-                if (s < KS) {
-                    const float *rs = recv + (s * 3 * UO + ui) * kRecvStride + b;
-                    ghr += rs[0];
-                    ghz += rs[UO * kRecvStride];
-                    ghn += rs[2 * UO * kRecvStride];
+                if (!RB) {
+                    const float rg = sigmoidf_fast(gxr[k] + ghr);
+                    const float zg = sigmoidf_fast(gxz[k] + ghz);
+                    const float ng = tanhf_fast(gxn[k] + rg * ghn);
+                    const float hn = (1.0f - zg) * ng + zg * hprev[k];
+                    hprev[k] = hn;
+                    hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
+                } else if (ph == 0) {
+                    const float rg = sigmoidf_fast(gxr[k] + ghr);
+                    zsave[k] = sigmoidf_fast(gxz[k] + ghz);
+                    rhx_t[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(rg * hprev[k]);
+                } else {
+                    const float ng = tanhf_fast(gxn[k] + ghn);
+                    const float hn = (1.0f - zsave[k]) * ng + zsave[k] * hprev[k];
+                    hprev[k] = hn;
+                    hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
                 }
             }
-            const float rg = sigmoidf_fast(gxr[k] + ghr);
-            const float zg = sigmoidf_fast(gxz[k] + ghz);
-            const float ng = tanhf_fast(gxn[k] + rg * ghn);
-            const float hn = (1.0f - zg) * ng + zg * hprev[k];
-            hprev[k] = hn;
-            hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
+            if (ph == nph - 1) last_t = t;  // hprev holds h_t, not yet in h_out
+            // Publish first (the release then waits only for the exchange-buffer
+            // stores), then write this step's h_t to h_out.
+            fence_proxy_async_global();
+            __syncthreads();
+            if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
+                red_release_gpu_add(p.counter, 1u);
+            // recv is consumed: arm the barrier for the next round's partial
+            // rows (bytes that land before this are counted all the same).
+            if (tid == 0) mbar_arrive_expect_tx(red_full, round_bytes((ph + 1) % nph));
+            __syncwarp();
+            tc_fence_after();
         }
-        last_t = t;  // hprev holds h_t, not yet in h_out
-        // Publish first (the release then waits only for the exchange-buffer
-        // stores), then write this step's h_t to h_out.
-        fence_proxy_async_global();
-        __syncthreads();
-        if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
-            red_release_gpu_add(p.counter, 1u);
-        // recv is consumed: arm the barrier for the next step's partial rows
-        // (bytes that land before this are counted all the same).
-        if (tid == 0) mbar_arrive_expect_tx(red_full, recv_bytes);
-        __syncwarp();
-        tc_fence_after();
     }
     // h_T of the last step reached (or the step the loop left at).
     if (last_t >= 0) {
@@ -398,8 +445,9 @@ int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
 // Tensor maps of the recurrence: U as [3 gates][H rows][H] (box: 96 rows of
 // one group over one 64-wide K atom) and the two exchange buffers as
 // [H/64 atoms][32 batch rows][64] (box: one CTA's h piece).
-int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tmU, CUtensorMap *tmH0,
-                   CUtensorMap *tmH1) {
+// Also the r * h exchange buffers' maps (tmR0 / tmR1 over rhx; skipped when null).
+int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, int H, CUtensorMap *tmU,
+                   CUtensorMap *tmH0, CUtensorMap *tmH1, CUtensorMap *tmR0, CUtensorMap *tmR1) {
     int rc;
     const int ka = H / gru_splits(H) / 64;
     const int nq = (ka % 4 == 0) ? 4 : (ka % 3 == 0) ? 3 : (ka % 2 == 0) ? 2 : 1;
@@ -416,8 +464,16 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tm
         if ((rc = make_tmap_3d_bf16(i ? tmH1 : tmH0, hx + static_cast<size_t>(i) * kBatchPad * H, dims,
                                     strides, box)))
             return rc;
+        if (tmR0 && (rc = make_tmap_3d_bf16(i ? tmR1 : tmR0, rhx + static_cast<size_t>(i) * kBatchPad * H,
+                                            dims, strides, box)))
+            return rc;
     }
     return ISAM_OK;
+}
+
+int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tmU, CUtensorMap *tmH0,
+                   CUtensorMap *tmH1) {
+    return recurrent_maps(U, hx, nullptr, H, tmU, tmH0, tmH1, nullptr, nullptr);
 }
 
 // Fills the shape fields of p and launches the recurrence: one cluster of KS
@@ -425,7 +481,8 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tm
 // driver accepts it with clusters, otherwise after checking that every
 // cluster fits at once (the step counter needs every CTA resident).
 int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tmH0,
-                     const CUtensorMap &tmH1, size_t smem, cudaStream_t stream) {
+                     const CUtensorMap &tmH1, const CUtensorMap &tmR0, const CUtensorMap &tmR1, size_t smem,
+                     cudaStream_t stream) {
     const int H = p.H;
     p.ks = gru_splits(H);
     p.ka = H / p.ks / 64;
@@ -447,7 +504,7 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
     cfg.stream = stream;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, tmR0, tmR1, p);
     if (e == cudaSuccess) return ISAM_OK;
     (void)cudaGetLastError();
     cfg.numAttrs = 1;
@@ -458,7 +515,7 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
         return set_error(ISAM_ERR_UNSUPPORTED,
                          "GRU recurrence: %d CTAs in clusters of %d cannot be co-resident (%d clusters fit)",
                          p.n_cta, p.ks, max_clusters);
-    e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, p);
+    e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, tmR0, tmR1, p);
     if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel");
     return ISAM_OK;
 }
@@ -467,7 +524,7 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
 
 int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
                const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
-               cudaStream_t stream) {
+               cudaStream_t stream, int reset_before) {
     const int H = hidden;
     if (batch > kBatchPad || H % 64 != 0 || H > 1024 || H < 64)
         return set_error(ISAM_ERR_UNSUPPORTED,
@@ -490,7 +547,8 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
     if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_gx), &ds.gru_gx_bytes, gx_bytes,
                         "allocating the GRU projection workspace")))
         return rc;
-    const size_t hx_bytes = static_cast<size_t>(2) * kBatchPad * H * sizeof(uint16_t);
+    // Exchange buffers: h (2 slots) then r * h (2 slots, the reset-before form).
+    const size_t hx_bytes = static_cast<size_t>(4) * kBatchPad * H * sizeof(uint16_t);
     if (ds.gru_hx_bytes < hx_bytes) {
         if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_hx), &ds.gru_hx_bytes, hx_bytes,
                             "allocating the GRU exchange buffer")))
@@ -511,9 +569,12 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
     if ((rc = gemm_launch(g, plan, ds, stream))) return rc;
 
     // 2. Recurrence.
-    CUtensorMap tmU, tmH0, tmH1;
-    if ((rc = recurrent_maps(U, ds.gru_hx, H, &tmU, &tmH0, &tmH1))) return rc;
+    CUtensorMap tmU, tmH0, tmH1, tmR0, tmR1;
+    uint16_t *rhx = ds.gru_hx + static_cast<size_t>(2) * kBatchPad * H;
+    if ((rc = recurrent_maps(U, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1))) return rc;
     GruParams p{};
+    p.rhx = rhx;
+    p.reset_before = reset_before ? 1 : 0;
     p.T = T;
     p.batch = batch;
     p.H = H;
@@ -537,7 +598,7 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
         if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
         attr_set = true;
     }
-    return launch_recurrent(p, tmU, tmH0, tmH1, smem, stream);
+    return launch_recurrent(p, tmU, tmH0, tmH1, tmR0, tmR1, smem, stream);
 }
 
 }  // namespace isam
@@ -709,7 +770,9 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         p.skip_publish_cta = -1;
         p.timeout_ns = wait_timeout_ns();
         p.err = err;
-        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, smem, stream))) return rc;
+        p.rhx = hx;  // the reset-after form only
+        p.reset_before = 0;
+        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, tmH0, tmH1, smem, stream))) return rc;
     }
     // Report device-side timeouts of this call before returning.
     if ((e = cudaStreamSynchronize(stream)) != cudaSuccess)

@@ -79,9 +79,10 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
 // Independent GEMMs in one persistent launch (1 <= count <= 64).
 int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStream_t s);
 
+// reset_before: the candidate's recurrent input is U_n (r * h) (two rounds per step).
 int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
                const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
-               cudaStream_t s);
+               cudaStream_t s, int reset_before = 0);
 
 int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
                  const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t s);

@@ -60,10 +60,11 @@ def load():
         lib.isam_gemm_fp8.argtypes = [i, i, i, f, P, P, f, P]
         lib.isam_gemm_grouped_fp8.argtypes = [i, P, P, P, P, P, P, P, P]
         lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
+        lib.isam_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
                      "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
-                     "isam_gru_forward",
+                     "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_dwsep_conv"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
@@ -200,8 +201,9 @@ def gemm_plan(M, N, K, transA, transB, beta=0.0) -> dict:
     return dict(zip(("BN", "split", "stages", "group_m", "grid", "smem"), list(out)))
 
 
-def gru_forward(T, batch, hidden, x, W, U, b, h0, h_out) -> None:
-    """isam_gru_forward (x, W, U bf16; b, h0, h_out fp32; h0 may be None)."""
+def gru_forward(T, batch, hidden, x, W, U, b, h0, h_out, reset_before=False) -> None:
+    """isam_gru_forward, or isam_gru_forward_reset_before with reset_before
+    (x, W, U bf16; b, h0, h_out fp32; h0 may be None)."""
     import torch
     lib = load()
     H = hidden
@@ -213,8 +215,8 @@ def gru_forward(T, batch, hidden, x, W, U, b, h0, h_out) -> None:
         _dev(h0, torch.float32, batch * H, "h0")
     _dev(h_out, torch.float32, T * batch * H, "h_out")
     _use_current_stream(lib)
-    check(lib.isam_gru_forward(T, batch, H, _ptr(x), _ptr(W), _ptr(U), _ptr(b), _ptr(h0),
-                               _ptr(h_out)))
+    fn = lib.isam_gru_forward_reset_before if reset_before else lib.isam_gru_forward
+    check(fn(T, batch, H, _ptr(x), _ptr(W), _ptr(U), _ptr(b), _ptr(h0), _ptr(h_out)))
 
 
 def dwsep_conv(N, H, W, Cin, Cout, x, dw_w, pw_w, out) -> None:

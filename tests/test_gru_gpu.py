@@ -1,6 +1,6 @@
-"""GRU forward parity on the GPU through the C ABI (isam_gru_forward) against
-the fp64 oracle.  Tolerance: normalised max error over every step's hidden
-state (all of h_out) <= 1e-2."""
+"""GRU forward parity on the GPU through the C ABI (isam_gru_forward and
+isam_gru_forward_reset_before) against the fp64 oracle.  Tolerance: normalised
+max error over every step's hidden state (all of h_out) <= 1e-2."""
 import os
 import subprocess
 import sys
@@ -29,13 +29,13 @@ def _lib():
     isam.sync()
 
 
-def run_gru(x, W, U, b, h0):
+def run_gru(x, W, U, b, h0, reset_before=False):
     import torch
     T, batch, H = x.shape
     out = Guarded(T * batch * H)
     h0d = None if h0 is None else torch.from_numpy(np.ascontiguousarray(h0, np.float32)).cuda()
     isam.gru_forward(T, batch, H, dev_bf16(x), dev_bf16(W), dev_bf16(U),
-                     torch.from_numpy(b).cuda(), h0d, out.t)
+                     torch.from_numpy(b).cuda(), h0d, out.t, reset_before=reset_before)
     isam.sync()
     assert out.guards_intact(), "write outside h_out"
     return out.numpy().reshape(T, batch, H)
@@ -115,10 +115,12 @@ def test_gru_unsupported_shapes_rejected():
     assert lib.isam_gru_forward(1, 1, 960, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
 
 
-def test_gru_missing_participant_times_out_cleanly():
+@pytest.mark.parametrize("reset_before", [False, True])
+def test_gru_missing_participant_times_out_cleanly(reset_before):
     """One CTA never signals the step counter (a flag nothing sets): every
     bounded wait runs out, the kernel returns, isam_sync reports
     ISAM_ERR_TIMEOUT, and the context stays usable for a correct call."""
+    rb = bool(reset_before)
     code = textwrap.dedent(f"""
         import sys, numpy as np, torch
         sys.path.insert(0, {ROOT!r}); sys.path.insert(0, {os.path.join(ROOT, 'tests')!r})
@@ -132,13 +134,13 @@ def test_gru_missing_participant_times_out_cleanly():
         args = [dev_bf16(x), dev_bf16(W), dev_bf16(U), torch.from_numpy(b).cuda(), None]
         out = torch.zeros(T * batch * H, device="cuda")
         os.environ["ISAM_DEBUG_GRU_SKIP_CTA"] = "0"
-        isam.gru_forward(T, batch, H, *args, out)
+        isam.gru_forward(T, batch, H, *args, out, reset_before={rb!r})
         rc = isam.load().isam_sync()
         assert rc == isam.ISAM_ERR_TIMEOUT, rc
         del os.environ["ISAM_DEBUG_GRU_SKIP_CTA"]
-        isam.gru_forward(T, batch, H, *args, out)
+        isam.gru_forward(T, batch, H, *args, out, reset_before={rb!r})
         isam.sync()
-        ref = oracle.gru_forward(x, W, U, b, None)
+        ref = oracle.gru_forward(x, W, U, b, None, reset_before={rb!r})
         assert nmax_err(out.cpu().numpy().reshape(T, batch, H), ref) <= 1e-2
         print("TIMEOUT_OK")
     """)
@@ -146,3 +148,65 @@ def test_gru_missing_participant_times_out_cleanly():
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
                        timeout=300)
     assert r.returncode == 0 and "TIMEOUT_OK" in r.stdout, r.stdout + r.stderr
+
+
+# ---- reset gate applied before the candidate's recurrent product:
+# n = tanh(W_n x + b_in + U_n (r * h_{t-1}) + b_hn).
+
+def test_gru_reset_before_benchmark_shape_full_oracle():
+    T, batch, H = 128, 32, 1024
+    x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=synth.stream_seed(synth.BASE_SEED, 3))
+    got = run_gru(x, W, U, b, h0, reset_before=True)
+    ref = oracle.gru_forward(x, W, U, b, h0, reset_before=True)
+    assert nmax_err(got, ref) <= TOL
+    assert nmax_err(got[-1], ref[-1]) <= TOL
+    # the two forms really differ at this shape (the test would not see a mix-up otherwise)
+    other = oracle.gru_forward(x, W, U, b, h0)
+    assert nmax_err(other, ref) > 10 * TOL
+
+
+@pytest.mark.parametrize("T,batch,H", [(1, 1, 64), (5, 3, 64), (7, 17, 192), (9, 32, 128),
+                                       (3, 31, 320), (16, 8, 1024), (6, 32, 768), (4, 5, 896),
+                                       (3, 2, 832)])
+def test_gru_reset_before_shapes_with_initial_state(T, batch, H):
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 1000 + batch * 10 + H + 1)
+    h0 = synth.f32_uniform(T + batch + H + 1, (batch, H))
+    got = run_gru(x, W, U, b, h0, reset_before=True)
+    ref = oracle.gru_forward(x, W, U, b, h0, reset_before=True)
+    assert nmax_err(got, ref) <= TOL
+
+
+def test_gru_reset_before_open_reset_gate_matches_reset_after():
+    """A reset gate saturated at 1 (b_ir = 30) makes both forms the same
+    function; the two kernels then see the same bf16 operands and the same
+    summation order, so their outputs agree to fp32 rounding of the gates."""
+    T, batch, H = 8, 32, 512
+    x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=21)
+    b = b.copy()
+    b[:H] = 30.0
+    rb = run_gru(x, W, U, b, h0, reset_before=True)
+    ra = run_gru(x, W, U, b, h0)
+    assert nmax_err(rb, ra) <= 1e-4
+    assert nmax_err(rb, oracle.gru_forward(x, W, U, b, h0, reset_before=True)) <= TOL
+
+
+def test_gru_reset_before_zero_weights_closed_form():
+    T, batch, H = 6, 4, 128
+    zero = np.zeros((3 * H, H), np.uint16)
+    x = synth.bf16_normal(1, (T, batch, H))
+    b = synth.f32_uniform(2, (6 * H,), -2.0, 2.0)
+    h0 = synth.f32_uniform(3, (batch, H))
+    got = run_gru(x, zero, zero, b, h0, reset_before=True)
+    ref = oracle.gru_forward(x, zero, zero, b, h0, reset_before=True)
+    assert np.max(np.abs(got - ref)) <= 1e-5
+
+
+def test_gru_reset_before_repeat_and_interleaved_calls_identical():
+    """Both forms share the exchange workspace: interleaving them changes nothing."""
+    T, batch, H = 12, 32, 256
+    x, W, U, b, h0 = synth.gru_operands(T, batch, H, seed=13)
+    a = run_gru(x, W, U, b, h0, reset_before=True)
+    m = run_gru(x, W, U, b, h0)
+    c = run_gru(x, W, U, b, h0, reset_before=True)
+    d = run_gru(x, W, U, b, h0)
+    assert np.array_equal(a, c) and np.array_equal(m, d)
