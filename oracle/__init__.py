@@ -58,6 +58,8 @@ def _load():
             lib.oracle_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
             lib.oracle_gru_forward_reset_before.restype = ctypes.c_int
             lib.oracle_gemm_fp8.restype = ctypes.c_int
+            lib.oracle_gru_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
+            lib.oracle_gru_stack.restype = ctypes.c_int
             for f in (lib.oracle_gemm_rows, lib.oracle_gemm, lib.oracle_gru_forward,
                       lib.oracle_dwsep, lib.oracle_num_threads):
                 f.restype = ctypes.c_int
@@ -138,6 +140,27 @@ def gru_forward(x, W, U, b, h0=None, reset_before=False):
     rc = fn(T, batch, H, _p(x), _p(W), _p(U), _p(b), _p(h0), _p(out))
     if rc != 0:
         raise ValueError("oracle_gru_forward: invalid argument")
+    return out
+
+
+def gru_stack(x, W, U, b, h0=None, reset_before=False):
+    """Every layer's hidden states [layers, T, batch, H] float64 of a stacked
+    GRU: W, U [layers, 3H, H] bf16 bits, b [layers, 6H], h0 [layers, batch, H]
+    or None; layer l > 0 reads layer l - 1's states unrounded."""
+    x, W, U = _u16(x), _u16(W), _u16(U)
+    T, batch, H = x.shape
+    L = W.shape[0]
+    assert W.shape == (L, 3 * H, H) and U.shape == (L, 3 * H, H)
+    b = np.ascontiguousarray(b, dtype=np.float32)
+    assert b.size == L * 6 * H
+    if h0 is not None:
+        h0 = np.ascontiguousarray(h0, dtype=np.float32)
+        assert h0.size == L * batch * H
+    out = np.empty((L, T, batch, H), dtype=np.float64)
+    rc = _load().oracle_gru_stack(L, T, batch, H, int(bool(reset_before)), _p(x), _p(W), _p(U),
+                                  _p(b), _p(h0), _p(out))
+    if rc != 0:
+        raise ValueError("oracle_gru_stack: invalid argument")
     return out
 
 

@@ -263,6 +263,96 @@ int oracle_gru_forward_reset_before(int T, int batch, int H, const uint16_t *x, 
 }
 
 /*
+ * One GRU layer over one sequence s, for the stacked form below: the input
+ * at step t is either bf16 (x16, the first layer) or double (x64, the hidden
+ * states of the layer underneath, taken unrounded).  Gate order r, z, n;
+ * reset_before selects U_n (r * h_{t-1}) over r * (U_n h_{t-1} + b_hn) in the
+ * candidate.  h_out row (t, s) receives h_t.
+ */
+static void gru_layer_sequence(int T, int batch, int H, int s, int reset_before,
+                               const uint16_t *x16, const double *x64, const uint16_t *W,
+                               const uint16_t *U, const float *b, const float *h0,
+                               double *h_out, double *h, double *xin, double *gx, double *gh,
+                               double *rh) {
+    const int G = 3 * H;
+    for (int j = 0; j < H; ++j) h[j] = h0 ? (double)h0[(size_t)s * H + j] : 0.0;
+    for (int t = 0; t < T; ++t) {
+        const size_t row = ((size_t)t * batch + s) * H;
+        for (int k = 0; k < H; ++k) xin[k] = x16 ? bf(x16[row + k]) : x64[row + k];
+        for (int g = 0; g < G; ++g) {  /* input projection, every gate */
+            double a = 0.0;
+            const uint16_t *wr = W + (size_t)g * H;
+            for (int k = 0; k < H; ++k) a += bf(wr[k]) * xin[k];
+            gx[g] = a + (double)b[g];
+        }
+        for (int g = 0; g < 2 * H; ++g) {  /* recurrent product of r and z */
+            double a = 0.0;
+            const uint16_t *ur = U + (size_t)g * H;
+            for (int k = 0; k < H; ++k) a += bf(ur[k]) * h[k];
+            gh[g] = a + (double)b[G + g];
+        }
+        for (int j = 0; j < H; ++j) {
+            const double r = sigmoid(gx[j] + gh[j]);
+            rh[j] = reset_before ? r * h[j] : h[j];
+            gh[j] = r;  /* r kept for the reset-after candidate */
+        }
+        for (int j = 0; j < H; ++j) {  /* candidate's recurrent product */
+            double a = 0.0;
+            const uint16_t *un = U + (size_t)(2 * H + j) * H;
+            for (int k = 0; k < H; ++k) a += bf(un[k]) * rh[k];
+            gh[2 * H + j] = a + (double)b[G + 2 * H + j];
+        }
+        double *ho = h_out + row;
+        for (int j = 0; j < H; ++j) {
+            const double r = gh[j];
+            const double z = sigmoid(gx[H + j] + gh[H + j]);
+            const double n = reset_before ? tanh(gx[2 * H + j] + gh[2 * H + j])
+                                          : tanh(gx[2 * H + j] + r * gh[2 * H + j]);
+            ho[j] = (1.0 - z) * n + z * h[j];
+        }
+        for (int j = 0; j < H; ++j) h[j] = ho[j];
+    }
+}
+
+/*
+ * Stacked GRU: `layers` GRU layers of width H (Section 5.1.2's cell, gate
+ * order r, z, n), layer 0 reading x and layer l > 0 reading the hidden
+ * states h^{l-1}_t of the layer below at the same step, in double precision
+ * (no rounding between layers).
+ *
+ * x [T][batch][H] bf16; W, U [layers][3H][H] bf16 (layer l's input and
+ * recurrent weights); b [layers][6H] fp32 (b_ih | b_hh per layer);
+ * h0 [layers][batch][H] fp32 or NULL (zeros); h_out [layers][T][batch][H]
+ * double, every layer's states.  Returns 0, or 1 on an invalid argument.
+ */
+int oracle_gru_stack(int layers, int T, int batch, int H, int reset_before, const uint16_t *x,
+                     const uint16_t *W, const uint16_t *U, const float *b, const float *h0,
+                     double *h_out) {
+    if (layers < 1 || T < 1 || batch < 1 || H < 1 || !x || !W || !U || !b || !h_out) return 1;
+    const size_t wsz = (size_t)3 * H * H, seq = (size_t)T * batch * H;
+    for (int l = 0; l < layers; ++l) {
+        const uint16_t *x16 = l == 0 ? x : NULL;
+        const double *x64 = l == 0 ? NULL : h_out + (size_t)(l - 1) * seq;
+        const float *h0l = h0 ? h0 + (size_t)l * batch * H : NULL;
+#pragma omp parallel
+        {
+            double *h = (double *)malloc(sizeof(double) * (size_t)H);
+            double *xin = (double *)malloc(sizeof(double) * (size_t)H);
+            double *rh = (double *)malloc(sizeof(double) * (size_t)H);
+            double *gx = (double *)malloc(sizeof(double) * (size_t)3 * H);
+            double *gh = (double *)malloc(sizeof(double) * (size_t)3 * H);
+#pragma omp for schedule(dynamic, 1)
+            for (int s = 0; s < batch; ++s)
+                gru_layer_sequence(T, batch, H, s, reset_before, x16, x64, W + (size_t)l * wsz,
+                                   U + (size_t)l * wsz, b + (size_t)l * 6 * H, h0l,
+                                   h_out + (size_t)l * seq, h, xin, gx, gh, rh);
+            free(h); free(xin); free(rh); free(gx); free(gh);
+        }
+    }
+    return 0;
+}
+
+/*
  * Separable depthwise convolution, Listing 3, with stride s = 1, channel
  * multiplier c = 1 (so r = 0 and P is indexed P[q][k]) and a zero border of
  * one pixel (input row i + di - 1, column j + dj - 1), taken in the factored

@@ -429,3 +429,72 @@ def test_gru_reset_before_saturated_reset_gate(oracle_lib):
     a = oracle_lib.gru_forward(x, W, U, b0, h0, reset_before=True)
     c = oracle_lib.gru_forward(x, W, U0, b0, h0)
     assert np.max(np.abs(a - c)) < 1e-10
+
+
+# ---- stacked GRU (layer l > 0 reads layer l - 1's states)
+
+def _stack_operands(L, T, B, H, seed):
+    x, _, _, _, _ = synth.gru_operands(T, B, H, seed=seed)
+    W = np.stack([synth.gru_operands(1, 1, H, seed=seed + 10 * l + 1)[1] for l in range(L)])
+    U = np.stack([synth.gru_operands(1, 1, H, seed=seed + 10 * l + 2)[2] for l in range(L)])
+    b = np.stack([synth.gru_operands(1, 1, H, seed=seed + 10 * l + 3)[3] for l in range(L)])
+    h0 = synth.f32_uniform(seed + 7, (L, B, H))
+    return x, W, U, b, h0
+
+
+@pytest.mark.parametrize("reset_before", [False, True])
+def test_gru_stack_one_layer_is_the_single_layer_gru(oracle_lib, reset_before):
+    T, B, H = 5, 3, 16
+    x, W, U, b, h0 = _stack_operands(1, T, B, H, seed=50)
+    got = oracle_lib.gru_stack(x, W, U, b, h0, reset_before=reset_before)
+    ref = oracle_lib.gru_forward(x, W[0], U[0], b[0], h0[0], reset_before=reset_before)
+    assert np.max(np.abs(got[0] - ref)) < 1e-12
+
+
+def test_gru_stack_matches_torch_float64(oracle_lib):
+    """torch.nn.GRU(num_layers=3) feeds each layer's output sequence to the
+    next layer, with per-layer initial states: an independent implementation
+    of the same stack (reset gate after the recurrent product)."""
+    torch = pytest.importorskip("torch")
+    L, T, B, H = 3, 6, 4, 20
+    x, W, U, b, h0 = _stack_operands(L, T, B, H, seed=60)
+    got = oracle_lib.gru_stack(x, W, U, b, h0)
+    gru = torch.nn.GRU(H, H, num_layers=L, bias=True).double()
+    with torch.no_grad():
+        for l in range(L):
+            getattr(gru, f"weight_ih_l{l}").copy_(torch.from_numpy(f64(W[l])))
+            getattr(gru, f"weight_hh_l{l}").copy_(torch.from_numpy(f64(U[l])))
+            getattr(gru, f"bias_ih_l{l}").copy_(torch.from_numpy(b[l, :3 * H].astype(np.float64)))
+            getattr(gru, f"bias_hh_l{l}").copy_(torch.from_numpy(b[l, 3 * H:].astype(np.float64)))
+        out, hT = gru(torch.from_numpy(f64(x)), torch.from_numpy(h0.astype(np.float64)))
+    np.testing.assert_allclose(got[-1], out.numpy(), rtol=0, atol=1e-12)
+    for l in range(L):
+        np.testing.assert_allclose(got[l, -1], hT[l].numpy(), rtol=0, atol=1e-12)
+
+
+def test_gru_stack_reset_before_matches_python_loops(oracle_lib):
+    L, T, B, H = 2, 3, 2, 4
+    x, W, U, b, h0 = _stack_operands(L, T, B, H, seed=70)
+    got = oracle_lib.gru_stack(x, W, U, b, h0, reset_before=True)
+    inp = f64(x)
+    for l in range(L):
+        ref = _gru_rb_python(inp, f64(W[l]), f64(U[l]), b[l].astype(np.float64),
+                             h0[l].astype(np.float64))
+        assert np.max(np.abs(got[l] - ref)) < 1e-12
+        inp = ref
+
+
+@pytest.mark.parametrize("reset_before", [False, True])
+def test_gru_stack_lower_layers_ignore_upper_weights(oracle_lib, reset_before):
+    """Layer l depends on layers 0..l only: changing the top layer's weights
+    leaves every lower layer's states bit for bit unchanged, and changes the
+    top layer's."""
+    L, T, B, H = 3, 4, 2, 12
+    x, W, U, b, h0 = _stack_operands(L, T, B, H, seed=80)
+    a = oracle_lib.gru_stack(x, W, U, b, h0, reset_before=reset_before)
+    W2, U2 = W.copy(), U.copy()
+    W2[-1] = W[0]
+    U2[-1] = U[1]
+    c = oracle_lib.gru_stack(x, W2, U2, b, h0, reset_before=reset_before)
+    assert np.array_equal(a[:-1], c[:-1])
+    assert np.max(np.abs(a[-1] - c[-1])) > 1e-3
