@@ -395,6 +395,31 @@ def hot_path_rows(isam, dev, peaks):
         "us_per_step": round(ms * 1e3 / T, 3), "tflops": round(tf, 2),
         "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4)}
     del x, W, U, b, h0, hout
+    # Two stacked layers (the second layer's projection fused into the first
+    # layer's recurrence), against the same stack as one call per layer.
+    L = 2
+    x = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 5, 1), T * batch * H, dev)
+    W = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 5, 2), L * 3 * H * H, dev, -s, s)
+    U = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 5, 3), L * 3 * H * H, dev, -s, s)
+    b = synth.f32_uniform_torch(synth.stream_seed(synth.BASE_SEED, 5, 4), L * 6 * H, dev, -0.1, 0.1)
+    hout = torch.empty(L * T * batch * H, dtype=torch.float32, device=dev)
+    ms = time_call(lambda: isam.gru_forward_stack(L, T, batch, H, x, W, U, b, None, hout), reps=10,
+                   warmup=3, flush=flush)
+    seq = T * batch * H
+    x1 = torch.empty(seq, dtype=torch.bfloat16, device=dev)
+
+    def per_layer():
+        isam.gru_forward(T, batch, H, x, W[:3 * H * H], U[:3 * H * H], b[:6 * H], None, hout[:seq])
+        x1.copy_(hout[:seq])
+        isam.gru_forward(T, batch, H, x1, W[3 * H * H:], U[3 * H * H:], b[6 * H:], None, hout[seq:])
+    ms_pl = time_call(per_layer, reps=10, warmup=3, flush=flush)
+    out["gru_stack2_h1024_b32_t128"] = {
+        "ms": round(ms, 4), "layer_timesteps_per_s": round(L * T / (ms / 1e3), 1),
+        "us_per_layer_step": round(ms * 1e3 / (L * T), 3),
+        "per_layer_calls_ms": round(ms_pl, 4),
+        "what": "2 layers in one isam_gru_forward_stack call; per_layer_calls_ms: two "
+                "isam_gru_forward calls with a bf16 cast (torch) between"}
+    del x, W, U, b, hout, x1
     # Separable depthwise layer.
     N, Hh, Ww, Cin, Cout = 32, 56, 56, 128, 256
     xd = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 4, 1), N * Hh * Ww * Cin, dev)
@@ -515,7 +540,8 @@ def run_case(args):
     """Times one hot-path call on its own (for profiling and sweeps):
     sweep (the 32 sweep GEMMs in one grouped call) | gemm:M,N,K,transA,transB,beta |
     gru[:T,batch,hidden] | gru_rb[:T,batch,hidden] (reset gate before the candidate's
-    product) | dwsep[:N,H,W,Cin,Cout]."""
+    product) | gru_stack[:L,T,batch,hidden] | gru_stack_rb[:...] | gru_layers[:...] (the
+    stack as one call per layer) | dwsep[:N,H,W,Cin,Cout]."""
     import torch
     from paper_1810_09958_gb300 import build, isam, synth
     torch.cuda.set_device(0)
@@ -553,6 +579,31 @@ def run_case(args):
         rb = kind == "gru_rb"
         fn = lambda: isam.gru_forward(T, batch, H, x, W, U, b, None, hout, reset_before=rb)
         work = {"tflops": 2.0 * T * batch * 3 * H * 2 * H / 1e12, "timesteps": T}
+    elif kind in ("gru_stack", "gru_stack_rb", "gru_layers"):
+        L, T, batch, H = (int(v) for v in vals) if vals else (2, 128, 32, 1024)
+        s = H ** -0.5
+        x = synth.bf16_normal_torch(21, T * batch * H, dev)
+        W = synth.bf16_uniform_torch(22, L * 3 * H * H, dev, -s, s)
+        U = synth.bf16_uniform_torch(23, L * 3 * H * H, dev, -s, s)
+        b = synth.f32_uniform_torch(24, L * 6 * H, dev, -0.1, 0.1)
+        hout = torch.empty(L * T * batch * H, dtype=torch.float32, device=dev)
+        if kind == "gru_layers":
+            # the same stack as one isam_gru_forward call per layer, with a bf16
+            # cast of each layer's states (a torch kernel) as the next input
+            xs = [x] + [torch.empty(T * batch * H, dtype=torch.bfloat16, device=dev) for _ in range(L - 1)]
+            seq = T * batch * H
+
+            def fn():
+                for l in range(L):
+                    if l > 0:
+                        xs[l].copy_(hout[(l - 1) * seq:l * seq])
+                    isam.gru_forward(T, batch, H, xs[l], W[l * 3 * H * H:(l + 1) * 3 * H * H],
+                                     U[l * 3 * H * H:(l + 1) * 3 * H * H], b[l * 6 * H:(l + 1) * 6 * H],
+                                     None, hout[l * seq:(l + 1) * seq])
+        else:
+            rb = kind == "gru_stack_rb"
+            fn = lambda: isam.gru_forward_stack(L, T, batch, H, x, W, U, b, None, hout, reset_before=rb)
+        work = {"tflops": L * 2.0 * T * batch * 3 * H * 2 * H / 1e12, "timesteps": T}
     elif kind == "dwsep":
         N, H, W, Cin, Cout = (int(v) for v in vals) if vals else (32, 56, 56, 128, 256)
         x = synth.bf16_normal_torch(31, N * H * W * Cin, dev)

@@ -205,6 +205,38 @@ int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 
                                   const float *h0, float *h_out);
 
 /*
+ * Stacked GRU: `layers` GRU layers of width `hidden`, layer 0 reading x and
+ * layer l > 0 reading the hidden states of layer l - 1 at the same step
+ * (Section 5.1.2's cell, stacked; the recurrent scheduling of Section 3.6 per
+ * layer).  reset_before = 0 gives isam_gru_forward's cell, 1 that of
+ * isam_gru_forward_reset_before.
+ *
+ *   x      [T][batch][hidden]            bf16, layer 0's input
+ *   W, U   [layers][3*hidden][hidden]    bf16, each layer's input and
+ *                                        recurrent weights (r, z, n rows)
+ *   b      [layers][6*hidden]            fp32, b_ih | b_hh per layer
+ *   h0     [layers][batch][hidden]       fp32 or NULL (zeros)
+ *   h_out  [layers][T][batch][hidden]    fp32, every layer's states; layer
+ *                                        layers - 1 is the stack's output
+ *
+ * Only layer 0's input projection is a separate GEMM.  Layer l's persistent
+ * kernel also keeps its K quarter of layer l + 1's W resident and multiplies
+ * it by the bf16(h_{t-1}) tile it loads for its own recurrent product, so
+ * layer l + 1's projection is computed while layer l runs (one extra round
+ * at the end covers h_{T-1}); layer l + 1 reads it as per-K-rank partial
+ * sums (fixed order: deterministic).  The next layer therefore sees
+ * bf16(h^l_t), as the recurrent product sees bf16(h_{t-1}).
+ *
+ * Supported: as isam_gru_forward; with layers > 1, also the shared memory
+ * for both weight slices, which excludes hidden 576, 704, 832 and 960
+ * (ISAM_ERR_UNSUPPORTED).  Workspace: 2 x ks x T x batch x 3*hidden fp32
+ * (ks = 4, 2 or 1 K splits) beside isam_gru_forward's.
+ */
+int isam_gru_forward_stack(int layers, int T, int batch, int hidden, int reset_before,
+                           const isam_bf16 *x, const isam_bf16 *W, const isam_bf16 *U,
+                           const float *b, const float *h0, float *h_out);
+
+/*
  * GRU forward that allocates nothing.  The paper has no counterpart: this is a
  * deployment variant of isam_gru_forward for callers that cannot let a library
  * call cudaMalloc -- a process whose device memory is all reserved up front by

@@ -246,6 +246,7 @@ int isam_shutdown(void) {
         cudaFree(ds->gru_gx);
         cudaFree(ds->gru_hx);
         cudaFree(ds->gru_counter);
+        cudaFree(ds->gru_gxp);
         delete ds;
         g_dev[d] = nullptr;
     }
@@ -371,6 +372,22 @@ int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 
     DeviceState *ds = device_state(&rc);
     if (!ds) return rc;
     return gru_launch(T, batch, hidden, x, W, U, b, h0, h_out, *ds, current_stream(), 1);
+}
+
+int isam_gru_forward_stack(int layers, int T, int batch, int hidden, int reset_before,
+                          const isam_bf16 *x, const isam_bf16 *W, const isam_bf16 *U, const float *b,
+                          const float *h0, float *h_out) {
+    if (layers < 1 || T < 1 || batch < 1 || hidden < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_stack: sizes must be >= 1");
+    if (reset_before != 0 && reset_before != 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_stack: reset_before must be 0 or 1");
+    if (!x || !W || !U || !b || !h_out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_stack: null pointer");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gru_stack_launch(layers, T, batch, hidden, reset_before, x, W, U, b, h0, h_out, *ds,
+                            current_stream());
 }
 
 int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,

@@ -56,7 +56,9 @@ enum : uint32_t {
     SITE_GRU_H = 0x203,
     SITE_GRU_MMA = 0x204,
     SITE_GRU_RED = 0x205,
+    SITE_GRU_W = 0x206,
 };
+
 
 struct GruParams {
     int T, batch, H;
@@ -72,6 +74,11 @@ struct GruParams {
     uint16_t *hx;              // [2][32][H] bf16 exchange of h
     uint16_t *rhx;             // [2][32][H] bf16 exchange of r * h (reset_before)
     int reset_before;          // candidate's recurrent input U_n (r * h): two rounds per step
+    int gx_parts;              // slabs summed into each projection value (1: gx = x W^T + b_ih)
+    size_t gx_slab;            // floats between two slabs of gx
+    const float *b_ih;         // [3H], added to the slab sum when gx_parts > 1 (else null)
+    int has_next;              // also multiply the next layer's W by every loaded h
+    float *gxp_out;            // [ks][T*batch][3H]: the next layer's projection, one slab per K rank
     uint32_t *counter;         // step counter (zeroed before launch)
     int skip_publish_cta;      // debug: this CTA never publishes (-1: none)
     unsigned long long timeout_ns;
@@ -116,42 +123,53 @@ __device__ bool wait_counter(const uint32_t *counter, uint32_t target, const Wai
 }
 
 struct GruLayout {
-    int off_u, off_h, off_recv, off_bars, total;
+    int off_u, off_w, off_h, off_recv, off_bars, total;
 };
 
-__host__ __device__ inline GruLayout gru_layout(int ka) {
+// U slice | next layer's W slice (has_next) | pad | h piece | partial rows | barriers.
+__host__ __device__ inline GruLayout gru_layout(int ka, bool has_next) {
     GruLayout L;
     L.off_u = 0;
-    L.off_h = ka * kAtomU + kUPad;
+    L.off_w = ka * kAtomU;
+    L.off_h = L.off_w + (has_next ? ka * kAtomU : 0) + kUPad;
     L.off_recv = L.off_h + ka * kAtomH;
     L.off_bars = L.off_recv + kRecvBytes;
     L.total = L.off_bars + 128 + 1024;
     return L;
 }
 
-constexpr int kMaxPairs = 8;  // (unit, batch) pairs per thread when one CTA owns all 32 units
-
+// Template argument KS: K splits per unit group (cluster size, 4, 2 or 1).
+// A CTA evaluates the gates of UO = 32 / KS units over 32 batch rows, NP =
+// 8 / KS (unit, batch) pairs per thread.
+template <int KS>
 __global__ void __launch_bounds__(kThreads, 1)
     gru_recurrent_kernel(const __grid_constant__ CUtensorMap tmU,
                          const __grid_constant__ CUtensorMap tmH0,
                          const __grid_constant__ CUtensorMap tmH1,
                          const __grid_constant__ CUtensorMap tmR0,
-                         const __grid_constant__ CUtensorMap tmR1, const GruParams p) {
-    if (!launch_shape_ok(p.err, static_cast<uint32_t>(p.ks), static_cast<uint32_t>(p.n_cta), 0x3F0u))
+                         const __grid_constant__ CUtensorMap tmR1,
+                         const __grid_constant__ CUtensorMap tmWn, const GruParams p) {
+    constexpr int UO = kGroup / KS;
+    constexpr int NP = UO * kBatchPad / kThreads;
+    constexpr int BSTEP = kThreads / UO;
+    if (!launch_shape_ok(p.err, static_cast<uint32_t>(KS), static_cast<uint32_t>(p.n_cta), 0x3F0u))
         return;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
-    const GruLayout L = gru_layout(p.ka);
+    const bool HN = p.has_next != 0;
+    const GruLayout L = gru_layout(p.ka, HN);
     uint8_t *sU = smem + L.off_u;
+    uint8_t *sW = smem + L.off_w;
     uint8_t *sH = smem + L.off_h;
     float *recv = reinterpret_cast<float *>(smem + L.off_recv);  // [ks src][3 gates][uo][32 batch]
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + L.off_bars);
-    uint64_t *ubar = bars;                  // U slice landed
+    uint64_t *ubar = bars;                  // U (and next W) slice landed
     uint64_t *hbar = bars + 1;              // [kMaxPieces] h piece landed
     uint64_t *mma_done = hbar + kMaxPieces; // MMAs of the step complete
     uint64_t *red_full = mma_done + 1;      // all partial rows of my units arrived
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(red_full + 1);
+    uint64_t *w_done = red_full + 1;        // next layer's projection MMAs complete
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(w_done + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int tid = threadIdx.x;
@@ -159,8 +177,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lane = tid & 31;
     const int H = p.H;
     const int G = 3 * H;
-    const int KS = p.ks;
-    const int UO = p.uo;
     const int group = blockIdx.x / KS;
     const uint32_t rank = KS > 1 ? cluster_ctarank() : 0u;
     const int unit0 = group * kGroup;
@@ -172,12 +188,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int q = 0; q < kMaxPieces; ++q) mbar_init(&hbar[q], 1);
         mbar_init(mma_done, 1);
         mbar_init(red_full, 1);  // armed with the bytes of a step's partial rows
+        mbar_init(w_done, 1);
         *abort_flag = 0;
         fence_mbar_init();
     }
     __syncwarp();
+    // Columns 0-31: the recurrent product; 32-95: the next layer's projection,
+    // double-buffered by step parity.
+    const uint32_t tmem_cols = HN ? 128u : 32u;
     if (warp == 0) {
-        tmem_alloc(tmem_slot, 32);
+        tmem_alloc(tmem_slot, tmem_cols);
         tmem_relinquish();
     }
     tc_fence_before();
@@ -205,24 +225,27 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_prefetch_desc(&tmR0);
             tma_prefetch_desc(&tmR1);
         }
-        mbar_arrive_expect_tx(ubar, static_cast<uint32_t>(p.ka * kAtomU));
+        mbar_arrive_expect_tx(ubar, static_cast<uint32_t>(p.ka * kAtomU * (HN ? 2 : 1)));
         for (int a = 0; a < p.ka; ++a)
             tma_load_3d(&tmU, ubar, sU + a * kAtomU, (atom0 + a) * 64, unit0, 0);
+        if (HN)
+            for (int a = 0; a < p.ka; ++a)
+                tma_load_3d(&tmWn, ubar, sW + a * kAtomU, (atom0 + a) * 64, unit0, 0);
     }
     __syncwarp();
     // This CTA evaluates the gates of units unit0 + rank*UO + [0, UO); thread
-    // tid takes unit ui = tid % UO and batch rows b = tid / UO + k * (128 / UO).
+    // tid takes unit ui = tid % UO and batch rows b = tid / UO + k * BSTEP.
     const int ui = tid % UO;
-    const int bstep = kThreads / UO;
-    const int np = UO * kBatchPad / kThreads;
     const int j = unit0 + static_cast<int>(rank) * UO + ui;
     const float bh_r = p.b_hh[j], bh_z = p.b_hh[H + j], bh_n = p.b_hh[2 * H + j];
-    float hprev[kMaxPairs];
+    const float bi_r = p.b_ih ? p.b_ih[j] : 0.0f, bi_z = p.b_ih ? p.b_ih[H + j] : 0.0f,
+                bi_n = p.b_ih ? p.b_ih[2 * H + j] : 0.0f;
+    float hprev[NP];
 #pragma unroll
-    for (int k = 0; k < kMaxPairs; ++k) {
-        const int b = tid / UO + k * bstep;
-        hprev[k] = (k < np && p.h0 != nullptr && b < p.batch) ? p.h0[static_cast<size_t>(b) * H + j] : 0.0f;
-        if (k < np && b < p.batch) p.hx[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hprev[k]);
+    for (int k = 0; k < NP; ++k) {
+        const int b = tid / UO + k * BSTEP;
+        hprev[k] = (p.h0 != nullptr && b < p.batch) ? p.h0[static_cast<size_t>(b) * H + j] : 0.0f;
+        if (b < p.batch) p.hx[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hprev[k]);
     }
     fence_proxy_async_global();
     __syncwarp();
@@ -235,34 +258,80 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t idesc = idesc_bf16_f32(128, kBatchPad, false, false);
     int issued_phase = -1;  // last round whose h loads were issued (for the drain)
     // Input projection of a step (independent of h), loaded one step ahead so
-    // its memory latency is off the recurrence's critical path.
-    float gxr[kMaxPairs], gxz[kMaxPairs], gxn[kMaxPairs];
+    // its memory latency is off the recurrence's critical path: gx is one slab
+    // holding x W^T + b_ih (the GEMM's output), or KS slabs of K-rank partial
+    // products computed by the layer below.  The loads land in registers
+    // (KS x NP = 8 per gate whatever KS) and are summed, after b_ih and in
+    // rank order, only where the gates use them.
+    float gxr[KS * NP], gxz[KS * NP], gxn[KS * NP];
     auto load_gx = [&](int tt) {
 #pragma unroll
-        for (int k = 0; k < kMaxPairs; ++k) {
-            const int b = tid / UO + k * bstep;
-            if (k < np && b < p.batch && tt < p.T) {
-                const float *g = p.gx + (static_cast<size_t>(tt) * p.batch + b) * G + j;
-                gxr[k] = __ldg(g);
-                gxz[k] = __ldg(g + H);
-                gxn[k] = __ldg(g + 2 * H);
-            } else {
-                gxr[k] = gxz[k] = gxn[k] = 0.0f;
+        for (int k = 0; k < NP; ++k) {
+            const int b = tid / UO + k * BSTEP;
+            const float *g = p.gx + (static_cast<size_t>(tt) * p.batch + b) * G + j;
+#pragma unroll
+            for (int s = 0; s < KS; ++s) {
+                const int i = k * KS + s;
+                if (b < p.batch && tt < p.T && s < p.gx_parts) {
+                    const float *gs = g + static_cast<size_t>(s) * p.gx_slab;
+                    gxr[i] = __ldg(gs);
+                    gxz[i] = __ldg(gs + H);
+                    gxn[i] = __ldg(gs + 2 * H);
+                } else {
+                    gxr[i] = gxz[i] = gxn[i] = 0.0f;
+                }
             }
         }
+    };
+    auto sum_gx = [&](const float (&v)[KS * NP], float bias, int k) {
+        float a = bias;
+#pragma unroll
+        for (int s = 0; s < KS; ++s) a += v[k * KS + s];
+        return a;
     };
     load_gx(0);
     int last_t = -1;  // step whose h (in hprev) still has to go to h_out
 
-    // ---- recursive iteration, T times (in nph rounds each).
-    float zsave[kMaxPairs];  // update gate between the two rounds of a step
+    // ---- recursive iteration, T times (in nph rounds each), then, when the
+    // next layer's projection is fused in, a finish iteration that only
+    // multiplies its W by h_{T-1}.  Phase 0 of step t >= 1 multiplies the
+    // next layer's W by the h_{t-1} it has just loaded (the next layer's
+    // projection of step t - 1 over this CTA's K range) into a second
+    // accumulator, after the recurrent product: the h tile serves both.  That
+    // product's A operand starts 32 rows early, so W's r, z and n rows land in
+    // TMEM lanes 32-127, which warps 1-3 drain; warp 0 stays free to poll.
+    float zsave[NP];  // update gate between the two rounds of a step
     bool alive = true;
-    for (int t = 0; t < p.T && alive; ++t) {
-        for (int ph = 0; ph < nph; ++ph) {
+    int w_pending = -1;  // parity of the last next-layer product committed to w_done
+    int w_issued = -1;   // issuing thread: parity of its product not yet drained
+    auto issue_w = [&](uint32_t col, uint32_t wp) {
+        for (int a = 0; a < p.ka; ++a) {
+            // 32 rows (4 KB) before the atom: still inside shared memory (the
+            // U slice precedes W).
+            const uint32_t wa = smem_u32(sW + a * kAtomU) - 32u * 128u;
+            const uint32_t ha = smem_u32(sH + a * kAtomH);
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                umma_bf16(tmem_d + col, sdesc_sw128(wa + k * 32, 16, 1024), sdesc_sw128(ha + k * 32, 16, 1024),
+                          idesc, (a > 0 || k > 0) ? 1u : 0u);
+        }
+        umma_commit(w_done);
+        w_issued = static_cast<int>(wp);
+    };
+    const int t_end = p.T + (HN ? 1 : 0);
+    for (int t = 0; t < t_end && alive; ++t) {
+        const bool finish = t == p.T;
+        const int nround = finish ? 1 : nph;
+        for (int ph = 0; ph < nround; ++ph) {
             const int round = t * nph + ph;
             const uint32_t par = static_cast<uint32_t>(round & 1);
+            const bool wnow = HN && t > 0 && ph == 0;
+            const uint32_t wpar = static_cast<uint32_t>((t - 1) & 1);
+            const uint32_t wcol = 32u + 32u * wpar;
             if (tid == 0 && !*abort_flag) {
-                if (wait_counter(p.counter, static_cast<uint32_t>((round + 1) * p.n_cta), w)) {
+                // The next layer's product of the previous round still reads sH.
+                if (wait_counter(p.counter, static_cast<uint32_t>((round + 1) * p.n_cta), w) &&
+                    (w_pending < 0 || bounded_wait(w_done, static_cast<uint32_t>(w_pending), w, SITE_GRU_W))) {
                     fence_proxy_async_global();
                     const CUtensorMap *m = ph == 0 ? ((t & 1) ? &tmH1 : &tmH0) : ((t & 1) ? &tmR1 : &tmR0);
                     for (int q = 0; q < p.nq; ++q) {
@@ -273,15 +342,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             __syncwarp();
-            if (ph == 0) {
+            if (ph == 0 && !finish) {
                 // Off thread 0's path to the next counter poll: h_{t-1} to
                 // h_out and this step's input projection (still ahead of its
                 // use in the gates).
                 if (last_t >= 0) {
 #pragma unroll
-                    for (int k = 0; k < kMaxPairs; ++k) {
-                        const int b = tid / UO + k * bstep;
-                        if (k < np && b < p.batch)
+                    for (int k = 0; k < NP; ++k) {
+                        const int b = tid / UO + k * BSTEP;
+                        if (b < p.batch)
                             p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
                     }
                     last_t = -1;
@@ -295,6 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc_fence_after();
+                    if (finish) continue;
                     for (int a = q * p.qk; a < (q + 1) * p.qk; ++a) {
                         const uint32_t ua = smem_u32(sU + a * kAtomU);
                         const uint32_t ha = smem_u32(sH + a * kAtomH);
@@ -305,54 +375,58 @@ __global__ void __launch_bounds__(kThreads, 1)
                                       (a > 0 || k > 0) ? 1u : 0u);
                     }
                 }
-                if (ok) umma_commit(mma_done);
+                if (ok && !finish) umma_commit(mma_done);
+                if (ok && finish) issue_w(wcol, wpar);
             }
             __syncwarp();
-            // Block-uniform decision: every thread leaves at the same round.
-            if (!__syncthreads_and(bounded_wait(mma_done, par, w, SITE_GRU_MMA) ? 1 : 0)) {
-                alive = false;
-                break;
-            }
-            tc_fence_after();
-            // Push: row gate*32 + u of the partial product (TMEM lane = row)
-            // goes to the cluster CTA that owns unit u, into its slot for this
-            // source rank.  Round 0 of a reset-before step sends the r and z
-            // rows, round 1 the n rows.
-            const bool pushes = RB ? (ph == 0 ? warp < 2 : warp == 2) : warp < 3;
-            if (pushes) {
-                uint32_t r[32];
-                tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
-                tmem_ld_wait();
-                const uint32_t owner = static_cast<uint32_t>(lane / UO);
-                const int oui = lane % UO;
-                const uint32_t dst = mapa_shared(
-                    smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kRecvStride), owner);
-                const uint32_t rbar = mapa_shared(smem_u32(red_full), owner);
-                // Asynchronous remote stores: each counts its bytes on the
-                // owner's barrier, so nothing here waits for them to land.
+            if (!finish) {
+                // Block-uniform decision: every thread leaves at the same round.
+                if (!__syncthreads_and(bounded_wait(mma_done, par, w, SITE_GRU_MMA) ? 1 : 0)) {
+                    alive = false;
+                    break;
+                }
+                tc_fence_after();
+                // The next layer's product goes to the tensor pipe now that the
+                // recurrent one is done, issued by warp 3, which pushes nothing.
+                if (tid == 96 && wnow) issue_w(wcol, wpar);
+                // Push: row gate*32 + u of the partial product (TMEM lane = row)
+                // goes to the cluster CTA that owns unit u, into its slot for this
+                // source rank.  Round 0 of a reset-before step sends the r and z
+                // rows, round 1 the n rows.
+                const bool pushes = RB ? (ph == 0 ? warp < 2 : warp == 2) : warp < 3;
+                if (pushes) {
+                    uint32_t r[32];
+                    tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
+                    tmem_ld_wait(r);
+                    const uint32_t owner = static_cast<uint32_t>(lane / UO);
+                    const int oui = lane % UO;
+                    const uint32_t dst = mapa_shared(
+                        smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kRecvStride), owner);
+                    const uint32_t rbar = mapa_shared(smem_u32(red_full), owner);
+                    // Asynchronous remote stores: each counts its bytes on the
+                    // owner's barrier, so nothing here waits for them to land.
 #pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    st_async_f4(dst + c * 16,
-                                make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
-                                            __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
-                                rbar);
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (!__syncthreads_and(bounded_wait<true>(red_full, par, w, SITE_GRU_RED) ? 1 : 0)) {
-                alive = false;
-                break;
-            }
-            uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
-            uint16_t *rhx_t = p.rhx + static_cast<size_t>(t & 1) * kBatchPad * H;
+                    for (int c = 0; c < 8; ++c)
+                        st_async_f4(dst + c * 16,
+                                    make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
+                                                __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
+                                    rbar);
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (!__syncthreads_and(bounded_wait<true>(red_full, par, w, SITE_GRU_RED) ? 1 : 0)) {
+                    alive = false;
+                    break;
+                }
+                uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
+                uint16_t *rhx_t = p.rhx + static_cast<size_t>(t & 1) * kBatchPad * H;
 #pragma unroll
-            for (int k = 0; k < kMaxPairs; ++k) {
-                const int b = tid / UO + k * bstep;
-                if (k >= np || b >= p.batch) continue;
-                float ghr = bh_r, ghz = bh_z, ghn = bh_n;
+                for (int k = 0; k < NP; ++k) {
+                    const int b = tid / UO + k * BSTEP;
+                    if (b >= p.batch) continue;
+                    float ghr = bh_r, ghz = bh_z, ghn = bh_n;
 #pragma unroll
-                for (int s = 0; s < 4; ++s) {  // KS <= 4 sources, summed in rank order
-                    if (s < KS) {
+                    for (int s = 0; s < KS; ++s) {  // partials summed in rank order
                         const float *rs = recv + (s * 3 * UO + ui) * kRecvStride + b;
                         if (!RB || ph == 0) {
                             ghr += rs[0];
@@ -360,49 +434,80 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         if (!RB || ph == 1) ghn += rs[2 * UO * kRecvStride];
                     }
+                    if (!RB) {
+                        const float rg = sigmoidf_fast(sum_gx(gxr, bi_r, k) + ghr);
+                        const float zg = sigmoidf_fast(sum_gx(gxz, bi_z, k) + ghz);
+                        const float ng = tanhf_fast(sum_gx(gxn, bi_n, k) + rg * ghn);
+                        const float hn = (1.0f - zg) * ng + zg * hprev[k];
+                        hprev[k] = hn;
+                        hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
+                    } else if (ph == 0) {
+                        const float rg = sigmoidf_fast(sum_gx(gxr, bi_r, k) + ghr);
+                        zsave[k] = sigmoidf_fast(sum_gx(gxz, bi_z, k) + ghz);
+                        rhx_t[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(rg * hprev[k]);
+                    } else {
+                        const float ng = tanhf_fast(sum_gx(gxn, bi_n, k) + ghn);
+                        const float hn = (1.0f - zsave[k]) * ng + zsave[k] * hprev[k];
+                        hprev[k] = hn;
+                        hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
+                    }
                 }
-                if (!RB) {
-                    const float rg = sigmoidf_fast(gxr[k] + ghr);
-                    const float zg = sigmoidf_fast(gxz[k] + ghz);
-                    const float ng = tanhf_fast(gxn[k] + rg * ghn);
-                    const float hn = (1.0f - zg) * ng + zg * hprev[k];
-                    hprev[k] = hn;
-                    hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
-                } else if (ph == 0) {
-                    const float rg = sigmoidf_fast(gxr[k] + ghr);
-                    zsave[k] = sigmoidf_fast(gxz[k] + ghz);
-                    rhx_t[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(rg * hprev[k]);
-                } else {
-                    const float ng = tanhf_fast(gxn[k] + ghn);
-                    const float hn = (1.0f - zsave[k]) * ng + zsave[k] * hprev[k];
-                    hprev[k] = hn;
-                    hx_next[static_cast<size_t>(b) * H + j] = f32_to_bf16_rne(hn);
-                }
+                if (ph == nph - 1) last_t = t;  // hprev holds h_t, not yet in h_out
+                // Publish first (the release then waits only for the exchange-buffer
+                // stores), then write this step's h_t to h_out.
+                fence_proxy_async_global();
+                __syncthreads();
+                if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
+                    red_release_gpu_add(p.counter, 1u);
+                // recv is consumed: arm the barrier for the next round's partial
+                // rows (bytes that land before this are counted all the same).
+                if (tid == 0) mbar_arrive_expect_tx(red_full, round_bytes((ph + 1) % nph));
+                __syncwarp();
+                tc_fence_after();
             }
-            if (ph == nph - 1) last_t = t;  // hprev holds h_t, not yet in h_out
-            // Publish first (the release then waits only for the exchange-buffer
-            // stores), then write this step's h_t to h_out.
-            fence_proxy_async_global();
-            __syncthreads();
-            if (tid == 0 && static_cast<int>(blockIdx.x) != p.skip_publish_cta)
-                red_release_gpu_add(p.counter, 1u);
-            // recv is consumed: arm the barrier for the next round's partial
-            // rows (bytes that land before this are counted all the same).
-            if (tid == 0) mbar_arrive_expect_tx(red_full, round_bytes((ph + 1) % nph));
-            __syncwarp();
-            tc_fence_after();
+            if (wnow) {
+                // Next layer's projection of step t - 1 over this CTA's K range:
+                // TMEM lane 32 + gate*32 + u holds unit unit0 + u of that gate
+                // for the 32 batch rows; row b goes to slab `rank`.  The step
+                // counter is already published, so this is off the recurrence's
+                // critical path (thread 0 polls meanwhile, and waits for the
+                // product itself before it reloads sH).
+                w_pending = static_cast<int>(wpar);
+                if (warp >= 1) {
+                    if (__all_sync(0xffffffffu, bounded_wait(w_done, wpar, w, SITE_GRU_W) ? 1 : 0)) {
+                        tc_fence_after();
+                        uint32_t r[32];
+                        tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16) + wcol, r);
+                        tmem_ld_wait(r);
+                        float *dst = p.gxp_out + static_cast<size_t>(rank) * p.gx_slab +
+                                     static_cast<size_t>(t - 1) * p.batch * G + (warp - 1) * H + unit0 + lane;
+#pragma unroll
+                        for (int c = 0; c < 32; ++c)
+                            if (c < p.batch) dst[static_cast<size_t>(c) * G] = __uint_as_float(r[c]);
+                        w_issued = -1;
+                    }
+                    tc_fence_before();
+                }
+                __syncwarp();
+            }
         }
     }
     // h_T of the last step reached (or the step the loop left at).
     if (last_t >= 0) {
 #pragma unroll
-        for (int k = 0; k < kMaxPairs; ++k) {
-            const int b = tid / UO + k * bstep;
-            if (k < np && b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
+        for (int k = 0; k < NP; ++k) {
+            const int b = tid / UO + k * BSTEP;
+            if (b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
         }
     }
 
-    // ---- teardown: let issued copies land, release TMEM.
+    // ---- teardown: let issued copies and products land, release TMEM.
+    if ((tid == 32 || tid == 96) && w_issued >= 0) {  // only after an abort
+        const uint32_t a = smem_u32(w_done);
+        const unsigned long long t0 = globaltimer();
+        while (!mbar_try_wait(a, static_cast<uint32_t>(w_issued)))
+            if (globaltimer() - t0 > p.timeout_ns) break;
+    }
     if (tid == 0 && issued_phase >= 0 && *abort_flag) {
         for (int q = 0; q < p.nq; ++q) {
             const uint32_t a = smem_u32(&hbar[q]);
@@ -420,16 +525,40 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (KS > 1) cluster_sync_all();
     if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tmem_d, 32);
+        tmem_dealloc(tmem_d, tmem_cols);
     }
 }
 
 // K splits for a hidden size: each CTA's K range must be whole 64-wide atoms.
 int gru_splits(int H) { return (H % 256 == 0) ? 4 : (H % 128 == 0) ? 2 : 1; }
 
-size_t gru_smem_bytes(int H) { return static_cast<size_t>(gru_layout(H / gru_splits(H) / 64).total); }
+size_t gru_smem_bytes(int H, bool has_next = false) {
+    return static_cast<size_t>(gru_layout(H / gru_splits(H) / 64, has_next).total);
+}
 
 int gru_cta_count(int H) { return H / kGroup * gru_splits(H); }
+
+using GruKernel = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap,
+                           const CUtensorMap, const CUtensorMap, const GruParams);
+
+GruKernel gru_kernel_for(int ks) {
+    return ks == 4 ? gru_recurrent_kernel<4> : ks == 2 ? gru_recurrent_kernel<2> : gru_recurrent_kernel<1>;
+}
+
+// Opts every instantiation in to `bytes` of dynamic shared memory (once per process).
+int gru_smem_attr(int bytes) {
+    static std::mutex mu;
+    static bool done = false;
+    std::lock_guard<std::mutex> lk(mu);
+    if (done) return ISAM_OK;
+    const int ks[3] = {1, 2, 4};
+    for (int k : ks) {
+        cudaError_t e = cudaFuncSetAttribute(gru_kernel_for(k), cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
+    }
+    done = true;
+    return ISAM_OK;
+}
 
 int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
     if (*cap >= need) return ISAM_OK;
@@ -445,9 +574,12 @@ int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
 // Tensor maps of the recurrence: U as [3 gates][H rows][H] (box: 96 rows of
 // one group over one 64-wide K atom) and the two exchange buffers as
 // [H/64 atoms][32 batch rows][64] (box: one CTA's h piece).
-// Also the r * h exchange buffers' maps (tmR0 / tmR1 over rhx; skipped when null).
+// Also the r * h exchange buffers' maps (tmR0 / tmR1 over rhx; skipped when
+// null) and the next layer's input weights (tmWn over Wn, laid out as U;
+// skipped when null).
 int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, int H, CUtensorMap *tmU,
-                   CUtensorMap *tmH0, CUtensorMap *tmH1, CUtensorMap *tmR0, CUtensorMap *tmR1) {
+                   CUtensorMap *tmH0, CUtensorMap *tmH1, CUtensorMap *tmR0, CUtensorMap *tmR1,
+                   const uint16_t *Wn = nullptr, CUtensorMap *tmWn = nullptr) {
     int rc;
     const int ka = H / gru_splits(H) / 64;
     const int nq = (ka % 4 == 0) ? 4 : (ka % 3 == 0) ? 3 : (ka % 2 == 0) ? 2 : 1;
@@ -456,6 +588,7 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, i
         const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, static_cast<uint64_t>(H) * H * 2};
         const uint32_t box[3] = {64, kGroup, 3};
         if ((rc = make_tmap_3d_bf16(tmU, U, dims, strides, box))) return rc;
+        if (Wn && (rc = make_tmap_3d_bf16(tmWn, Wn, dims, strides, box))) return rc;
     }
     for (int i = 0; i < 2; ++i) {
         const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(H / 64)};
@@ -481,8 +614,8 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tm
 // driver accepts it with clusters, otherwise after checking that every
 // cluster fits at once (the step counter needs every CTA resident).
 int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tmH0,
-                     const CUtensorMap &tmH1, const CUtensorMap &tmR0, const CUtensorMap &tmR1, size_t smem,
-                     cudaStream_t stream) {
+                     const CUtensorMap &tmH1, const CUtensorMap &tmR0, const CUtensorMap &tmR1,
+                     const CUtensorMap &tmWn, size_t smem, cudaStream_t stream) {
     const int H = p.H;
     p.ks = gru_splits(H);
     p.ka = H / p.ks / 64;
@@ -504,27 +637,28 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
     cfg.stream = stream;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, tmR0, tmR1, p);
+    const GruKernel kern = gru_kernel_for(p.ks);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmU, tmH0, tmH1, tmR0, tmR1, tmWn, p);
     if (e == cudaSuccess) return ISAM_OK;
     (void)cudaGetLastError();
     cfg.numAttrs = 1;
     int max_clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&max_clusters, gru_recurrent_kernel, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
     if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveClusters(gru)");
     if (max_clusters * p.ks < p.n_cta)
         return set_error(ISAM_ERR_UNSUPPORTED,
                          "GRU recurrence: %d CTAs in clusters of %d cannot be co-resident (%d clusters fit)",
                          p.n_cta, p.ks, max_clusters);
-    e = cudaLaunchKernelEx(&cfg, gru_recurrent_kernel, tmU, tmH0, tmH1, tmR0, tmR1, p);
+    e = cudaLaunchKernelEx(&cfg, kern, tmU, tmH0, tmH1, tmR0, tmR1, tmWn, p);
     if (e != cudaSuccess) return cuda_error(e, "launch gru_recurrent_kernel");
     return ISAM_OK;
 }
 
 }  // namespace
 
-int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
-               const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
-               cudaStream_t stream, int reset_before) {
+int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before, const uint16_t *x,
+                     const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
+                     DeviceState &ds, cudaStream_t stream) {
     const int H = hidden;
     if (batch > kBatchPad || H % 64 != 0 || H > 1024 || H < 64)
         return set_error(ISAM_ERR_UNSUPPORTED,
@@ -538,14 +672,29 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
     const int n_cta = gru_cta_count(H);
     if (n_cta > ds.num_sms)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: %d CTAs cannot be co-resident", n_cta);
-    const size_t smem = gru_smem_bytes(H);
-    if (smem > static_cast<size_t>(ds.max_smem_optin))
+    const size_t smem_last = gru_smem_bytes(H, false);
+    const size_t smem_next = gru_smem_bytes(H, true);
+    if (smem_last > static_cast<size_t>(ds.max_smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: hidden too large for shared memory");
+    if (layers > 1 && smem_next > static_cast<size_t>(ds.max_smem_optin))
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_gru_forward_stack: hidden %d leaves no room for the next layer's "
+                         "weights beside the recurrent ones (%zu bytes of shared memory)",
+                         H, smem_next);
 
     int rc;
-    const size_t gx_bytes = static_cast<size_t>(T) * batch * 3 * H * sizeof(float);
-    if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_gx), &ds.gru_gx_bytes, gx_bytes,
+    const size_t seq_rows = static_cast<size_t>(T) * batch;
+    const size_t gx_floats = seq_rows * 3 * H;
+    if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_gx), &ds.gru_gx_bytes, gx_floats * sizeof(float),
                         "allocating the GRU projection workspace")))
+        return rc;
+    // Next layers' projections: two sets (read by layer l, written by layer l)
+    // of ks slabs, one per K rank.
+    const int ks = gru_splits(H);
+    if (layers > 1 &&
+        (rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_gxp), &ds.gru_gxp_bytes,
+                        2 * static_cast<size_t>(ks) * gx_floats * sizeof(float),
+                        "allocating the stacked GRU projection workspace")))
         return rc;
     // Exchange buffers: h (2 slots) then r * h (2 slots, the reset-before form).
     const size_t hx_bytes = static_cast<size_t>(4) * kBatchPad * H * sizeof(uint16_t);
@@ -560,45 +709,67 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
         cudaError_t e = cudaMalloc(&ds.gru_counter, 256);
         if (e != cudaSuccess) return cuda_error(e, "allocating the GRU step counter");
     }
+    if ((rc = gru_smem_attr(ds.max_smem_optin))) return rc;
 
-    // 1. Input projection for all steps: gx = x W^T + b_ih  (M = T*batch, N = 3H, K = H).
+    // 1. Input projection of the first layer for all steps: gx = x W_0^T + b_ih
+    //    (M = T*batch, N = 3H, K = H).
     GemmDesc g{T * batch, 3 * H, H, 0, 1, 1.0f, 0.0f, x, W, ds.gru_gx, b};
     GemmPlan plan;
     if ((rc = gemm_validate(g))) return rc;
     if ((rc = gemm_plan(g, ds, &plan))) return rc;
     if ((rc = gemm_launch(g, plan, ds, stream))) return rc;
 
-    // 2. Recurrence.
-    CUtensorMap tmU, tmH0, tmH1, tmR0, tmR1;
+    // 2. One recurrence per layer; layer l also computes layer l + 1's
+    //    projection (its slabs), which layer l + 1 sums as it goes.
+    const size_t wsz = static_cast<size_t>(3) * H * H;
     uint16_t *rhx = ds.gru_hx + static_cast<size_t>(2) * kBatchPad * H;
-    if ((rc = recurrent_maps(U, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1))) return rc;
-    GruParams p{};
-    p.rhx = rhx;
-    p.reset_before = reset_before ? 1 : 0;
-    p.T = T;
-    p.batch = batch;
-    p.H = H;
-    p.gx = ds.gru_gx;
-    p.b_hh = b + 3 * H;
-    p.h0 = h0;
-    p.h_out = h_out;
-    p.hx = ds.gru_hx;
-    p.counter = ds.gru_counter;
-    p.skip_publish_cta = -1;
-    if (const char *s = getenv("ISAM_DEBUG_GRU_SKIP_CTA")) p.skip_publish_cta = atoi(s);
-    p.timeout_ns = wait_timeout_ns();
-    p.err = ds.err_word;
-
-    cudaError_t e = cudaMemsetAsync(ds.gru_counter, 0, sizeof(uint32_t), stream);
-    if (e != cudaSuccess) return cuda_error(e, "clearing the GRU step counter");
-    static bool attr_set = false;
-    if (!attr_set) {
-        e = cudaFuncSetAttribute(gru_recurrent_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 ds.max_smem_optin);
-        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
-        attr_set = true;
+    for (int l = 0; l < layers; ++l) {
+        const bool has_next = l + 1 < layers;
+        const uint16_t *Ul = U + l * wsz;
+        const uint16_t *Wn = has_next ? W + (l + 1) * wsz : nullptr;
+        CUtensorMap tmU, tmH0, tmH1, tmR0, tmR1, tmWn;
+        if ((rc = recurrent_maps(Ul, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1, Wn, &tmWn)))
+            return rc;
+        GruParams p{};
+        p.T = T;
+        p.batch = batch;
+        p.H = H;
+        if (l == 0) {
+            p.gx = ds.gru_gx;
+            p.gx_parts = 1;
+            p.b_ih = nullptr;
+        } else {
+            p.gx = ds.gru_gxp + static_cast<size_t>((l - 1) & 1) * ks * gx_floats;
+            p.gx_parts = ks;
+            p.b_ih = b + static_cast<size_t>(l) * 6 * H;
+        }
+        p.gx_slab = gx_floats;
+        p.has_next = has_next ? 1 : 0;
+        p.gxp_out = has_next ? ds.gru_gxp + static_cast<size_t>(l & 1) * ks * gx_floats : nullptr;
+        p.b_hh = b + static_cast<size_t>(l) * 6 * H + 3 * H;
+        p.h0 = h0 ? h0 + static_cast<size_t>(l) * batch * H : nullptr;
+        p.h_out = h_out + static_cast<size_t>(l) * seq_rows * H;
+        p.hx = ds.gru_hx;
+        p.rhx = rhx;
+        p.reset_before = reset_before ? 1 : 0;
+        p.counter = ds.gru_counter;
+        p.skip_publish_cta = -1;
+        if (const char *sk = getenv("ISAM_DEBUG_GRU_SKIP_CTA")) p.skip_publish_cta = atoi(sk);
+        p.timeout_ns = wait_timeout_ns();
+        p.err = ds.err_word;
+        cudaError_t e = cudaMemsetAsync(ds.gru_counter, 0, sizeof(uint32_t), stream);
+        if (e != cudaSuccess) return cuda_error(e, "clearing the GRU step counter");
+        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, tmR0, tmR1, has_next ? tmWn : tmU,
+                                   has_next ? smem_next : smem_last, stream)))
+            return rc;
     }
-    return launch_recurrent(p, tmU, tmH0, tmH1, tmR0, tmR1, smem, stream);
+    return ISAM_OK;
+}
+
+int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
+               const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
+               cudaStream_t stream, int reset_before) {
+    return gru_stack_launch(1, T, batch, hidden, reset_before, x, W, U, b, h0, h_out, ds, stream);
 }
 
 }  // namespace isam
@@ -642,7 +813,6 @@ struct NoAllocDevice {
 };
 NoAllocDevice g_noalloc[64];
 std::mutex g_noalloc_mu;
-bool g_noalloc_attr = false;
 
 // Once per device, with that device current: the array's device address and
 // the device limits the launches need.  No allocation happens here.
@@ -714,12 +884,8 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
             if (rc) return rc;
         }
         nd = g_noalloc[dev];
-        if (!g_noalloc_attr) {
-            e = cudaFuncSetAttribute(gru_recurrent_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     nd.smem_optin);
-            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
-            g_noalloc_attr = true;
-        }
+        int rc0 = gru_smem_attr(nd.smem_optin);
+        if (rc0) return rc0;
     }
     const int n_cta = gru_cta_count(H);
     const size_t smem = gru_smem_bytes(H);
@@ -772,7 +938,12 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         p.err = err;
         p.rhx = hx;  // the reset-after form only
         p.reset_before = 0;
-        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, tmH0, tmH1, smem, stream))) return rc;
+        p.gx_parts = 1;
+        p.gx_slab = 0;
+        p.b_ih = nullptr;
+        p.has_next = 0;
+        p.gxp_out = nullptr;
+        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, tmH0, tmH1, tmU, smem, stream))) return rc;
     }
     // Report device-side timeouts of this call before returning.
     if ((e = cudaStreamSynchronize(stream)) != cudaSuccess)

@@ -27,6 +27,8 @@ struct DeviceState {
     uint16_t *gru_hx = nullptr;    // 2 x [32][H] bf16 hidden-state exchange
     size_t gru_hx_bytes = 0;
     uint32_t *gru_counter = nullptr;  // step counter (1 x uint32, padded)
+    float *gru_gxp = nullptr;      // 2 x [ks][T*batch][3H] fp32 stacked layers' projections
+    size_t gru_gxp_bytes = 0;
 };
 
 DeviceState *device_state(int *status);  // current device; null + status on failure
@@ -83,6 +85,9 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
 int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
                const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
                cudaStream_t s, int reset_before = 0);
+int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before, const uint16_t *x,
+                     const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
+                     DeviceState &ds, cudaStream_t stream);
 
 int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
                  const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t s);

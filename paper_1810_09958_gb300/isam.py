@@ -61,10 +61,12 @@ def load():
         lib.isam_gemm_grouped_fp8.argtypes = [i, P, P, P, P, P, P, P, P]
         lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
+        lib.isam_gru_forward_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
                      "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
                      "isam_gru_forward", "isam_gru_forward_reset_before",
+                     "isam_gru_forward_stack",
                      "isam_dwsep_conv"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
@@ -217,6 +219,24 @@ def gru_forward(T, batch, hidden, x, W, U, b, h0, h_out, reset_before=False) -> 
     _use_current_stream(lib)
     fn = lib.isam_gru_forward_reset_before if reset_before else lib.isam_gru_forward
     check(fn(T, batch, H, _ptr(x), _ptr(W), _ptr(U), _ptr(b), _ptr(h0), _ptr(h_out)))
+
+
+def gru_forward_stack(layers, T, batch, hidden, x, W, U, b, h0, h_out, reset_before=False) -> None:
+    """isam_gru_forward_stack: x [T,batch,H] bf16; W, U [layers,3H,H] bf16;
+    b [layers,6H], h0 [layers,batch,H] (or None), h_out [layers,T,batch,H] fp32."""
+    import torch
+    lib = load()
+    H, L = hidden, layers
+    _dev(x, torch.bfloat16, T * batch * H, "x")
+    _dev(W, torch.bfloat16, L * 3 * H * H, "W")
+    _dev(U, torch.bfloat16, L * 3 * H * H, "U")
+    _dev(b, torch.float32, L * 6 * H, "b")
+    if h0 is not None:
+        _dev(h0, torch.float32, L * batch * H, "h0")
+    _dev(h_out, torch.float32, L * T * batch * H, "h_out")
+    _use_current_stream(lib)
+    check(lib.isam_gru_forward_stack(L, T, batch, H, int(bool(reset_before)), _ptr(x), _ptr(W),
+                                     _ptr(U), _ptr(b), _ptr(h0), _ptr(h_out)))
 
 
 def dwsep_conv(N, H, W, Cin, Cout, x, dw_w, pw_w, out) -> None:

@@ -299,6 +299,18 @@ def gru_operands(T, batch, hidden, seed):
     return x, W, U, b, h0
 
 
+def gru_stack_operands(layers, T, batch, hidden, seed):
+    """A stack of GRU layers drawn as gru_operands per layer: x [T,batch,H];
+    W, U [layers,3H,H]; b [layers,6H]; h0 [layers,batch,H] U(-1,1)."""
+    x = gru_operands(T, batch, hidden, seed)[0]
+    per = [gru_operands(1, 1, hidden, stream_seed(seed, 100 + l)) for l in range(layers)]
+    W = np.stack([q[1] for q in per])
+    U = np.stack([q[2] for q in per])
+    b = np.stack([q[3] for q in per])
+    h0 = f32_uniform(stream_seed(seed, 99), (layers, batch, hidden))
+    return x, W, U, b, h0
+
+
 def dwsep_operands(N, H, W, Cin, Cout, seed):
     """x NHWC bf16 N(0,1); dw_w [3,3,Cin] bf16 U(+-1/3) (fan-in 9);
     pw_w [Cin,Cout] bf16 U(+-1/sqrt(Cin))."""

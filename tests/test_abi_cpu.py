@@ -49,6 +49,9 @@ def test_gru_and_dwsep_reject_bad_args_without_cuda(lib):
     assert lib.isam_gru_forward(1, 1, 128, None, p, p, p, None, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_gru_forward_reset_before(1, 0, 128, p, p, p, p, None, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_gru_forward_reset_before(1, 1, 128, p, p, None, p, None, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gru_forward_stack(0, 1, 1, 128, 0, p, p, p, p, None, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gru_forward_stack(2, 1, 1, 128, 2, p, p, p, p, None, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gru_forward_stack(2, 1, 1, 128, 0, p, p, p, None, None, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_dwsep_conv(1, 0, 4, 16, 16, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_dwsep_conv(1, 4, 4, 16, 16, p, None, p, p) == isam.ISAM_ERR_INVALID_ARG
 
