@@ -151,6 +151,15 @@ int isam_gemm_grouped_fp8(int count, const int *M, const int *N, const int *K, c
 int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta, int *out);
 
 /*
+ * isam_gemm_plan_info with two more outputs (out: host, 8 ints): out[0..5]
+ * as above, out[6] tile height (128, or 256 for a CTA-pair plan), out[7] CTAs
+ * whose tensor cores issue one MMA together (1, or 2: the two CTAs of a
+ * cluster each hold 128 rows of A and half the tile's columns of B, and one
+ * of them issues M = 256 MMAs over both; the pair's tile is 256 x BN).
+ */
+int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta, int *out);
+
+/*
  * GRU forward inference over T steps (input size == hidden).
  *
  * The recurrent model the paper schedules with a priming, a recursive and a

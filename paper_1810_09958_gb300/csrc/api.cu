@@ -350,6 +350,20 @@ int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta,
     return ISAM_OK;
 }
 
+int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta, int *out) {
+    int rc = isam_gemm_plan_info(M, N, K, transA, transB, beta, out);
+    if (rc) return rc;
+    GemmDesc g{M, N, K, transA, transB, 1.0f, beta, reinterpret_cast<const uint16_t *>(16),
+               reinterpret_cast<const uint16_t *>(16), reinterpret_cast<float *>(16), nullptr};
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    GemmPlan plan;
+    if ((rc = gemm_plan(g, *ds, &plan))) return rc;
+    out[6] = plan.pair ? 256 : 128;
+    out[7] = plan.pair ? 2 : 1;
+    return ISAM_OK;
+}
+
 int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x, const isam_bf16 *W,
                      const isam_bf16 *U, const float *b, const float *h0, float *h_out) {
     if (T < 1 || batch < 1 || hidden < 1)

@@ -724,6 +724,7 @@ int gemm_validate(const GemmDesc &g) {
 }
 
 int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
+    if (!getenv("ISAM_FORCE_TILE") && gemm_pair_plan(g, ds, plan)) return ISAM_OK;
     const bool b_mn = g.transB == 0;
     const int nsm = ds.num_sms;
     const int kb = ceil_div(g.K, g.fp8 ? 2 * kBK : kBK);
@@ -774,6 +775,7 @@ int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
 }
 
 int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t stream) {
+    if (plan.pair) return gemm_pair_launch(g, plan, ds, stream);
     const bool a_mn = g.transA == 1;
     const bool b_mn = g.transB == 0;
     CUtensorMap ta, tb, tc;

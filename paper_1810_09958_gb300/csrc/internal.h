@@ -72,11 +72,16 @@ struct GemmPlan {
     int grid;     // CTAs launched (persistent)
     size_t smem;  // dynamic shared memory bytes
     double est_us;
+    int pair = 0; // 1: 256 x 256 tiles on CTA pairs (cta_group::2), see gemm_pair.cu
 };
 
 int gemm_validate(const GemmDesc &g);
 int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan);
 int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t s);
+// The CTA-pair kernel: fills *plan and returns 1 when the problem suits it
+// (K-major A, bf16, N % 4 == 0, at least one 256 x 256 tile per SM pair).
+int gemm_pair_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan);
+int gemm_pair_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t s);
 
 // Independent GEMMs in one persistent launch (1 <= count <= 64).
 int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStream_t s);

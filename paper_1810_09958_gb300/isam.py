@@ -56,6 +56,7 @@ def load():
         lib.isam_shutdown.argtypes = []
         lib.isam_gemm.argtypes = [i, i, i, i, i, f, P, P, f, P]
         lib.isam_gemm_plan_info.argtypes = [i, i, i, i, i, f, P]
+        lib.isam_gemm_plan_info2.argtypes = [i, i, i, i, i, f, P]
         lib.isam_gemm_grouped.argtypes = [i, P, P, P, P, P, P, P, P, P, P]
         lib.isam_gemm_fp8.argtypes = [i, i, i, f, P, P, f, P]
         lib.isam_gemm_grouped_fp8.argtypes = [i, P, P, P, P, P, P, P, P]
@@ -64,7 +65,7 @@ def load():
         lib.isam_gru_forward_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
-                     "isam_gemm_plan_info", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
+                     "isam_gemm_plan_info", "isam_gemm_plan_info2", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
                      "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_gru_forward_stack",
                      "isam_dwsep_conv"):
@@ -198,9 +199,9 @@ def gemm_grouped(problems) -> None:
 def gemm_plan(M, N, K, transA, transB, beta=0.0) -> dict:
     """The tile plan the library's cost model picks (nothing is launched)."""
     lib = load()
-    out = (ctypes.c_int * 6)()
-    check(lib.isam_gemm_plan_info(M, N, K, int(transA), int(transB), float(beta), out))
-    return dict(zip(("BN", "split", "stages", "group_m", "grid", "smem"), list(out)))
+    out = (ctypes.c_int * 8)()
+    check(lib.isam_gemm_plan_info2(M, N, K, int(transA), int(transB), float(beta), out))
+    return dict(zip(("BN", "split", "stages", "group_m", "grid", "smem", "tile_m", "cta_pair"), list(out)))
 
 
 def gru_forward(T, batch, hidden, x, W, U, b, h0, h_out, reset_before=False) -> None:
