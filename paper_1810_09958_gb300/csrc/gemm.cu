@@ -637,14 +637,17 @@ constexpr double kLaunchGapUs = 1.3;
 constexpr double kTileOverheadUs = 0.3;
 constexpr double kSplitTailUs = 1.5;   // push + owner reduce of a split tile
 
-double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out) {
+double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int cluster_cap, int *grid_out) {
     const int m_tiles = ceil_div(g.M, kBM);
     const int n_tiles = ceil_div(g.N, BN);
     const long long tiles = static_cast<long long>(m_tiles) * n_tiles;
     const int eb = g.fp8 ? 1 : 2;                  // bytes per operand element
     const int kb = ceil_div(g.K, kBK * 2 / eb);     // 128-byte K atoms
     const int kb_per = ceil_div(kb, S);
-    const int clusters_max = std::max(1, num_sms / S);
+    // Clusters that can be resident at once: the CTAs of a cluster share one
+    // GPC, so fewer clusters of 4 or 8 fit than num_sms / S; a cluster
+    // beyond that would wait for a whole resident one to finish.
+    const int clusters_max = std::max(1, std::min(num_sms / S, cluster_cap));
     const int clusters = static_cast<int>(std::min<long long>(tiles, clusters_max));
     *grid_out = clusters * S;
     const int tiles_per_cluster = ceil_div(tiles, clusters);
@@ -663,6 +666,49 @@ double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int *grid_out)
     const double tail = (S > 1 ? kSplitTailUs : 0.0) + kBM * BN * 4.0 / S / kSmStoreBw * 1e6;
     return kFirstDataUs + std::max({t_steady, t_hbm, t_flops}) + tail + kLaunchGapUs;
 }
+
+int ensure_smem_attr(KernelFn fn, size_t smem);
+
+}  // namespace
+
+// Clusters of `size` CTAs (one CTA per SM, as every GEMM plan here uses) that
+// the device keeps resident at once, from cudaOccupancyMaxActiveClusters;
+// cached per device.  Falls back to num_sms / size if the query fails.
+int gemm_cluster_capacity(const DeviceState &ds, int size) {
+    if (size <= 1) return ds.num_sms;
+    const int idx = size == 2 ? 0 : size == 4 ? 1 : size == 8 ? 2 : -1;
+    if (idx < 0 || ds.device < 0 || ds.device >= 64) return std::max(1, ds.num_sms / size);
+    static std::mutex mu;
+    static int cache[64][3] = {};
+    std::lock_guard<std::mutex> lk(mu);
+    int &c = cache[ds.device][idx];
+    if (c > 0) return c;
+    int n = 0;
+    KernelFn fn = pick_kernel(128, false, false);
+    if (ensure_smem_attr(fn, static_cast<size_t>(ds.max_smem_optin)) == ISAM_OK) {
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = static_cast<unsigned>(size);
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(static_cast<unsigned>(size * std::max(1, ds.num_sms / size)), 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = static_cast<size_t>(ds.max_smem_optin);
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) {
+            (void)cudaGetLastError();
+            n = 0;
+        }
+    } else {
+        (void)cudaGetLastError();
+    }
+    c = n > 0 ? std::min(n, ds.num_sms / size) : std::max(1, ds.num_sms / size);
+    return c;
+}
+
+namespace {
 
 struct AttrCache {
     std::mutex mu;
@@ -738,7 +784,7 @@ int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
             if (S > kb) continue;
             if (S > 1 && BN > 128) continue;
             int grid = 0;
-            const double t = estimate_us(g, BN, S, nsm, &grid);
+            const double t = estimate_us(g, BN, S, nsm, gemm_cluster_capacity(ds, S), &grid);
             if (t < best * 0.999) {
                 best = t;
                 bp.BN = BN;
@@ -759,7 +805,7 @@ int gemm_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
                 bp.BN = fbn;
                 bp.split = fs;
                 bp.ka = ka;
-                estimate_us(g, fbn, fs, nsm, &bp.grid);
+                estimate_us(g, fbn, fs, nsm, gemm_cluster_capacity(ds, fs), &bp.grid);
                 if (fst >= 2) bp.stages = fst;
             }
         }

@@ -377,7 +377,7 @@ int gemm_pair_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan) {
     if (const char *s = getenv("ISAM_NO_PAIR"))
         if (s[0] == '1') return 0;
     const long long tiles = static_cast<long long>((g.M + kPM - 1) / kPM) * ((g.N + kPN - 1) / kPN);
-    const int pairs = ds.num_sms / 2;
+    const int pairs = gemm_cluster_capacity(ds, 2);  // pairs resident at once
     if (pairs < 1 || tiles < pairs) return 0;  // smaller problems spread better as 128-row tiles
     int st = 8;
     while (st > 2 && pair_smem_bytes(st) > static_cast<size_t>(ds.max_smem_optin)) --st;

@@ -81,6 +81,8 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
 // The CTA-pair kernel: fills *plan and returns 1 when the problem suits it
 // (K-major A, bf16, N % 4 == 0, at least one 256 x 256 tile per SM pair).
 int gemm_pair_plan(const GemmDesc &g, const DeviceState &ds, GemmPlan *plan);
+// Clusters of `size` CTAs (one per SM) resident at once on this device.
+int gemm_cluster_capacity(const DeviceState &ds, int size);
 int gemm_pair_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaStream_t s);
 
 // Independent GEMMs in one persistent launch (1 <= count <= 64).
