@@ -228,13 +228,19 @@ int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 
  *   h_out  [layers][T][batch][hidden]    fp32, every layer's states; layer
  *                                        layers - 1 is the stack's output
  *
- * Only layer 0's input projection is a separate GEMM.  Layer l's persistent
- * kernel also keeps its K quarter of layer l + 1's W resident and multiplies
- * it by the bf16(h_{t-1}) tile it loads for its own recurrent product, so
- * layer l + 1's projection is computed while layer l runs (one extra round
- * at the end covers h_{T-1}); layer l + 1 reads it as per-K-rank partial
- * sums (fixed order: deterministic).  The next layer therefore sees
- * bf16(h^l_t), as the recurrent product sees bf16(h_{t-1}).
+ With the reset gate after the product and hidden a multiple of 256, layers
+ * run in pairs in one persistent kernel: in round r it advances the lower
+ * layer to step r and the upper one to step r - 1, computing the upper
+ * layer's input projection from the same bf16 tile of the lower layer's
+ * states (T + 1 rounds for two layers); between pairs, and for an odd last
+ * layer, the states below are rounded to bf16 and projected by the GEMM.
+ * Otherwise (the reset-before form, other hidden sizes) layer l's kernel
+ * keeps its K quarter of layer l + 1's W resident and multiplies it by the
+ * bf16(h_{t-1}) tile it loads for its own recurrent product, so layer
+ * l + 1's projection is computed while layer l runs (one extra round covers
+ * h_{T-1}); layer l + 1 reads it as per-K-rank partial sums (fixed order:
+ * deterministic).  Either way the next layer sees bf16(h^l_t), as the
+ * recurrent product sees bf16(h_{t-1}).
  *
  * Supported: as isam_gru_forward; with layers > 1, also the shared memory
  * for both weight slices, which excludes hidden 576, 704, 832 and 960

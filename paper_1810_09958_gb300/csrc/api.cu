@@ -247,6 +247,7 @@ int isam_shutdown(void) {
         cudaFree(ds->gru_hx);
         cudaFree(ds->gru_counter);
         cudaFree(ds->gru_gxp);
+        cudaFree(ds->gru_xb);
         delete ds;
         g_dev[d] = nullptr;
     }

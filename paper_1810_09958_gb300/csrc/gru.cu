@@ -24,12 +24,14 @@
 //      low: at this size each M = 128 instruction costs about the same
 //      whatever its N, so the step time is set by instructions per CTA.
 //      Every wait is bounded in time.
+#include <algorithm>
 #include <cstdio>
 #include <cstdlib>
 #include <mutex>
 
 #include <cuda_bf16.h>
 
+#include "gru_common.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -51,7 +53,6 @@ constexpr int kRecvBytes = kRowsG * kRecvStride * 4;
 constexpr int kMaxPieces = 4;
 
 enum : uint32_t {
-    SITE_GRU_STEP = 0x201,
     SITE_GRU_U = 0x202,
     SITE_GRU_H = 0x203,
     SITE_GRU_MMA = 0x204,
@@ -84,43 +85,6 @@ struct GruParams {
     unsigned long long timeout_ns;
     uint32_t *err;
 };
-
-__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
-__device__ __forceinline__ void red_release_gpu_add(uint32_t *p, uint32_t v) {
-    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-// Branch-free gate nonlinearities (a data-dependent branch in the gate code
-// would split warps for the rest of the step): __expf and the approximate
-// __fdividef, exact in the limits (exp overflow gives 0 and +-1).
-__device__ __forceinline__ float sigmoidf_fast(float v) { return __fdividef(1.0f, 1.0f + __expf(-v)); }
-// tanh(v) = 1 - 2 / (1 + e^{2v})
-__device__ __forceinline__ float tanhf_fast(float v) { return 1.0f - __fdividef(2.0f, 1.0f + __expf(2.0f * v)); }
-
-__device__ __forceinline__ uint16_t f32_to_bf16_rne(float f) {
-    return __bfloat16_as_ushort(__float2bfloat16_rn(f));
-}
-
-// Spins (bounded) until the step counter reaches target.
-__device__ bool wait_counter(const uint32_t *counter, uint32_t target, const WaitCtx &w) {
-    if (ld_acquire_gpu(counter) >= target) return true;
-    const unsigned long long t0 = globaltimer();
-    for (uint32_t i = 1;; ++i) {
-        if (ld_acquire_gpu(counter) >= target) return true;
-        if ((i & 15u) == 0u) {
-            if (*w.abort_flag) return false;
-            if (globaltimer() - t0 > w.timeout_ns) {
-                report_timeout(w, SITE_GRU_STEP);
-                return false;
-            }
-        }
-    }
-}
 
 struct GruLayout {
     int off_u, off_w, off_h, off_recv, off_bars, total;
@@ -656,6 +620,21 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
 
 }  // namespace
 
+namespace {
+
+// bf16 copy of a layer's states (the next layer pair's GEMM input); n is a
+// multiple of 4, both pointers 16-byte aligned.
+__global__ void __launch_bounds__(256) states_to_bf16_kernel(const float4 *in, uint2 *out, size_t n4) {
+    for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n4;
+         i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const float4 v = in[i];
+        out[i] = make_uint2(static_cast<uint32_t>(f32_to_bf16_rne(v.x)) | (static_cast<uint32_t>(f32_to_bf16_rne(v.y)) << 16),
+                            static_cast<uint32_t>(f32_to_bf16_rne(v.z)) | (static_cast<uint32_t>(f32_to_bf16_rne(v.w)) << 16));
+    }
+}
+
+}  // namespace
+
 int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before, const uint16_t *x,
                      const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
                      DeviceState &ds, cudaStream_t stream) {
@@ -711,30 +690,32 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     }
     if ((rc = gru_smem_attr(ds.max_smem_optin))) return rc;
 
-    // 1. Input projection of the first layer for all steps: gx = x W_0^T + b_ih
-    //    (M = T*batch, N = 3H, K = H).
-    GemmDesc g{T * batch, 3 * H, H, 0, 1, 1.0f, 0.0f, x, W, ds.gru_gx, b};
-    GemmPlan plan;
-    if ((rc = gemm_validate(g))) return rc;
-    if ((rc = gemm_plan(g, ds, &plan))) return rc;
-    if ((rc = gemm_launch(g, plan, ds, stream))) return rc;
-
-    // 2. One recurrence per layer; layer l also computes layer l + 1's
-    //    projection (its slabs), which layer l + 1 sums as it goes.
     const size_t wsz = static_cast<size_t>(3) * H * H;
     uint16_t *rhx = ds.gru_hx + static_cast<size_t>(2) * kBatchPad * H;
-    for (int l = 0; l < layers; ++l) {
-        const bool has_next = l + 1 < layers;
-        const uint16_t *Ul = U + l * wsz;
+    // Input projection of layer l for all steps: gx = in W_l^T + b_ih_l
+    // (M = T*batch, N = 3H, K = H).
+    auto project = [&](const uint16_t *in, int l) {
+        GemmDesc g{T * batch, 3 * H, H, 0, 1, 1.0f, 0.0f, in, W + l * wsz, ds.gru_gx, b + static_cast<size_t>(l) * 6 * H};
+        GemmPlan plan;
+        int r;
+        if ((r = gemm_validate(g))) return r;
+        if ((r = gemm_plan(g, ds, &plan))) return r;
+        return gemm_launch(g, plan, ds, stream);
+    };
+    // One layer's recurrence.  Its projection is either ds.gru_gx (one slab,
+    // b_ih included) or, for layer l > 0 of the per-layer chain, the slabs the
+    // layer below computed; with has_next it computes layer l + 1's slabs.
+    auto recur = [&](int l, bool has_next, bool gx_from_below) {
         const uint16_t *Wn = has_next ? W + (l + 1) * wsz : nullptr;
         CUtensorMap tmU, tmH0, tmH1, tmR0, tmR1, tmWn;
-        if ((rc = recurrent_maps(Ul, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1, Wn, &tmWn)))
-            return rc;
+        int r;
+        if ((r = recurrent_maps(U + l * wsz, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1, Wn, &tmWn)))
+            return r;
         GruParams p{};
         p.T = T;
         p.batch = batch;
         p.H = H;
-        if (l == 0) {
+        if (!gx_from_below) {
             p.gx = ds.gru_gx;
             p.gx_parts = 1;
             p.b_ih = nullptr;
@@ -759,10 +740,55 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
         p.err = ds.err_word;
         cudaError_t e = cudaMemsetAsync(ds.gru_counter, 0, sizeof(uint32_t), stream);
         if (e != cudaSuccess) return cuda_error(e, "clearing the GRU step counter");
-        if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, tmR0, tmR1, has_next ? tmWn : tmU,
-                                   has_next ? smem_next : smem_last, stream)))
+        return launch_recurrent(p, tmU, tmH0, tmH1, tmR0, tmR1, has_next ? tmWn : tmU,
+                                has_next ? smem_next : smem_last, stream);
+    };
+
+    // Pairs of layers in one kernel (gru_wave.cu): layer l + 1 advances one
+    // step behind layer l, its projection computed from the same h tiles.
+    // Between pairs (and for an odd last layer) the layer below's states are
+    // rounded to bf16 and projected by the GEMM.
+    const char *nw = getenv("ISAM_NO_WAVE");
+    if (layers >= 2 && !reset_before && !(nw && nw[0] == '1') && gru_wave_supported(H, batch, ds)) {
+        if (layers > 2 && (rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_xb), &ds.gru_xb_bytes,
+                                          seq_rows * H * sizeof(uint16_t), "allocating the GRU layer-input buffer")))
             return rc;
+        for (int l = 0; l < layers;) {
+            const uint16_t *in = x;
+            if (l > 0) {
+                const size_t n4 = seq_rows * H / 4;
+                const int blocks = static_cast<int>(std::min<size_t>((n4 + 255) / 256, static_cast<size_t>(ds.num_sms) * 8));
+                states_to_bf16_kernel<<<blocks, 256, 0, stream>>>(
+                    reinterpret_cast<const float4 *>(h_out + static_cast<size_t>(l - 1) * seq_rows * H),
+                    reinterpret_cast<uint2 *>(ds.gru_xb), n4);
+                cudaError_t e = cudaGetLastError();
+                if (e != cudaSuccess) return cuda_error(e, "launch states_to_bf16_kernel");
+                in = ds.gru_xb;
+            }
+            if ((rc = project(in, l))) return rc;
+            if (l + 1 < layers) {
+                const size_t so = seq_rows * H;
+                if ((rc = gru_wave_launch(T, batch, H, ds.gru_gx, U + l * wsz, W + (l + 1) * wsz, U + (l + 1) * wsz,
+                                          b + static_cast<size_t>(l) * 6 * H, b + static_cast<size_t>(l + 1) * 6 * H,
+                                          h0 ? h0 + static_cast<size_t>(l) * batch * H : nullptr,
+                                          h0 ? h0 + static_cast<size_t>(l + 1) * batch * H : nullptr,
+                                          h_out + static_cast<size_t>(l) * so, h_out + static_cast<size_t>(l + 1) * so,
+                                          ds.gru_hx, rhx, ds.gru_counter, ds, stream)))
+                    return rc;
+                l += 2;
+            } else {
+                if ((rc = recur(l, false, false))) return rc;
+                l += 1;
+            }
+        }
+        return ISAM_OK;
     }
+
+    // One recurrence per layer; layer l also computes layer l + 1's
+    // projection (its slabs), which layer l + 1 sums as it goes.
+    if ((rc = project(x, 0))) return rc;
+    for (int l = 0; l < layers; ++l)
+        if ((rc = recur(l, l + 1 < layers, l > 0))) return rc;
     return ISAM_OK;
 }
 

@@ -29,6 +29,8 @@ struct DeviceState {
     uint32_t *gru_counter = nullptr;  // step counter (1 x uint32, padded)
     float *gru_gxp = nullptr;      // 2 x [ks][T*batch][3H] fp32 stacked layers' projections
     size_t gru_gxp_bytes = 0;
+    uint16_t *gru_xb = nullptr;    // [T*batch][H] bf16 states of a layer (next pair's input)
+    size_t gru_xb_bytes = 0;
 };
 
 DeviceState *device_state(int *status);  // current device; null + status on failure
@@ -92,6 +94,14 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
 int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
                const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,
                cudaStream_t s, int reset_before = 0);
+// Two stacked layers in one persistent kernel (reset gate after the
+// product, hidden a multiple of 256): layer a's projection gx_a is given,
+// layer b's comes from W_b and layer a's states inside the kernel.
+bool gru_wave_supported(int H, int batch, const DeviceState &ds);
+int gru_wave_launch(int T, int batch, int H, const float *gx_a, const uint16_t *U_a, const uint16_t *W_b,
+                    const uint16_t *U_b, const float *b_a, const float *b_b, const float *h0_a,
+                    const float *h0_b, float *out_a, float *out_b, uint16_t *hx_a, uint16_t *hx_b,
+                    uint32_t *counter, DeviceState &ds, cudaStream_t stream);
 int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before, const uint16_t *x,
                      const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
                      DeviceState &ds, cudaStream_t stream);
