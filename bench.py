@@ -395,8 +395,9 @@ def hot_path_rows(isam, dev, peaks):
         "us_per_step": round(ms * 1e3 / T, 3), "tflops": round(tf, 2),
         "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4)}
     del x, W, U, b, h0, hout
-    # Two stacked layers (the second layer's projection fused into the first
-    # layer's recurrence), against the same stack as one call per layer.
+    # Two stacked layers (one persistent kernel advancing both, the upper
+    # layer's projection computed from the lower layer's tiles), against the
+    # same stack as one call per layer.
     L = 2
     x = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 5, 1), T * batch * H, dev)
     W = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 5, 2), L * 3 * H * H, dev, -s, s)
@@ -417,8 +418,8 @@ def hot_path_rows(isam, dev, peaks):
         "ms": round(ms, 4), "layer_timesteps_per_s": round(L * T / (ms / 1e3), 1),
         "us_per_layer_step": round(ms * 1e3 / (L * T), 3),
         "per_layer_calls_ms": round(ms_pl, 4),
-        "what": "2 layers in one isam_gru_forward_stack call; per_layer_calls_ms: two "
-                "isam_gru_forward calls with a bf16 cast (torch) between"}
+        "what": "2 layers in one isam_gru_forward_stack call (both layers in one kernel); "
+                "per_layer_calls_ms: two isam_gru_forward calls with a bf16 cast (torch) between"}
     del x, W, U, b, hout, x1
     # Separable depthwise layer.
     N, Hh, Ww, Cin, Cout = 32, 56, 56, 128, 256
