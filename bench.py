@@ -10,7 +10,8 @@ GEMM finds its operands in L2 from the step before).  A step is one
 isam_gemm_grouped call over the 32 problems (one persistent launch).
 
 value  = GEMM TFLOP/s over the sweep (all ranks' flops / max rank time).
-e2e    = the same through host buffers: pinned host -> device copies of every
+e2e    = the same through host buffers (two device operand sets, so one step's
+         input copies overlap the previous step's GEMM): pinned host -> device copies of every
          operand, the grouped call, device -> host copies of every result.
 roofline: the sweep's kernel (gemm_group_kernel) is HBM-bound: algorithmic
          bytes (2MK + 2KN + 4MN per GEMM, summed) / per-launch CUDA-event time,
@@ -261,7 +262,10 @@ def time_grouped(isam, probs, steps, warmup):
 def time_e2e(isam, probs, steps, warmup):
     """The sweep through host buffers: per step, pinned host -> device copies of
     every operand, one isam_gemm_grouped launch, device -> host copies of every
-    result, all on the current stream."""
+    result.  Steps alternate between two device operand sets so that the input
+    copies of step k + 1 (copy stream) overlap the GEMM and the result copies
+    of step k; events order each set's copies, GEMM and read-back, and every
+    step still moves its own inputs in and its result out."""
     import torch
     host = []
     for p in probs:
@@ -269,27 +273,57 @@ def time_e2e(isam, probs, steps, warmup):
                      "C": torch.empty(p["M"] * p["N"], dtype=torch.float32).pin_memory()})
     h2d = sum(h["A"].numel() * 2 + h["B"].numel() * 2 for h in host)
     d2h = sum(h["C"].numel() * 4 for h in host)
-    call = isam.GroupedGemm([(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, p["A"], p["B"], 0.0, p["C"])
-                             for p in probs])
+    sets = [[{"A": p["A"], "B": p["B"], "C": p["C"]} for p in probs],
+            [{"A": torch.empty_like(p["A"]), "B": torch.empty_like(p["B"]), "C": torch.empty_like(p["C"])}
+             for p in probs]]
+    calls = [isam.GroupedGemm([(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, d["A"], d["B"], 0.0, d["C"])
+                               for p, d in zip(probs, ds)]) for ds in sets]
+    s_in, s_run, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev = {k: [torch.cuda.Event(), torch.cuda.Event()] for k in ("in", "run", "out")}
+    first = [True, True]
 
-    def one():
-        for p, h in zip(probs, host):
-            p["A"].copy_(h["A"], non_blocking=True)
-            p["B"].copy_(h["B"], non_blocking=True)
-        call()
-        for p, h in zip(probs, host):
-            h["C"].copy_(p["C"], non_blocking=True)
+    def one(k):
+        i = k & 1
+        with torch.cuda.stream(s_in):
+            if not first[i]:
+                s_in.wait_event(ev["run"][i])  # set i's operands are no longer read
+            for p, h in zip(sets[i], host):
+                p["A"].copy_(h["A"], non_blocking=True)
+                p["B"].copy_(h["B"], non_blocking=True)
+            ev["in"][i].record(s_in)
+        with torch.cuda.stream(s_run):
+            s_run.wait_event(ev["in"][i])
+            if not first[i]:
+                s_run.wait_event(ev["out"][i])  # set i's results have been read back
+            calls[i]()
+            ev["run"][i].record(s_run)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(ev["run"][i])
+            for p, h in zip(sets[i], host):
+                h["C"].copy_(p["C"], non_blocking=True)
+            ev["out"][i].record(s_out)
+        first[i] = False
 
-    for _ in range(warmup):
-        one()
+    def join(stream):
+        for s in (s_in, s_run, s_out):
+            e = torch.cuda.Event()
+            e.record(s)
+            stream.wait_event(e)
+
+    main = torch.cuda.current_stream()
+    for k in range(warmup):
+        one(k)
     torch.cuda.synchronize()
     barrier()
     start = torch.cuda.Event(enable_timing=True)
     end = torch.cuda.Event(enable_timing=True)
-    start.record()
-    for _ in range(steps):
-        one()
-    end.record()
+    start.record(main)
+    for s in (s_in, s_run, s_out):
+        s.wait_stream(main)
+    for k in range(steps):
+        one(warmup + k)
+    join(main)
+    end.record(main)
     torch.cuda.synchronize()
     isam.sync()
     return start.elapsed_time(end), h2d, d2h
@@ -722,7 +756,7 @@ def main(argv=None):
                                    "timed-region CUDA events on the replay stream / steps"},
             "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-                    "what": "pinned host operands copied in, isam_gemm_grouped, results copied out"},
+                    "what": "pinned host operands copied in, isam_gemm_grouped, results copied out; two device operand sets, step k+1 inputs copied while step k computes"},
             "gpu_launches": launches,
             "clocks": sampler.summary(*window) if sampler else None,
             "per_call_sweep": {
