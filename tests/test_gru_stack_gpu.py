@@ -135,3 +135,39 @@ def test_gru_stack_pairs_and_per_layer_chain_agree(L, monkeypatch):
         assert nmax_err(pairs[l], ref[l]) <= TOL
         assert nmax_err(chain[l], ref[l]) <= TOL
     assert np.array_equal(pairs[0], chain[0])
+
+
+def test_gru_stack_pair_kernel_missing_participant_times_out_cleanly():
+    """One CTA of the two-layer kernel never signals the round counter (a flag
+    nothing sets): every bounded wait runs out, the kernel returns, isam_sync
+    reports ISAM_ERR_TIMEOUT, and a correct call works afterwards."""
+    import os
+    import subprocess
+    import sys
+    import textwrap
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    code = textwrap.dedent(f"""
+        import os, sys, numpy as np, torch
+        sys.path.insert(0, {root!r}); sys.path.insert(0, {os.path.join(root, 'tests')!r})
+        from paper_1810_09958_gb300 import isam, synth
+        import oracle
+        from gpu_util import dev_bf16, nmax_err
+        torch.cuda.set_device(0)
+        L, T, batch, H = 2, 4, 8, 256
+        x, W, U, b, h0 = synth.gru_stack_operands(L, T, batch, H, seed=97)
+        args = [dev_bf16(x), dev_bf16(W), dev_bf16(U), torch.from_numpy(b.reshape(-1)).cuda(), None]
+        out = torch.zeros(L * T * batch * H, device="cuda")
+        os.environ["ISAM_DEBUG_GRU_SKIP_CTA"] = "0"
+        isam.gru_forward_stack(L, T, batch, H, *args, out)
+        rc = isam.load().isam_sync()
+        assert rc == isam.ISAM_ERR_TIMEOUT, rc
+        del os.environ["ISAM_DEBUG_GRU_SKIP_CTA"]
+        isam.gru_forward_stack(L, T, batch, H, *args, out)
+        isam.sync()
+        ref = oracle.gru_stack(x, W, U, b, None)
+        assert nmax_err(out.cpu().numpy().reshape(L, T, batch, H), ref) <= 1e-2
+        print("TIMEOUT_OK")
+    """)
+    env = dict(os.environ, ISAM_WAIT_TIMEOUT_MS="300")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0 and "TIMEOUT_OK" in r.stdout, r.stdout + r.stderr
