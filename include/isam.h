@@ -183,9 +183,11 @@ int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta
  * resident in shared memory and multiplies bf16(h_{t-1}) on the tensor cores
  * (h itself is carried in fp32).  Gates are evaluated in fp32.
  *
- * Supported: T >= 1, 1 <= batch <= 32, hidden a multiple of 64 in
+ * Supported: T >= 1, 1 <= batch <= 256, hidden a multiple of 64 in
  * [64, 1024] except 960; all pointers 16-byte aligned.  Otherwise
- * ISAM_ERR_UNSUPPORTED.  The recurrence runs on hidden / 32 clusters of 4, 2
+ * ISAM_ERR_UNSUPPORTED.  Batches above 32 run with the batch padded to 64 or
+ * 128 rows (the MMA's N; 128 only with 4 K splits), in chunks of that many
+ * rows, one launch per chunk; the rows are independent sequences.  The recurrence runs on hidden / 32 clusters of 4, 2
  * or 1 CTAs (4 when hidden is a multiple of 256, 2 for the other multiples of
  * 128, else 1), launched cooperatively so they are co-resident; each CTA keeps
  * a 96-row slice of U in shared memory, which for hidden = 960 (one CTA per
@@ -242,10 +244,13 @@ int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 
  * deterministic).  Either way the next layer sees bf16(h^l_t), as the
  * recurrent product sees bf16(h_{t-1}).
  *
- * Supported: as isam_gru_forward; with layers > 1, also the shared memory
- * for both weight slices, which excludes hidden 576, 704, 832 and 960
- * (ISAM_ERR_UNSUPPORTED).  Workspace: 2 x ks x T x batch x 3*hidden fp32
- * (ks = 4, 2 or 1 K splits) beside isam_gru_forward's.
+ * Supported: as isam_gru_forward (batch up to 256); with layers > 1 and
+ * batch <= 32, also the shared memory for both weight slices of the
+ * per-layer chain, which excludes hidden 576, 704, 832 and 960
+ * (ISAM_ERR_UNSUPPORTED).  Batches above 32 run layer by layer: the states
+ * below are rounded to bf16 and projected by the GEMM, and each layer's
+ * recurrence runs in chunks of padded rows.  Workspace: 2 x ks x T x batch x
+ * 3*hidden fp32 (ks = 4, 2 or 1 K splits) beside isam_gru_forward's.
  */
 int isam_gru_forward_stack(int layers, int T, int batch, int hidden, int reset_before,
                            const isam_bf16 *x, const isam_bf16 *W, const isam_bf16 *U,
@@ -259,9 +264,9 @@ int isam_gru_forward_stack(int layers, int T, int batch, int hidden, int reset_b
  * that pool), or a latency-bound request path that forbids cudaMalloc/cudaFree
  * because they can synchronise the whole device.
  *
- * Same arguments, layouts, equations and support limits as isam_gru_forward
- * (1 <= batch <= 32, hidden a multiple of 64 in [64, 1024] except 960, any
- * T >= 1).  The
+ * Same arguments, layouts and equations as isam_gru_forward; batch up to 32
+ * only (1 <= batch <= 32, hidden a multiple of 64 in [64, 1024] except 960,
+ * any T >= 1).  The
  * caller still passes every input and h_out.  The workspaces live in one
  * static 8 MiB device array inside libisam.so, which every GPU that loads the
  * library holds until the process exits; the input projection is computed in

@@ -41,15 +41,17 @@ namespace {
 
 constexpr int kGroup = 32;               // hidden units per group (one cluster)
 constexpr int kRowsG = 3 * kGroup;       // 96 U rows per group (r, z, n)
-constexpr int kBatchPad = 32;            // MMA N (batch rows, padded)
+constexpr int kBatchPad = 32;            // MMA N for batch <= 32 (the path with every feature)
+constexpr int kBatchMax = 256;           // larger batches run in chunks of the padded width
 constexpr int kThreads = 128;
 constexpr int kAtomU = kRowsG * 128;     // one 64-wide K atom of the U slice (12 KB)
-constexpr int kAtomH = kBatchPad * 128;  // one K atom of h (4 KB)
 constexpr int kUPad = 32 * 128;          // the M = 128 MMA reads 32 rows past an atom
-// Partial rows received per step: 96 rows of 32 batch values, each row padded
-// to 36 floats so the 8 units a warp reads fall into different banks.
-constexpr int kRecvStride = kBatchPad + 4;
-constexpr int kRecvBytes = kRowsG * kRecvStride * 4;
+// The padded batch BP (32, 64 or 128) is the MMA's N: one K atom of h is BP
+// rows of 128 bytes, and a received partial row holds BP batch values padded
+// to BP + 4 floats, so the 8 units a warp reads fall into different banks.
+__host__ __device__ constexpr int atom_h_bytes(int bp) { return bp * 128; }
+__host__ __device__ constexpr int recv_stride(int bp) { return bp + 4; }
+__host__ __device__ constexpr int recv_bytes(int bp) { return kRowsG * recv_stride(bp) * 4; }
 constexpr int kMaxPieces = 4;
 
 enum : uint32_t {
@@ -63,6 +65,7 @@ enum : uint32_t {
 
 struct GruParams {
     int T, batch, H;
+    int bstride;               // batch rows between two steps of gx / h_out (the full batch; batch is this chunk's rows)
     int ks;                    // K splits per unit group = cluster size
     int ka;                    // 64-wide K atoms per CTA (H / ks / 64)
     int uo;                    // units whose gates one CTA evaluates (32 / ks)
@@ -91,21 +94,23 @@ struct GruLayout {
 };
 
 // U slice | next layer's W slice (has_next) | pad | h piece | partial rows | barriers.
-__host__ __device__ inline GruLayout gru_layout(int ka, bool has_next) {
+__host__ __device__ inline GruLayout gru_layout(int ka, bool has_next, int bp = kBatchPad) {
     GruLayout L;
     L.off_u = 0;
     L.off_w = ka * kAtomU;
     L.off_h = L.off_w + (has_next ? ka * kAtomU : 0) + kUPad;
-    L.off_recv = L.off_h + ka * kAtomH;
-    L.off_bars = L.off_recv + kRecvBytes;
+    L.off_recv = L.off_h + ka * atom_h_bytes(bp);
+    L.off_bars = L.off_recv + recv_bytes(bp);
     L.total = L.off_bars + 128 + 1024;
     return L;
 }
 
-// Template argument KS: K splits per unit group (cluster size, 4, 2 or 1).
-// A CTA evaluates the gates of UO = 32 / KS units over 32 batch rows, NP =
-// 8 / KS (unit, batch) pairs per thread.
-template <int KS>
+// Template arguments: KS, the K splits per unit group (cluster size, 4, 2 or
+// 1), and BP, the padded batch (the MMA's N: 32, 64 or 128).  A CTA evaluates
+// the gates of UO = 32 / KS units over BP batch rows, NP = UO * BP / 128
+// (unit, batch) pairs per thread.  The next layer's product and the K-rank
+// projection slabs exist for BP = 32 only.
+template <int KS, int BP>
 __global__ void __launch_bounds__(kThreads, 1)
     gru_recurrent_kernel(const __grid_constant__ CUtensorMap tmU,
                          const __grid_constant__ CUtensorMap tmH0,
@@ -114,7 +119,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                          const __grid_constant__ CUtensorMap tmR1,
                          const __grid_constant__ CUtensorMap tmWn, const GruParams p) {
     constexpr int UO = kGroup / KS;
-    constexpr int NP = UO * kBatchPad / kThreads;
+    constexpr int NP = UO * BP / kThreads;
+    constexpr int SL = BP == kBatchPad ? KS : 1;  // projection slabs a value can sum
+    constexpr int AH = atom_h_bytes(BP);
+    constexpr int RS = recv_stride(BP);
     constexpr int BSTEP = kThreads / UO;
     if (!launch_shape_ok(p.err, static_cast<uint32_t>(KS), static_cast<uint32_t>(p.n_cta), 0x3F0u))
         return;
@@ -122,7 +130,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~static_cast<uintptr_t>(1023));
     const bool HN = p.has_next != 0;
-    const GruLayout L = gru_layout(p.ka, HN);
+    const GruLayout L = gru_layout(p.ka, HN, BP);
     uint8_t *sU = smem + L.off_u;
     uint8_t *sW = smem + L.off_w;
     uint8_t *sH = smem + L.off_h;
@@ -159,7 +167,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
     // Columns 0-31: the recurrent product; 32-95: the next layer's projection,
     // double-buffered by step parity.
-    const uint32_t tmem_cols = HN ? 128u : 32u;
+    const uint32_t tmem_cols = HN ? 128u : static_cast<uint32_t>(BP);
     if (warp == 0) {
         tmem_alloc(tmem_slot, tmem_cols);
         tmem_relinquish();
@@ -176,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool RB = p.reset_before != 0;
     const int nph = RB ? 2 : 1;
     auto round_bytes = [&](int ph) {
-        return static_cast<uint32_t>(KS * (RB ? (ph == 0 ? 2 : 1) : 3) * UO * kBatchPad * 4);
+        return static_cast<uint32_t>(KS * (RB ? (ph == 0 ? 2 : 1) : 3) * UO * BP * 4);
     };
     if (tid == 0) mbar_arrive_expect_tx(red_full, round_bytes(0));
 
@@ -219,7 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (tid == 32) ok = bounded_wait(ubar, 0, w, SITE_GRU_U);
     __syncwarp();
 
-    const uint32_t idesc = idesc_bf16_f32(128, kBatchPad, false, false);
+    const uint32_t idesc = idesc_bf16_f32(128, BP, false, false);
     int issued_phase = -1;  // last round whose h loads were issued (for the drain)
     // Input projection of a step (independent of h), loaded one step ahead so
     // its memory latency is off the recurrence's critical path: gx is one slab
@@ -227,15 +235,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     // products computed by the layer below.  The loads land in registers
     // (KS x NP = 8 per gate whatever KS) and are summed, after b_ih and in
     // rank order, only where the gates use them.
-    float gxr[KS * NP], gxz[KS * NP], gxn[KS * NP];
+    float gxr[SL * NP], gxz[SL * NP], gxn[SL * NP];
     auto load_gx = [&](int tt) {
 #pragma unroll
         for (int k = 0; k < NP; ++k) {
             const int b = tid / UO + k * BSTEP;
-            const float *g = p.gx + (static_cast<size_t>(tt) * p.batch + b) * G + j;
+            const float *g = p.gx + (static_cast<size_t>(tt) * p.bstride + b) * G + j;
 #pragma unroll
-            for (int s = 0; s < KS; ++s) {
-                const int i = k * KS + s;
+            for (int s = 0; s < SL; ++s) {
+                const int i = k * SL + s;
                 if (b < p.batch && tt < p.T && s < p.gx_parts) {
                     const float *gs = g + static_cast<size_t>(s) * p.gx_slab;
                     gxr[i] = __ldg(gs);
@@ -247,10 +255,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     };
-    auto sum_gx = [&](const float (&v)[KS * NP], float bias, int k) {
+    auto sum_gx = [&](const float (&v)[SL * NP], float bias, int k) {
         float a = bias;
 #pragma unroll
-        for (int s = 0; s < KS; ++s) a += v[k * KS + s];
+        for (int s = 0; s < SL; ++s) a += v[k * SL + s];
         return a;
     };
     load_gx(0);
@@ -273,7 +281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // 32 rows (4 KB) before the atom: still inside shared memory (the
             // U slice precedes W).
             const uint32_t wa = smem_u32(sW + a * kAtomU) - 32u * 128u;
-            const uint32_t ha = smem_u32(sH + a * kAtomH);
+            const uint32_t ha = smem_u32(sH + a * AH);
 #pragma unroll
             for (int k = 0; k < 4; ++k)
                 umma_bf16(tmem_d + col, sdesc_sw128(wa + k * 32, 16, 1024), sdesc_sw128(ha + k * 32, 16, 1024),
@@ -299,8 +307,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     fence_proxy_async_global();
                     const CUtensorMap *m = ph == 0 ? ((t & 1) ? &tmH1 : &tmH0) : ((t & 1) ? &tmR1 : &tmR0);
                     for (int q = 0; q < p.nq; ++q) {
-                        mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(p.qk * kAtomH));
-                        tma_load_3d(m, &hbar[q], sH + q * p.qk * kAtomH, 0, 0, atom0 + q * p.qk);
+                        mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(p.qk * AH));
+                        tma_load_3d(m, &hbar[q], sH + q * p.qk * AH, 0, 0, atom0 + q * p.qk);
                     }
                     issued_phase = round;
                 }
@@ -315,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int k = 0; k < NP; ++k) {
                         const int b = tid / UO + k * BSTEP;
                         if (b < p.batch)
-                            p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
+                            p.h_out[(static_cast<size_t>(last_t) * p.bstride + b) * H + j] = hprev[k];
                     }
                     last_t = -1;
                 }
@@ -331,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (finish) continue;
                     for (int a = q * p.qk; a < (q + 1) * p.qk; ++a) {
                         const uint32_t ua = smem_u32(sU + a * kAtomU);
-                        const uint32_t ha = smem_u32(sH + a * kAtomH);
+                        const uint32_t ha = smem_u32(sH + a * AH);
 #pragma unroll
                         for (int k = 0; k < 4; ++k)
                             umma_bf16(tmem_d, sdesc_sw128(ua + k * 32, 16, 1024),
@@ -359,22 +367,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // rows, round 1 the n rows.
                 const bool pushes = RB ? (ph == 0 ? warp < 2 : warp == 2) : warp < 3;
                 if (pushes) {
-                    uint32_t r[32];
-                    tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16), r);
-                    tmem_ld_wait(r);
                     const uint32_t owner = static_cast<uint32_t>(lane / UO);
                     const int oui = lane % UO;
                     const uint32_t dst = mapa_shared(
-                        smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * kRecvStride), owner);
+                        smem_u32(recv + ((static_cast<int>(rank) * 3 + warp) * UO + oui) * RS), owner);
                     const uint32_t rbar = mapa_shared(smem_u32(red_full), owner);
-                    // Asynchronous remote stores: each counts its bytes on the
-                    // owner's barrier, so nothing here waits for them to land.
 #pragma unroll
-                    for (int c = 0; c < 8; ++c)
-                        st_async_f4(dst + c * 16,
-                                    make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
-                                                __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
-                                    rbar);
+                    for (int cb = 0; cb < BP / 32; ++cb) {  // 32 batch columns at a time
+                        uint32_t r[32];
+                        tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(cb * 32), r);
+                        tmem_ld_wait(r);
+                        // Asynchronous remote stores: each counts its bytes on the
+                        // owner's barrier, so nothing here waits for them to land.
+#pragma unroll
+                        for (int c = 0; c < 8; ++c)
+                            st_async_f4(dst + cb * 128 + c * 16,
+                                        make_float4(__uint_as_float(r[4 * c]), __uint_as_float(r[4 * c + 1]),
+                                                    __uint_as_float(r[4 * c + 2]), __uint_as_float(r[4 * c + 3])),
+                                        rbar);
+                    }
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -382,8 +393,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     alive = false;
                     break;
                 }
-                uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * kBatchPad * H;
-                uint16_t *rhx_t = p.rhx + static_cast<size_t>(t & 1) * kBatchPad * H;
+                uint16_t *hx_next = p.hx + static_cast<size_t>((t + 1) & 1) * BP * H;
+                uint16_t *rhx_t = p.rhx + static_cast<size_t>(t & 1) * BP * H;
 #pragma unroll
                 for (int k = 0; k < NP; ++k) {
                     const int b = tid / UO + k * BSTEP;
@@ -391,12 +402,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                     float ghr = bh_r, ghz = bh_z, ghn = bh_n;
 #pragma unroll
                     for (int s = 0; s < KS; ++s) {  // partials summed in rank order
-                        const float *rs = recv + (s * 3 * UO + ui) * kRecvStride + b;
+                        const float *rs = recv + (s * 3 * UO + ui) * RS + b;
                         if (!RB || ph == 0) {
                             ghr += rs[0];
-                            ghz += rs[UO * kRecvStride];
+                            ghz += rs[UO * RS];
                         }
-                        if (!RB || ph == 1) ghn += rs[2 * UO * kRecvStride];
+                        if (!RB || ph == 1) ghn += rs[2 * UO * RS];
                     }
                     if (!RB) {
                         const float rg = sigmoidf_fast(sum_gx(gxr, bi_r, k) + ghr);
@@ -444,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tmem_ld32(tmem_d + (static_cast<uint32_t>(warp * 32) << 16) + wcol, r);
                         tmem_ld_wait(r);
                         float *dst = p.gxp_out + static_cast<size_t>(rank) * p.gx_slab +
-                                     static_cast<size_t>(t - 1) * p.batch * G + (warp - 1) * H + unit0 + lane;
+                                     static_cast<size_t>(t - 1) * p.bstride * G + (warp - 1) * H + unit0 + lane;
 #pragma unroll
                         for (int c = 0; c < 32; ++c)
                             if (c < p.batch) dst[static_cast<size_t>(c) * G] = __uint_as_float(r[c]);
@@ -461,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int k = 0; k < NP; ++k) {
             const int b = tid / UO + k * BSTEP;
-            if (b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.batch + b) * H + j] = hprev[k];
+            if (b < p.batch) p.h_out[(static_cast<size_t>(last_t) * p.bstride + b) * H + j] = hprev[k];
         }
     }
 
@@ -496,8 +507,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // K splits for a hidden size: each CTA's K range must be whole 64-wide atoms.
 int gru_splits(int H) { return (H % 256 == 0) ? 4 : (H % 128 == 0) ? 2 : 1; }
 
-size_t gru_smem_bytes(int H, bool has_next = false) {
-    return static_cast<size_t>(gru_layout(H / gru_splits(H) / 64, has_next).total);
+size_t gru_smem_bytes(int H, bool has_next = false, int bp = kBatchPad) {
+    return static_cast<size_t>(gru_layout(H / gru_splits(H) / 64, has_next, bp).total);
 }
 
 int gru_cta_count(int H) { return H / kGroup * gru_splits(H); }
@@ -505,8 +516,18 @@ int gru_cta_count(int H) { return H / kGroup * gru_splits(H); }
 using GruKernel = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap,
                            const CUtensorMap, const CUtensorMap, const GruParams);
 
-GruKernel gru_kernel_for(int ks) {
-    return ks == 4 ? gru_recurrent_kernel<4> : ks == 2 ? gru_recurrent_kernel<2> : gru_recurrent_kernel<1>;
+template <int BP>
+GruKernel gru_kernel_for_bp(int ks) {
+    return ks == 4 ? gru_recurrent_kernel<4, BP> : ks == 2 ? gru_recurrent_kernel<2, BP> : gru_recurrent_kernel<1, BP>;
+}
+
+// Padded batch widths a K-split count can run: 128 only with 4 splits (fewer
+// splits leave 16 or 32 (unit, batch) pairs per thread, beyond the registers).
+bool gru_bp_ok(int ks, int bp) { return bp == 32 || bp == 64 || (bp == 128 && ks == 4); }
+
+GruKernel gru_kernel_for(int ks, int bp = kBatchPad) {
+    if (bp == 128) return gru_recurrent_kernel<4, 128>;
+    return bp == 64 ? gru_kernel_for_bp<64>(ks) : gru_kernel_for_bp<32>(ks);
 }
 
 // Opts every instantiation in to `bytes` of dynamic shared memory (once per process).
@@ -515,11 +536,14 @@ int gru_smem_attr(int bytes) {
     static bool done = false;
     std::lock_guard<std::mutex> lk(mu);
     if (done) return ISAM_OK;
-    const int ks[3] = {1, 2, 4};
-    for (int k : ks) {
-        cudaError_t e = cudaFuncSetAttribute(gru_kernel_for(k), cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
-    }
+    const int ks[3] = {1, 2, 4}, bps[3] = {32, 64, 128};
+    for (int k : ks)
+        for (int bp : bps) {
+            if (!gru_bp_ok(k, bp)) continue;
+            cudaError_t e =
+                cudaFuncSetAttribute(gru_kernel_for(k, bp), cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
+        }
     done = true;
     return ISAM_OK;
 }
@@ -543,7 +567,7 @@ int ensure_ws(void **ptr, size_t *cap, size_t need, const char *what) {
 // skipped when null).
 int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, int H, CUtensorMap *tmU,
                    CUtensorMap *tmH0, CUtensorMap *tmH1, CUtensorMap *tmR0, CUtensorMap *tmR1,
-                   const uint16_t *Wn = nullptr, CUtensorMap *tmWn = nullptr) {
+                   const uint16_t *Wn = nullptr, CUtensorMap *tmWn = nullptr, int bp = kBatchPad) {
     int rc;
     const int ka = H / gru_splits(H) / 64;
     const int nq = (ka % 4 == 0) ? 4 : (ka % 3 == 0) ? 3 : (ka % 2 == 0) ? 2 : 1;
@@ -555,13 +579,13 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, i
         if (Wn && (rc = make_tmap_3d_bf16(tmWn, Wn, dims, strides, box))) return rc;
     }
     for (int i = 0; i < 2; ++i) {
-        const uint64_t dims[3] = {64, kBatchPad, static_cast<uint64_t>(H / 64)};
+        const uint64_t dims[3] = {64, static_cast<uint64_t>(bp), static_cast<uint64_t>(H / 64)};
         const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
-        const uint32_t box[3] = {64, kBatchPad, static_cast<uint32_t>(ka / nq)};
-        if ((rc = make_tmap_3d_bf16(i ? tmH1 : tmH0, hx + static_cast<size_t>(i) * kBatchPad * H, dims,
+        const uint32_t box[3] = {64, static_cast<uint32_t>(bp), static_cast<uint32_t>(ka / nq)};
+        if ((rc = make_tmap_3d_bf16(i ? tmH1 : tmH0, hx + static_cast<size_t>(i) * bp * H, dims,
                                     strides, box)))
             return rc;
-        if (tmR0 && (rc = make_tmap_3d_bf16(i ? tmR1 : tmR0, rhx + static_cast<size_t>(i) * kBatchPad * H,
+        if (tmR0 && (rc = make_tmap_3d_bf16(i ? tmR1 : tmR0, rhx + static_cast<size_t>(i) * bp * H,
                                             dims, strides, box)))
             return rc;
     }
@@ -579,7 +603,7 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tm
 // cluster fits at once (the step counter needs every CTA resident).
 int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tmH0,
                      const CUtensorMap &tmH1, const CUtensorMap &tmR0, const CUtensorMap &tmR1,
-                     const CUtensorMap &tmWn, size_t smem, cudaStream_t stream) {
+                     const CUtensorMap &tmWn, size_t smem, cudaStream_t stream, int bp = kBatchPad) {
     const int H = p.H;
     p.ks = gru_splits(H);
     p.ka = H / p.ks / 64;
@@ -601,7 +625,7 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
     cfg.stream = stream;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    const GruKernel kern = gru_kernel_for(p.ks);
+    const GruKernel kern = gru_kernel_for(p.ks, bp);
     cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmU, tmH0, tmH1, tmR0, tmR1, tmWn, p);
     if (e == cudaSuccess) return ISAM_OK;
     (void)cudaGetLastError();
@@ -639,9 +663,9 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
                      const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
                      DeviceState &ds, cudaStream_t stream) {
     const int H = hidden;
-    if (batch > kBatchPad || H % 64 != 0 || H > 1024 || H < 64)
+    if (batch > kBatchMax || H % 64 != 0 || H > 1024 || H < 64)
         return set_error(ISAM_ERR_UNSUPPORTED,
-                         "isam_gru_forward: needs batch <= 32 and hidden a multiple of 64 in "
+                         "isam_gru_forward: needs batch <= 256 and hidden a multiple of 64 in "
                          "[64, 1024] (batch=%d hidden=%d)",
                          batch, H);
     if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
@@ -651,11 +675,30 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     const int n_cta = gru_cta_count(H);
     if (n_cta > ds.num_sms)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: %d CTAs cannot be co-resident", n_cta);
-    const size_t smem_last = gru_smem_bytes(H, false);
+    // Padded batch of the recurrence (the MMA's N): 32 for batch <= 32, with
+    // every feature; above that the narrowest of 64 and 128 that holds the
+    // batch (else the widest that fits beside U), the batch running in chunks
+    // of that many rows (one launch each; each chunk's rows are independent
+    // sequences).  A step costs about the same whatever the width's fill.
+    const bool chunked = batch > kBatchPad;
+    int bp = kBatchPad;
+    if (chunked) {
+        auto fits = [&](int cand) {
+            return gru_bp_ok(gru_splits(H), cand) &&
+                   gru_smem_bytes(H, false, cand) <= static_cast<size_t>(ds.max_smem_optin);
+        };
+        if (batch <= 64 && fits(64))
+            bp = 64;
+        else if (fits(128))
+            bp = 128;
+        else if (fits(64))
+            bp = 64;
+    }
+    const size_t smem_last = gru_smem_bytes(H, false, bp);
     const size_t smem_next = gru_smem_bytes(H, true);
     if (smem_last > static_cast<size_t>(ds.max_smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: hidden too large for shared memory");
-    if (layers > 1 && smem_next > static_cast<size_t>(ds.max_smem_optin))
+    if (layers > 1 && !chunked && smem_next > static_cast<size_t>(ds.max_smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED,
                          "isam_gru_forward_stack: hidden %d leaves no room for the next layer's "
                          "weights beside the recurrent ones (%zu bytes of shared memory)",
@@ -670,13 +713,14 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     // Next layers' projections: two sets (read by layer l, written by layer l)
     // of ks slabs, one per K rank.
     const int ks = gru_splits(H);
-    if (layers > 1 &&
+    if (layers > 1 && !chunked &&
         (rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_gxp), &ds.gru_gxp_bytes,
                         2 * static_cast<size_t>(ks) * gx_floats * sizeof(float),
                         "allocating the stacked GRU projection workspace")))
         return rc;
-    // Exchange buffers: h (2 slots) then r * h (2 slots, the reset-before form).
-    const size_t hx_bytes = static_cast<size_t>(4) * kBatchPad * H * sizeof(uint16_t);
+    // Exchange buffers: h (2 slots) then r * h (2 slots, the reset-before form),
+    // bp rows each.
+    const size_t hx_bytes = static_cast<size_t>(4) * bp * H * sizeof(uint16_t);
     if (ds.gru_hx_bytes < hx_bytes) {
         if ((rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_hx), &ds.gru_hx_bytes, hx_bytes,
                             "allocating the GRU exchange buffer")))
@@ -691,7 +735,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     if ((rc = gru_smem_attr(ds.max_smem_optin))) return rc;
 
     const size_t wsz = static_cast<size_t>(3) * H * H;
-    uint16_t *rhx = ds.gru_hx + static_cast<size_t>(2) * kBatchPad * H;
+    uint16_t *rhx = ds.gru_hx + static_cast<size_t>(2) * bp * H;
     // Input projection of layer l for all steps: gx = in W_l^T + b_ih_l
     // (M = T*batch, N = 3H, K = H).
     auto project = [&](const uint16_t *in, int l) {
@@ -705,18 +749,20 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     // One layer's recurrence.  Its projection is either ds.gru_gx (one slab,
     // b_ih included) or, for layer l > 0 of the per-layer chain, the slabs the
     // layer below computed; with has_next it computes layer l + 1's slabs.
-    auto recur = [&](int l, bool has_next, bool gx_from_below) {
+    // Batch rows [b0, b0 + nb) of layer l (all rows unless chunked).
+    auto recur = [&](int l, bool has_next, bool gx_from_below, int b0, int nb) {
         const uint16_t *Wn = has_next ? W + (l + 1) * wsz : nullptr;
         CUtensorMap tmU, tmH0, tmH1, tmR0, tmR1, tmWn;
         int r;
-        if ((r = recurrent_maps(U + l * wsz, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1, Wn, &tmWn)))
+        if ((r = recurrent_maps(U + l * wsz, ds.gru_hx, rhx, H, &tmU, &tmH0, &tmH1, &tmR0, &tmR1, Wn, &tmWn, bp)))
             return r;
         GruParams p{};
         p.T = T;
-        p.batch = batch;
+        p.batch = nb;
+        p.bstride = batch;
         p.H = H;
         if (!gx_from_below) {
-            p.gx = ds.gru_gx;
+            p.gx = ds.gru_gx + static_cast<size_t>(b0) * 3 * H;
             p.gx_parts = 1;
             p.b_ih = nullptr;
         } else {
@@ -728,8 +774,8 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
         p.has_next = has_next ? 1 : 0;
         p.gxp_out = has_next ? ds.gru_gxp + static_cast<size_t>(l & 1) * ks * gx_floats : nullptr;
         p.b_hh = b + static_cast<size_t>(l) * 6 * H + 3 * H;
-        p.h0 = h0 ? h0 + static_cast<size_t>(l) * batch * H : nullptr;
-        p.h_out = h_out + static_cast<size_t>(l) * seq_rows * H;
+        p.h0 = h0 ? h0 + (static_cast<size_t>(l) * batch + b0) * H : nullptr;
+        p.h_out = h_out + static_cast<size_t>(l) * seq_rows * H + static_cast<size_t>(b0) * H;
         p.hx = ds.gru_hx;
         p.rhx = rhx;
         p.reset_before = reset_before ? 1 : 0;
@@ -741,8 +787,33 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
         cudaError_t e = cudaMemsetAsync(ds.gru_counter, 0, sizeof(uint32_t), stream);
         if (e != cudaSuccess) return cuda_error(e, "clearing the GRU step counter");
         return launch_recurrent(p, tmU, tmH0, tmH1, tmR0, tmR1, has_next ? tmWn : tmU,
-                                has_next ? smem_next : smem_last, stream);
+                                has_next ? smem_next : smem_last, stream, bp);
     };
+    // bf16 copy of layer l - 1's states as layer l's GEMM input.
+    auto states_below = [&](int l) {
+        const size_t n4 = seq_rows * H / 4;
+        const int blocks = static_cast<int>(std::min<size_t>((n4 + 255) / 256, static_cast<size_t>(ds.num_sms) * 8));
+        states_to_bf16_kernel<<<blocks, 256, 0, stream>>>(
+            reinterpret_cast<const float4 *>(h_out + static_cast<size_t>(l - 1) * seq_rows * H),
+            reinterpret_cast<uint2 *>(ds.gru_xb), n4);
+        cudaError_t e = cudaGetLastError();
+        return e == cudaSuccess ? ISAM_OK : cuda_error(e, "launch states_to_bf16_kernel");
+    };
+
+    // Batches wider than 32: every layer projects its input with the GEMM and
+    // runs its recurrence chunk by chunk.
+    if (chunked) {
+        if (layers > 1 && (rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_xb), &ds.gru_xb_bytes,
+                                          seq_rows * H * sizeof(uint16_t), "allocating the GRU layer-input buffer")))
+            return rc;
+        for (int l = 0; l < layers; ++l) {
+            if (l > 0 && (rc = states_below(l))) return rc;
+            if ((rc = project(l > 0 ? ds.gru_xb : x, l))) return rc;
+            for (int b0 = 0; b0 < batch; b0 += bp)
+                if ((rc = recur(l, false, false, b0, std::min(bp, batch - b0)))) return rc;
+        }
+        return ISAM_OK;
+    }
 
     // Pairs of layers in one kernel (gru_wave.cu): layer l + 1 advances one
     // step behind layer l, its projection computed from the same h tiles.
@@ -756,13 +827,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
         for (int l = 0; l < layers;) {
             const uint16_t *in = x;
             if (l > 0) {
-                const size_t n4 = seq_rows * H / 4;
-                const int blocks = static_cast<int>(std::min<size_t>((n4 + 255) / 256, static_cast<size_t>(ds.num_sms) * 8));
-                states_to_bf16_kernel<<<blocks, 256, 0, stream>>>(
-                    reinterpret_cast<const float4 *>(h_out + static_cast<size_t>(l - 1) * seq_rows * H),
-                    reinterpret_cast<uint2 *>(ds.gru_xb), n4);
-                cudaError_t e = cudaGetLastError();
-                if (e != cudaSuccess) return cuda_error(e, "launch states_to_bf16_kernel");
+                if ((rc = states_below(l))) return rc;
                 in = ds.gru_xb;
             }
             if ((rc = project(in, l))) return rc;
@@ -777,7 +842,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
                     return rc;
                 l += 2;
             } else {
-                if ((rc = recur(l, false, false))) return rc;
+                if ((rc = recur(l, false, false, 0, batch))) return rc;
                 l += 1;
             }
         }
@@ -788,7 +853,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     // projection (its slabs), which layer l + 1 sums as it goes.
     if ((rc = project(x, 0))) return rc;
     for (int l = 0; l < layers; ++l)
-        if ((rc = recur(l, l + 1 < layers, l > 0))) return rc;
+        if ((rc = recur(l, l + 1 < layers, l > 0, 0, batch))) return rc;
     return ISAM_OK;
 }
 
@@ -952,6 +1017,7 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         GruParams p{};
         p.T = tc;
         p.batch = batch;
+        p.bstride = batch;
         p.H = H;
         p.gx = gx;
         p.b_hh = b + 3 * H;

@@ -109,7 +109,7 @@ def test_gru_unsupported_shapes_rejected():
     lib = isam.load()
     import ctypes
     p = lambda t: ctypes.c_void_p(t.data_ptr())
-    assert lib.isam_gru_forward(1, 33, 64, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_gru_forward(1, 257, 64, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
     assert lib.isam_gru_forward(1, 1, 96, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
     # hidden 960: one CTA per cluster would need 15 K atoms of U (does not fit).
     assert lib.isam_gru_forward(1, 1, 960, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
@@ -210,3 +210,35 @@ def test_gru_reset_before_repeat_and_interleaved_calls_identical():
     c = run_gru(x, W, U, b, h0, reset_before=True)
     d = run_gru(x, W, U, b, h0)
     assert np.array_equal(a, c) and np.array_equal(m, d)
+
+
+# ---- batches wider than 32: the recurrence runs with a padded batch of 64 or
+# 128 (the MMA's N), in chunks of that many rows.
+
+@pytest.mark.parametrize("T,batch,H,rb", [(6, 33, 1024, False), (5, 64, 1024, False), (4, 100, 1024, True),
+                                          (6, 128, 1024, False), (3, 200, 1024, False), (3, 256, 1024, True),
+                                          (5, 96, 896, False), (4, 70, 448, True), (3, 129, 256, False),
+                                          (2, 256, 64, False)])
+def test_gru_wide_batch(T, batch, H, rb):
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 31 + batch * 7 + H)
+    h0 = synth.f32_uniform(batch + H + 5, (batch, H))
+    got = run_gru(x, W, U, b, h0, reset_before=rb)
+    ref = oracle.gru_forward(x, W, U, b, h0, reset_before=rb)
+    assert nmax_err(got, ref) <= TOL, nmax_err(got, ref)
+
+
+def test_gru_wide_batch_rows_independent_of_chunking():
+    """Rows are independent sequences: the first 32 rows of a batch of 160
+    (chunks of 128 padded rows) match the same rows run as a batch of 32.
+    Not bit for bit: the input projection's GEMM takes another tile plan at
+    M = 960 than at M = 192 (another fp32 summation order), and bf16 rounding
+    of h carries that over the steps; rows mixing across the chunk would show
+    errors of order 1."""
+    T, batch, H = 6, 160, 1024
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=515)
+    h0 = synth.f32_uniform(516, (batch, H))
+    wide = run_gru(x, W, U, b, h0)
+    narrow = run_gru(np.ascontiguousarray(x[:, :32]), W, U, b, np.ascontiguousarray(h0[:32]))
+    assert nmax_err(wide[:, :32], narrow) <= 1e-3
+    ref = oracle.gru_forward(x, W, U, b, h0)
+    assert nmax_err(wide, ref) <= TOL

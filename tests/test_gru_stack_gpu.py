@@ -113,7 +113,7 @@ def test_gru_stack_unsupported_shapes_rejected():
     # hidden 832: one CTA per cluster holds 13 K atoms; two weight slices do not fit.
     assert lib.isam_gru_forward_stack(2, 1, 1, 832, 0, p(z), p(z), p(z), p(f), None, p(f)) == \
         isam.ISAM_ERR_UNSUPPORTED
-    assert lib.isam_gru_forward_stack(2, 1, 33, 128, 0, p(z), p(z), p(z), p(f), None, p(f)) == \
+    assert lib.isam_gru_forward_stack(2, 1, 257, 128, 0, p(z), p(z), p(z), p(f), None, p(f)) == \
         isam.ISAM_ERR_UNSUPPORTED
     o = torch.zeros(832, dtype=torch.float32, device="cuda")
     assert lib.isam_gru_forward_stack(1, 1, 1, 832, 0, p(z), p(z), p(z), p(f), None, p(o)) == isam.ISAM_OK
@@ -171,3 +171,14 @@ def test_gru_stack_pair_kernel_missing_participant_times_out_cleanly():
     env = dict(os.environ, ISAM_WAIT_TIMEOUT_MS="300")
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0 and "TIMEOUT_OK" in r.stdout, r.stdout + r.stderr
+
+
+@pytest.mark.parametrize("L,T,batch,H,rb", [(2, 5, 48, 1024, False), (3, 4, 130, 512, True), (2, 3, 256, 256, False)])
+def test_gru_stack_wide_batch(L, T, batch, H, rb):
+    """Batches wider than 32: each layer projects the bf16 states below with
+    the GEMM and runs its recurrence in chunks of padded rows."""
+    x, W, U, b, h0 = synth.gru_stack_operands(L, T, batch, H, seed=L * 13 + batch + H)
+    got = run_stack(x, W, U, b, h0, rb)
+    ref = oracle.gru_stack(x, W, U, b, h0, reset_before=rb)
+    for l in range(L):
+        assert nmax_err(got[l], ref[l]) <= TOL, (l, nmax_err(got[l], ref[l]))
