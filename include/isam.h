@@ -183,9 +183,12 @@ int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta
  * resident in shared memory and multiplies bf16(h_{t-1}) on the tensor cores
  * (h itself is carried in fp32).  Gates are evaluated in fp32.
  *
- * Supported: T >= 1, 1 <= batch <= 256, hidden a multiple of 64 in
- * [64, 1024] except 960; all pointers 16-byte aligned.  Otherwise
- * ISAM_ERR_UNSUPPORTED.  Batches above 32 run with the batch padded to 64 or
+ * Supported: T >= 1, 1 <= batch <= 256, hidden a multiple of 32 in
+ * [32, 1024] except 864, 928, 960 and 992 (one CTA per group would need 14
+ * or 15 K atoms of U in shared memory); all pointers 16-byte aligned.
+ * Otherwise ISAM_ERR_UNSUPPORTED.  A hidden of 64 k + 32 runs with one CTA
+ * per group of 32 units and a last K atom half outside the matrix (zeros on
+ * both sides of the product).  Batches above 32 run with the batch padded to 64 or
  * 128 rows (the MMA's N; 128 only with 4 K splits), in chunks of that many
  * rows, one launch per chunk; the rows are independent sequences.  The recurrence runs on hidden / 32 clusters of 4, 2
  * or 1 CTAs (4 when hidden is a multiple of 256, 2 for the other multiples of

@@ -71,6 +71,7 @@ struct GruParams {
     int uo;                    // units whose gates one CTA evaluates (32 / ks)
     int n_cta;                 // (H / 32) * ks
     int nq, qk;                // h arrives in nq pieces of qk atoms (nq * qk == ka)
+    int h2d;                   // hidden % 64 == 32: h maps are 2-D, one box per atom (the last half outside)
     const float *gx;           // [T*batch][3H], includes b_ih
     const float *b_hh;         // [3H]
     const float *h0;           // [batch][H] or null
@@ -308,7 +309,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const CUtensorMap *m = ph == 0 ? ((t & 1) ? &tmH1 : &tmH0) : ((t & 1) ? &tmR1 : &tmR0);
                     for (int q = 0; q < p.nq; ++q) {
                         mbar_arrive_expect_tx(&hbar[q], static_cast<uint32_t>(p.qk * AH));
-                        tma_load_3d(m, &hbar[q], sH + q * p.qk * AH, 0, 0, atom0 + q * p.qk);
+                        if (p.h2d) {
+                            // The last atom's upper 32 columns lie past the row:
+                            // the 2-D box fills them with zeros (as U's map does).
+                            for (int a = q * p.qk; a < (q + 1) * p.qk; ++a)
+                                tma_load_2d(m, &hbar[q], sH + a * AH, (atom0 + a) * 64, 0);
+                        } else {
+                            tma_load_3d(m, &hbar[q], sH + q * p.qk * AH, 0, 0, atom0 + q * p.qk);
+                        }
                     }
                     issued_phase = round;
                 }
@@ -504,11 +512,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// K splits for a hidden size: each CTA's K range must be whole 64-wide atoms.
+// K splits for a hidden size: each CTA's K range must be whole 64-wide atoms
+// (a hidden of 64 k + 32 has one CTA per group and a last, half-filled atom).
 int gru_splits(int H) { return (H % 256 == 0) ? 4 : (H % 128 == 0) ? 2 : 1; }
 
+// 64-wide K atoms per CTA.
+int gru_atoms(int H) { return (H / gru_splits(H) + 63) / 64; }
+
 size_t gru_smem_bytes(int H, bool has_next = false, int bp = kBatchPad) {
-    return static_cast<size_t>(gru_layout(H / gru_splits(H) / 64, has_next, bp).total);
+    return static_cast<size_t>(gru_layout(gru_atoms(H), has_next, bp).total);
 }
 
 int gru_cta_count(int H) { return H / kGroup * gru_splits(H); }
@@ -569,7 +581,7 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, i
                    CUtensorMap *tmH0, CUtensorMap *tmH1, CUtensorMap *tmR0, CUtensorMap *tmR1,
                    const uint16_t *Wn = nullptr, CUtensorMap *tmWn = nullptr, int bp = kBatchPad) {
     int rc;
-    const int ka = H / gru_splits(H) / 64;
+    const int ka = gru_atoms(H);
     const int nq = (ka % 4 == 0) ? 4 : (ka % 3 == 0) ? 3 : (ka % 2 == 0) ? 2 : 1;
     {
         const uint64_t dims[3] = {static_cast<uint64_t>(H), static_cast<uint64_t>(H), 3};
@@ -579,6 +591,19 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, const uint16_t *rhx, i
         if (Wn && (rc = make_tmap_3d_bf16(tmWn, Wn, dims, strides, box))) return rc;
     }
     for (int i = 0; i < 2; ++i) {
+        if (H % 64 != 0) {
+            // [bp rows][H] with 64 x bp boxes, one per atom: the last atom's
+            // upper half lies outside the rows and reads as zeros.
+            const uint16_t *slot_h = hx + static_cast<size_t>(i) * bp * H;
+            if ((rc = make_tmap_2d_bf16(i ? tmH1 : tmH0, slot_h, static_cast<uint64_t>(H), static_cast<uint64_t>(bp),
+                                        static_cast<uint64_t>(H) * 2, 64, static_cast<uint32_t>(bp))))
+                return rc;
+            if (tmR0 && (rc = make_tmap_2d_bf16(i ? tmR1 : tmR0, rhx + static_cast<size_t>(i) * bp * H,
+                                                static_cast<uint64_t>(H), static_cast<uint64_t>(bp),
+                                                static_cast<uint64_t>(H) * 2, 64, static_cast<uint32_t>(bp))))
+                return rc;
+            continue;
+        }
         const uint64_t dims[3] = {64, static_cast<uint64_t>(bp), static_cast<uint64_t>(H / 64)};
         const uint64_t strides[2] = {static_cast<uint64_t>(H) * 2, 128};
         const uint32_t box[3] = {64, static_cast<uint32_t>(bp), static_cast<uint32_t>(ka / nq)};
@@ -606,7 +631,8 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
                      const CUtensorMap &tmWn, size_t smem, cudaStream_t stream, int bp = kBatchPad) {
     const int H = p.H;
     p.ks = gru_splits(H);
-    p.ka = H / p.ks / 64;
+    p.ka = gru_atoms(H);
+    p.h2d = H % 64 != 0 ? 1 : 0;
     p.uo = kGroup / p.ks;
     p.n_cta = gru_cta_count(H);
     p.nq = (p.ka % 4 == 0) ? 4 : (p.ka % 3 == 0) ? 3 : (p.ka % 2 == 0) ? 2 : 1;
@@ -663,10 +689,10 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
                      const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
                      DeviceState &ds, cudaStream_t stream) {
     const int H = hidden;
-    if (batch > kBatchMax || H % 64 != 0 || H > 1024 || H < 64)
+    if (batch > kBatchMax || H % 32 != 0 || H > 1024 || H < 32)
         return set_error(ISAM_ERR_UNSUPPORTED,
-                         "isam_gru_forward: needs batch <= 256 and hidden a multiple of 64 in "
-                         "[64, 1024] (batch=%d hidden=%d)",
+                         "isam_gru_forward: needs batch <= 256 and hidden a multiple of 32 in "
+                         "[32, 1024] (batch=%d hidden=%d)",
                          batch, H);
     if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
          reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |

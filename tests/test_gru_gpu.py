@@ -110,7 +110,7 @@ def test_gru_unsupported_shapes_rejected():
     import ctypes
     p = lambda t: ctypes.c_void_p(t.data_ptr())
     assert lib.isam_gru_forward(1, 257, 64, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
-    assert lib.isam_gru_forward(1, 1, 96, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_gru_forward(1, 1, 80, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
     # hidden 960: one CTA per cluster would need 15 K atoms of U (does not fit).
     assert lib.isam_gru_forward(1, 1, 960, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
 
@@ -242,3 +242,16 @@ def test_gru_wide_batch_rows_independent_of_chunking():
     assert nmax_err(wide[:, :32], narrow) <= 1e-3
     ref = oracle.gru_forward(x, W, U, b, h0)
     assert nmax_err(wide, ref) <= TOL
+
+
+# ---- hidden a multiple of 32 but not of 64: one CTA per group of 32 units,
+# the last 64-wide K atom half outside the matrix (zero-filled on both sides).
+
+@pytest.mark.parametrize("T,batch,H,rb", [(5, 3, 32, False), (4, 17, 96, False), (6, 32, 160, True),
+                                          (3, 8, 480, False), (4, 50, 224, False), (3, 5, 800, True)])
+def test_gru_hidden_odd_multiple_of_32(T, batch, H, rb):
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 17 + batch + H * 3)
+    h0 = synth.f32_uniform(H + batch, (batch, H))
+    got = run_gru(x, W, U, b, h0, reset_before=rb)
+    ref = oracle.gru_forward(x, W, U, b, h0, reset_before=rb)
+    assert nmax_err(got, ref) <= TOL, nmax_err(got, ref)

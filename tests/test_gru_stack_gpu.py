@@ -182,3 +182,12 @@ def test_gru_stack_wide_batch(L, T, batch, H, rb):
     ref = oracle.gru_stack(x, W, U, b, h0, reset_before=rb)
     for l in range(L):
         assert nmax_err(got[l], ref[l]) <= TOL, (l, nmax_err(got[l], ref[l]))
+
+
+@pytest.mark.parametrize("L,T,batch,H,rb", [(2, 4, 9, 96, False), (3, 3, 32, 352, True)])
+def test_gru_stack_hidden_odd_multiple_of_32(L, T, batch, H, rb):
+    x, W, U, b, h0 = synth.gru_stack_operands(L, T, batch, H, seed=L + T + batch + H)
+    got = run_stack(x, W, U, b, h0, rb)
+    ref = oracle.gru_stack(x, W, U, b, h0, reset_before=rb)
+    for l in range(L):
+        assert nmax_err(got[l], ref[l]) <= TOL, (l, nmax_err(got[l], ref[l]))
