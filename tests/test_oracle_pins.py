@@ -154,6 +154,27 @@ def test_gru_saturated_update_gate_keeps_h0(oracle_lib):
         np.testing.assert_allclose(got[t], h0.astype(np.float64), rtol=0, atol=1e-11)
 
 
+def test_gru_closed_update_gate_follows_candidate(oracle_lib):
+    """b_z = -30 drives z to ~1e-13, so h_t is the candidate alone: h_t = n_t
+    with n_t = tanh(W_n x_t + b_in + r_t * (U_n h_{t-1} + b_hn)) and
+    r_t = sigmoid(W_r x_t + b_ir + U_r h_{t-1} + b_hr), evaluated step by step
+    in float64 numpy (the one-step formula, no update-gate term)."""
+    T, batch, H = 6, 3, 24
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=14)
+    b = b.copy()
+    b[H:2 * H] = -30.0
+    h0 = synth.f32_uniform(15, (batch, H))
+    got = oracle_lib.gru_forward(x, W, U, b, h0)
+    Wf, Uf, xf, bb = f64(W), f64(U), f64(x), b.astype(np.float64)
+    h = h0.astype(np.float64)
+    for t in range(T):
+        gx = xf[t] @ Wf.T + bb[:3 * H]
+        gh = h @ Uf.T + bb[3 * H:]
+        r = sig(gx[:, :H] + gh[:, :H])
+        h = np.tanh(gx[:, 2 * H:] + r * gh[:, 2 * H:])
+        np.testing.assert_allclose(got[t], h, rtol=0, atol=1e-11)
+
+
 def test_gru_matches_torch_float64(oracle_lib):
     """torch.nn.GRU uses the same (r, z, n) order with the reset gate applied
     after the recurrent product, so it is an independent implementation."""
