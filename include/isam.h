@@ -306,13 +306,29 @@ int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam_bf16 *x,
  *   out   [N][H][W][Cout] fp32
  *
  * The depthwise result is formed in fp32 and rounded to bf16 for the tensor
- * cores; it never leaves the chip.
+ * cores; it never leaves the chip.  The pointwise weights stay resident in
+ * shared memory; where Cin x Cout of them do not fit beside the kernel's
+ * other buffers (Cin = Cout = 256, for one), the output channels are split
+ * into blocks of equal width (a multiple of 16), one launch per block, each
+ * recomputing the depthwise stage.
  * Supported: Cin % 16 == 0, 16 <= Cin <= 256, Cout % 16 == 0,
  * 16 <= Cout <= 256; pointers 16-byte aligned.  Otherwise
  * ISAM_ERR_UNSUPPORTED.
  */
 int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
                     const isam_bf16 *dw_w, const isam_bf16 *pw_w, float *out);
+
+/*
+ * The plan isam_dwsep_conv takes for an image W pixels wide with Cin -> Cout
+ * channels (it does not depend on N or H); nothing is launched.  out[4]:
+ *   out[0]  kernel: 0 = whole image rows per tile with an input-row ring in
+ *           shared memory, 1 = 128 pixels per tile, loaded per pixel
+ *   out[1]  image rows per tile (kernel 0), else 0
+ *   out[2]  output-channel blocks (launches)
+ *   out[3]  channels per block (the last block may be narrower)
+ * Returns ISAM_ERR_UNSUPPORTED for channel counts isam_dwsep_conv rejects.
+ */
+int isam_dwsep_plan_info(int W, int Cin, int Cout, int *out);
 
 #ifdef __cplusplus
 }

@@ -417,4 +417,13 @@ int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
     return dwsep_launch(N, H, W, Cin, Cout, x, dw_w, pw_w, out, *ds, current_stream());
 }
 
+int isam_dwsep_plan_info(int W, int Cin, int Cout, int *out) {
+    if (W < 1 || Cin < 1 || Cout < 1 || !out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_dwsep_plan_info: sizes must be >= 1, out non-null");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return dwsep_plan(W, Cin, Cout, *ds, out);
+}
+
 }  // extern "C"

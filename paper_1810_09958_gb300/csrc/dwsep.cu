@@ -17,6 +17,7 @@
 // The depthwise intermediate never leaves the chip.
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cstdio>
 #include <type_traits>
 
@@ -379,7 +380,8 @@ struct DwRowParams {
     int row_bytes;       // one ring slot: W * Cin * 2 bytes of pixels + >= one pixel of zeros, rounded to 128
     int ring;            // input rows resident per CTA (2 * rt + 2 <= kRingMax)
     const uint16_t *dw;
-    float *out;
+    float *out;          // first output column of this launch's channel block
+    int ldo;             // output row pitch in elements (all Cout channels of the layer)
     unsigned long long timeout_ns;
     uint32_t *err;
 };
@@ -856,7 +858,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
                         if (lane < cols) {
                             const int pos = (lane >> 2) ^ (rr & 7);
                             const float v = *reinterpret_cast<const float *>(sb + rr * 128 + pos * 16 + (lane & 3) * 4);
-                            p.out[(row0 + rr) * Cout + c + lane] = v;
+                            p.out[(row0 + rr) * p.ldo + c + lane] = v;
                         }
                     }
                     __syncwarp();
@@ -885,36 +887,42 @@ __global__ void __launch_bounds__(kRThreads, 1)
     }
 }
 
-}  // namespace
-
-int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
-                 const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t stream) {
-    if (Cin % 16 != 0 || Cin < 16 || Cin > 256 || Cout % 16 != 0 || Cout < 16 || Cout > 256)
-        return set_error(ISAM_ERR_UNSUPPORTED,
-                         "isam_dwsep_conv: needs Cin and Cout multiples of 16 in [16, 256] "
-                         "(Cin=%d Cout=%d)",
-                         Cin, Cout);
-    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dw) |
-         reinterpret_cast<uintptr_t>(pw) | reinterpret_cast<uintptr_t>(out)) & 15u)
-        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: pointers must be 16-byte aligned");
-    const long long M = static_cast<long long>(N) * H * W;
-    if (M > (1ll << 31) - 256)
-        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: N*H*W too large");
-    int rc;
-    // Row-ring path: rt image rows per tile, 2 * rt + 2 rows resident.
+// Image rows per tile of the row-ring kernel for a block of pc output
+// channels, or 0 where that kernel does not apply (an image wider than one
+// MMA block, a channel count its thread mapping does not divide, or no ring
+// that fits shared memory beside the block's weights).
+int dw_rows_per_tile(int W, int Cin, int pc, const DeviceState &ds) {
     int rt = (W <= kBM && kRProd % (Cin / 4) == 0) ? kBM / W : 0;
     if (rt > (kRingMax - 2) / 2) rt = (kRingMax - 2) / 2;
-    while (rt > 1 && dw_row_layout(W, Cin, Cout, 2 * rt + 2).total > ds.max_smem_optin) --rt;
-    const DwRowLayout RL = dw_row_layout(W, Cin, Cout, 2 * rt + 2);
-    if (rt >= 1 && RL.total <= ds.max_smem_optin) {
+    while (rt > 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total > ds.max_smem_optin) --rt;
+    return (rt >= 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total <= ds.max_smem_optin) ? rt : 0;
+}
+
+bool dw_block_fits(int W, int Cin, int pc, const DeviceState &ds) {
+    return dw_rows_per_tile(W, Cin, pc, ds) > 0 || dw_layout(Cin, pc).total <= ds.max_smem_optin;
+}
+
+// One launch for output channels c0 .. c0 + pc - 1 of a layer with Cout
+// channels: the block's columns of pw_w and out, addressed with the layer's
+// full row pitches.
+int dwsep_block(int N, int H, int W, int Cin, int Cout, int c0, int pc, const uint16_t *x, const uint16_t *dw,
+                const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t stream) {
+    const long long M = static_cast<long long>(N) * H * W;
+    const uint16_t *pwb = pw + c0;
+    float *outb = out + c0;
+    int rc;
+    const int rt = dw_rows_per_tile(W, Cin, pc, ds);
+    if (rt > 0) {
+        // Row-ring path: rt image rows per tile, 2 * rt + 2 rows resident.
+        const DwRowLayout RL = dw_row_layout(W, Cin, pc, 2 * rt + 2);
         CUtensorMap tmW, tmOut, tmOut16, tmOut8;
-        if ((rc = make_tmap_2d_bf16(&tmW, pw, static_cast<uint64_t>(Cout), static_cast<uint64_t>(Cin),
+        if ((rc = make_tmap_2d_bf16(&tmW, pwb, static_cast<uint64_t>(pc), static_cast<uint64_t>(Cin),
                                     static_cast<uint64_t>(Cout) * 2, 64, 64)))
             return rc;
         // Output boxes of 32 columns x 32, 16 and 8 rows.
         CUtensorMap *outs[3] = {&tmOut, &tmOut16, &tmOut8};
         for (int i = 0; i < 3; ++i)
-            if ((rc = make_tmap_2d_f32(outs[i], out, static_cast<uint64_t>(Cout), static_cast<uint64_t>(M),
+            if ((rc = make_tmap_2d_f32(outs[i], outb, static_cast<uint64_t>(pc), static_cast<uint64_t>(M),
                                        static_cast<uint64_t>(Cout) * 4, 32, 32u >> i)))
                 return rc;
         DwRowParams q{};
@@ -922,17 +930,18 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
         q.H = H;
         q.W = W;
         q.Cin = Cin;
-        q.Cout = Cout;
+        q.Cout = pc;
         q.rt = rt;
         q.ring = 2 * rt + 2;
         q.tiles_per_img = (H + q.rt - 1) / q.rt;
         q.tiles = N * q.tiles_per_img;
         q.kb = (Cin + 63) / 64;
-        q.nchunks = (Cout + 63) / 64;
+        q.nchunks = (pc + 63) / 64;
         q.row_bytes = dw_ring_row_bytes(W, Cin);
         q.x = x;
         q.dw = dw;
-        q.out = out;
+        q.out = outb;
+        q.ldo = Cout;
         q.timeout_ns = wait_timeout_ns();
         q.err = ds.err_word;
         static bool rattr = false;
@@ -948,15 +957,16 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
         if (e != cudaSuccess) return cuda_error(e, "launch dwsep_rows_kernel");
         return ISAM_OK;
     }
-    const DwLayout L = dw_layout(Cin, Cout);
+    const DwLayout L = dw_layout(Cin, pc);
     if (L.total > ds.max_smem_optin)
         return set_error(ISAM_ERR_UNSUPPORTED,
-                         "isam_dwsep_conv: Cin=%d, Cout=%d does not fit shared memory", Cin, Cout);
+                         "isam_dwsep_conv: Cin=%d with %d output channels per launch does not fit shared memory",
+                         Cin, pc);
     CUtensorMap tmW, tmOut;
-    if ((rc = make_tmap_2d_bf16(&tmW, pw, static_cast<uint64_t>(Cout), static_cast<uint64_t>(Cin),
+    if ((rc = make_tmap_2d_bf16(&tmW, pwb, static_cast<uint64_t>(pc), static_cast<uint64_t>(Cin),
                                 static_cast<uint64_t>(Cout) * 2, 64, 64)))
         return rc;
-    if ((rc = make_tmap_2d_f32(&tmOut, out, static_cast<uint64_t>(Cout), static_cast<uint64_t>(M),
+    if ((rc = make_tmap_2d_f32(&tmOut, outb, static_cast<uint64_t>(pc), static_cast<uint64_t>(M),
                                static_cast<uint64_t>(Cout) * 4, 32, 32)))
         return rc;
     DwParams p{};
@@ -964,12 +974,12 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
     p.H = H;
     p.W = W;
     p.Cin = Cin;
-    p.Cout = Cout;
+    p.Cout = pc;
     p.M = M;
     p.tiles = static_cast<int>((M + kBM - 1) / kBM);
     p.atoms = (Cin + 63) / 64;
     p.kb = (Cin + 63) / 64;
-    p.nchunks = (Cout + 63) / 64;
+    p.nchunks = (pc + 63) / 64;
     p.x = x;
     p.dw = dw;
     p.timeout_ns = wait_timeout_ns();
@@ -986,6 +996,57 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
     dwsep_fused_kernel<<<grid, kThreads, L.total, stream>>>(tmW, tmOut, p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_error(e, "launch dwsep_fused_kernel");
+    return ISAM_OK;
+}
+
+}  // namespace
+
+// Output channels in blocks of pc (a multiple of 16): the widest block whose
+// resident pointwise weights fit shared memory beside the A tiles, the input
+// ring and the epilogue staging.  Returns the block width, 0 if none fits.
+int dw_block_width(int W, int Cin, int Cout, const DeviceState &ds) {
+    for (int blocks = 1; blocks <= Cout / 16; ++blocks) {
+        const int pc = ((Cout + blocks - 1) / blocks + 15) / 16 * 16;
+        if (dw_block_fits(W, Cin, pc, ds)) return pc;
+    }
+    return 0;
+}
+
+int dwsep_plan(int W, int Cin, int Cout, const DeviceState &ds, int *out) {
+    if (Cin % 16 != 0 || Cin < 16 || Cin > 256 || Cout % 16 != 0 || Cout < 16 || Cout > 256)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_plan_info: needs Cin and Cout multiples of 16 in [16, 256]");
+    const int pc = dw_block_width(W, Cin, Cout, ds);
+    if (pc < 1) return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_plan_info: Cin=%d does not fit shared memory", Cin);
+    const int rt = dw_rows_per_tile(W, Cin, pc, ds);
+    out[0] = rt > 0 ? 0 : 1;
+    out[1] = rt;
+    out[2] = (Cout + pc - 1) / pc;
+    out[3] = pc;
+    return ISAM_OK;
+}
+
+int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
+                 const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t stream) {
+    if (Cin % 16 != 0 || Cin < 16 || Cin > 256 || Cout % 16 != 0 || Cout < 16 || Cout > 256)
+        return set_error(ISAM_ERR_UNSUPPORTED,
+                         "isam_dwsep_conv: needs Cin and Cout multiples of 16 in [16, 256] "
+                         "(Cin=%d Cout=%d)",
+                         Cin, Cout);
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dw) |
+         reinterpret_cast<uintptr_t>(pw) | reinterpret_cast<uintptr_t>(out)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: pointers must be 16-byte aligned");
+    const long long M = static_cast<long long>(N) * H * W;
+    if (M > (1ll << 31) - 256)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: N*H*W too large");
+    // One channel block at the benchmark layer; wide layers (Cin = Cout =
+    // 256, say) take several launches, each of which recomputes the
+    // depthwise stage for its block.
+    const int pc = dw_block_width(W, Cin, Cout, ds);
+    if (pc < 1) return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: Cin=%d does not fit shared memory", Cin);
+    for (int c0 = 0; c0 < Cout; c0 += pc) {
+        const int rc = dwsep_block(N, H, W, Cin, Cout, c0, std::min(pc, Cout - c0), x, dw, pw, out, ds, stream);
+        if (rc != ISAM_OK) return rc;
+    }
     return ISAM_OK;
 }
 

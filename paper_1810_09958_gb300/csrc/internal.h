@@ -108,5 +108,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
 
 int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
                  const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t s);
+// out[4]: kernel (0 row ring, 1 per-pixel), image rows per tile, channel blocks, block width.
+int dwsep_plan(int W, int Cin, int Cout, const DeviceState &ds, int *out);
 
 }  // namespace isam

@@ -64,11 +64,12 @@ def load():
         lib.isam_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_gru_forward_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
+        lib.isam_dwsep_plan_info.argtypes = [i, i, i, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
                      "isam_gemm_plan_info", "isam_gemm_plan_info2", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
                      "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_gru_forward_stack",
-                     "isam_dwsep_conv"):
+                     "isam_dwsep_conv", "isam_dwsep_plan_info"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
         return lib
@@ -250,3 +251,12 @@ def dwsep_conv(N, H, W, Cin, Cout, x, dw_w, pw_w, out) -> None:
     _dev(out, torch.float32, N * H * W * Cout, "out")
     _use_current_stream(lib)
     check(lib.isam_dwsep_conv(N, H, W, Cin, Cout, _ptr(x), _ptr(dw_w), _ptr(pw_w), _ptr(out)))
+
+
+def dwsep_plan(W, Cin, Cout) -> dict:
+    """isam_dwsep_plan_info: the kernel, tile rows and output-channel blocks
+    isam_dwsep_conv takes for this width and channel counts (nothing is launched)."""
+    lib = load()
+    out = (ctypes.c_int * 4)()
+    check(lib.isam_dwsep_plan_info(W, Cin, Cout, out))
+    return dict(zip(("kernel", "rows_per_tile", "blocks", "block_cout"), list(out)))

@@ -54,6 +54,8 @@ def test_gru_and_dwsep_reject_bad_args_without_cuda(lib):
     assert lib.isam_gru_forward_stack(2, 1, 1, 128, 0, p, p, p, None, None, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_dwsep_conv(1, 0, 4, 16, 16, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_dwsep_conv(1, 4, 4, 16, 16, p, None, p, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_dwsep_plan_info(0, 16, 16, p) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_dwsep_plan_info(4, 16, 16, None) == isam.ISAM_ERR_INVALID_ARG
 
 
 def test_binding_has_no_fallback(monkeypatch, tmp_path):

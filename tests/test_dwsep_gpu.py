@@ -85,6 +85,50 @@ def test_dwsep_ones_window_boundary_pattern():
         assert np.array_equal(got[0, :, :, k].astype(np.float64), want)
 
 
+def test_dwsep_benchmark_layer_plan():
+    """The benchmark layer runs as one launch of the row-ring kernel, two
+    image rows (112 pixels) per tile."""
+    assert isam.dwsep_plan(56, 128, 256) == {"kernel": 0, "rows_per_tile": 2, "blocks": 1, "block_cout": 256}
+
+
+# (N, H, W, Cin, Cout) with the plan the shared-memory budget gives: wide
+# layers whose resident pointwise weights do not fit in one launch run as
+# several output-channel blocks, each block's columns written with the
+# layer's full row pitch (unwritten outputs would keep the canary value).
+BLOCKED = [
+    ((2, 5, 8, 256, 256), (0, 6, 2, 128)),     # row ring, 6 rows per tile, 2 blocks
+    ((1, 6, 56, 192, 256), (0, 1, 2, 128)),    # row ring, one row per tile, 2 blocks
+    ((1, 4, 56, 256, 256), (1, 0, 4, 64)),     # per-pixel kernel, 4 blocks
+    ((1, 3, 130, 256, 256), (1, 0, 4, 64)),    # wider than one MMA block
+    ((2, 3, 11, 208, 80), (1, 0, 2, 48)),      # 48-wide blocks (a 16-column TMEM tail)
+    ((2, 4, 33, 144, 208), (1, 0, 2, 112)),
+    ((3, 2, 1, 256, 256), (0, 15, 2, 128)),    # one-pixel-wide images
+]
+
+
+@pytest.mark.parametrize("shape,plan", BLOCKED, ids=[str(s[0]) for s in BLOCKED])
+def test_dwsep_channel_blocks(shape, plan):
+    N, H, W, Cin, Cout = shape
+    got_plan = isam.dwsep_plan(W, Cin, Cout)
+    assert (got_plan["kernel"], got_plan["rows_per_tile"], got_plan["blocks"], got_plan["block_cout"]) == plan
+    x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=sum(shape) * 17 + Cout)
+    got = run_dwsep(x, dw, pw)
+    ref = oracle.dwsep(x, dw, pw)
+    assert nmax_err(got, ref) <= TOL, shape
+
+
+def test_dwsep_channel_blocks_integer_bit_exact():
+    """256 -> 256 channels in two blocks of 128: exact on integer data."""
+    N, H, W, Cin, Cout = 2, 5, 8, 256, 256
+    assert isam.dwsep_plan(W, Cin, Cout)["blocks"] == 2
+    x = synth.bf16_integers(11, (N, H, W, Cin), -3, 3)
+    dw = synth.bf16_integers(12, (3, 3, Cin), -2, 2)
+    pw = synth.bf16_integers(13, (Cin, Cout), -2, 2)
+    got = run_dwsep(x, dw, pw)
+    ref = oracle.dwsep(x, dw, pw)
+    assert np.array_equal(got.astype(np.float64), ref)
+
+
 def test_dwsep_unsupported_rejected():
     import ctypes
     import torch
@@ -94,4 +138,6 @@ def test_dwsep_unsupported_rejected():
     p = lambda t: ctypes.c_void_p(t.data_ptr())
     assert lib.isam_dwsep_conv(1, 4, 4, 24, 16, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
     assert lib.isam_dwsep_conv(1, 4, 4, 16, 272, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
-    assert lib.isam_dwsep_conv(1, 4, 4, 256, 256, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_dwsep_conv(1, 4, 4, 272, 16, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    out = (ctypes.c_int * 4)()
+    assert lib.isam_dwsep_plan_info(4, 16, 8, out) == isam.ISAM_ERR_UNSUPPORTED
