@@ -184,17 +184,17 @@ int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta
  * (h itself is carried in fp32).  Gates are evaluated in fp32.
  *
  * Supported: T >= 1, 1 <= batch <= 256, hidden a multiple of 32 in
- * [32, 1024] except 864, 928, 960 and 992 (one CTA per group would need 14
- * or 15 K atoms of U in shared memory); all pointers 16-byte aligned.
- * Otherwise ISAM_ERR_UNSUPPORTED.  A hidden of 64 k + 32 runs with one CTA
- * per group of 32 units and a last K atom half outside the matrix (zeros on
- * both sides of the product).  Batches above 32 run with the batch padded to 64 or
- * 128 rows (the MMA's N; 128 only with 4 K splits), in chunks of that many
- * rows, one launch per chunk; the rows are independent sequences.  The recurrence runs on hidden / 32 clusters of 4, 2
- * or 1 CTAs (4 when hidden is a multiple of 256, 2 for the other multiples of
- * 128, else 1), launched cooperatively so they are co-resident; each CTA keeps
- * a 96-row slice of U in shared memory, which for hidden = 960 (one CTA per
- * cluster, 15 K atoms) does not fit.
+ * [32, 1024]; all pointers 16-byte aligned.  Otherwise ISAM_ERR_UNSUPPORTED.
+ * Batches above 32 run with the batch padded to 64 or 128 rows (the MMA's N;
+ * 128 only with 4 K splits), in chunks of that many rows, one launch per
+ * chunk; the rows are independent sequences.  The recurrence runs on
+ * hidden / 32 clusters of K-split CTAs, launched cooperatively so they are
+ * co-resident: 4 splits when hidden is a multiple of 256, 2 for the other
+ * multiples of 128, otherwise 1 up to hidden 448, 2 up to 896 and 4 above.
+ * Each CTA keeps a 96-row slice of U over ceil(atoms / splits) 64-wide K
+ * atoms in shared memory; where the last CTA's range ends past the matrix (a
+ * hidden of 64 j + 32, or atoms not divisible by the splits) the tensor maps
+ * read zeros on both sides of the product.
  */
 int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x,
                      const isam_bf16 *W, const isam_bf16 *U, const float *b,
@@ -247,10 +247,9 @@ int isam_gru_forward_reset_before(int T, int batch, int hidden, const isam_bf16 
  * deterministic).  Either way the next layer sees bf16(h^l_t), as the
  * recurrent product sees bf16(h_{t-1}).
  *
- * Supported: as isam_gru_forward (batch up to 256); with layers > 1 and
- * batch <= 32, also the shared memory for both weight slices of the
- * per-layer chain, which excludes hidden 576, 704, 832 and 960
- * (ISAM_ERR_UNSUPPORTED).  Batches above 32 run layer by layer: the states
+ * Supported: as isam_gru_forward (batch up to 256, every multiple of 32
+ * for hidden; the K splits are chosen so that both weight slices of the
+ * per-layer chain fit).  Batches above 32 run layer by layer: the states
  * below are rounded to bf16 and projected by the GEMM, and each layer's
  * recurrence runs in chunks of padded rows.  Workspace: 2 x ks x T x batch x
  * 3*hidden fp32 (ks = 4, 2 or 1 K splits) beside isam_gru_forward's.
@@ -268,8 +267,8 @@ int isam_gru_forward_stack(int layers, int T, int batch, int hidden, int reset_b
  * because they can synchronise the whole device.
  *
  * Same arguments, layouts and equations as isam_gru_forward; batch up to 32
- * only (1 <= batch <= 32, hidden a multiple of 64 in [64, 1024] except 960,
- * any T >= 1).  The
+ * only (1 <= batch <= 32, hidden a multiple of 32 in [32, 1024], any
+ * T >= 1).  The
  * caller still passes every input and h_out.  The workspaces live in one
  * static 8 MiB device array inside libisam.so, which every GPU that loads the
  * library holds until the process exits; the input projection is computed in

@@ -67,7 +67,7 @@ struct GruParams {
     int T, batch, H;
     int bstride;               // batch rows between two steps of gx / h_out (the full batch; batch is this chunk's rows)
     int ks;                    // K splits per unit group = cluster size
-    int ka;                    // 64-wide K atoms per CTA (H / ks / 64)
+    int ka;                    // 64-wide K atoms per CTA (all atoms of H, rounded up, / ks)
     int uo;                    // units whose gates one CTA evaluates (32 / ks)
     int n_cta;                 // (H / 32) * ks
     int nq, qk;                // h arrives in nq pieces of qk atoms (nq * qk == ka)
@@ -512,12 +512,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-// K splits for a hidden size: each CTA's K range must be whole 64-wide atoms
-// (a hidden of 64 k + 32 has one CTA per group and a last, half-filled atom).
-int gru_splits(int H) { return (H % 256 == 0) ? 4 : (H % 128 == 0) ? 2 : 1; }
+// K splits for a hidden size (the cluster size).  CTA k of a cluster takes
+// the 64-wide K atoms k * ka .. k * ka + ka - 1 (ka = gru_atoms); the last
+// range may end past the matrix, and a hidden of 64 j + 32 ends half an atom
+// inside it: the tensor maps read zeros there on both sides of the product.
+// 4 splits for multiples of 256, 2 for the other multiples of 128; otherwise
+// one CTA per group up to 7 atoms (hidden <= 448), 2 up to 14 atoms and 4
+// above, so that a CTA's slice of U, the next layer's slice of W (stacks) and
+// its h tiles fit shared memory together at every multiple of 32.
+int gru_splits(int H) {
+    if (H % 256 == 0) return 4;
+    if (H % 128 == 0) return 2;
+    return H <= 448 ? 1 : H <= 896 ? 2 : 4;
+}
 
-// 64-wide K atoms per CTA.
-int gru_atoms(int H) { return (H / gru_splits(H) + 63) / 64; }
+// 64-wide K atoms per CTA: the hidden's atoms, rounded up, over the splits.
+int gru_atoms(int H) {
+    const int ks = gru_splits(H);
+    return ((H + 63) / 64 + ks - 1) / ks;
+}
 
 size_t gru_smem_bytes(int H, bool has_next = false, int bp = kBatchPad) {
     return static_cast<size_t>(gru_layout(gru_atoms(H), has_next, bp).total);
@@ -967,10 +980,10 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_noalloc: sizes must be >= 1");
     if (!x || !W || !U || !b || !h_out)
         return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_forward_noalloc: null pointer");
-    if (batch > kBatchPad || H % 64 != 0 || H > 1024 || H < 64)
+    if (batch > kBatchPad || H % 32 != 0 || H > 1024 || H < 32)
         return set_error(ISAM_ERR_UNSUPPORTED,
-                         "isam_gru_forward_noalloc: needs batch <= 32 and hidden a multiple of 64 "
-                         "in [64, 1024] (batch=%d hidden=%d)",
+                         "isam_gru_forward_noalloc: needs batch <= 32 and hidden a multiple of 32 "
+                         "in [32, 1024] (batch=%d hidden=%d)",
                          batch, H);
     if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
          reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |

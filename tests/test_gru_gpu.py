@@ -111,8 +111,7 @@ def test_gru_unsupported_shapes_rejected():
     p = lambda t: ctypes.c_void_p(t.data_ptr())
     assert lib.isam_gru_forward(1, 257, 64, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
     assert lib.isam_gru_forward(1, 1, 80, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
-    # hidden 960: one CTA per cluster would need 15 K atoms of U (does not fit).
-    assert lib.isam_gru_forward(1, 1, 960, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_gru_forward(1, 1, 1056, p(z), p(z), p(z), p(f), None, p(f)) == isam.ISAM_ERR_UNSUPPORTED
 
 
 @pytest.mark.parametrize("reset_before", [False, True])
@@ -248,10 +247,26 @@ def test_gru_wide_batch_rows_independent_of_chunking():
 # the last 64-wide K atom half outside the matrix (zero-filled on both sides).
 
 @pytest.mark.parametrize("T,batch,H,rb", [(5, 3, 32, False), (4, 17, 96, False), (6, 32, 160, True),
-                                          (3, 8, 480, False), (4, 50, 224, False), (3, 5, 800, True)])
+                                          (3, 8, 480, False), (4, 50, 224, False), (3, 5, 800, True),
+                                          (3, 6, 864, False), (3, 7, 992, True), (3, 40, 928, False)])
 def test_gru_hidden_odd_multiple_of_32(T, batch, H, rb):
     x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 17 + batch + H * 3)
     h0 = synth.f32_uniform(H + batch, (batch, H))
+    got = run_gru(x, W, U, b, h0, reset_before=rb)
+    ref = oracle.gru_forward(x, W, U, b, h0, reset_before=rb)
+    assert nmax_err(got, ref) <= TOL, nmax_err(got, ref)
+
+
+# ---- K ranges that end past the matrix: hidden 480 and 576-896 (other than
+# multiples of 128) run 2 K splits, 928-992 run 4, each CTA holding
+# ceil(atoms / splits) whole atoms; the last CTA's range ends in zeros read by
+# the tensor maps (at 960 with 4 splits its last atom lies wholly outside U).
+
+@pytest.mark.parametrize("T,batch,H,rb", [(3, 5, 960, False), (3, 32, 960, True), (4, 9, 576, False),
+                                          (3, 70, 960, False), (4, 12, 704, True)])
+def test_gru_uneven_k_splits(T, batch, H, rb):
+    x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=T * 29 + batch + H * 5)
+    h0 = synth.f32_uniform(H + batch + 1, (batch, H))
     got = run_gru(x, W, U, b, h0, reset_before=rb)
     ref = oracle.gru_forward(x, W, U, b, h0, reset_before=rb)
     assert nmax_err(got, ref) <= TOL, nmax_err(got, ref)

@@ -110,8 +110,7 @@ def test_gru_stack_unsupported_shapes_rejected():
     f = torch.zeros(1 << 22, dtype=torch.float32, device="cuda")
     lib = isam.load()
     p = lambda t: ctypes.c_void_p(t.data_ptr())
-    # hidden 832: one CTA per cluster holds 13 K atoms; two weight slices do not fit.
-    assert lib.isam_gru_forward_stack(2, 1, 1, 832, 0, p(z), p(z), p(z), p(f), None, p(f)) == \
+    assert lib.isam_gru_forward_stack(2, 1, 1, 80, 0, p(z), p(z), p(z), p(f), None, p(f)) == \
         isam.ISAM_ERR_UNSUPPORTED
     assert lib.isam_gru_forward_stack(2, 1, 257, 128, 0, p(z), p(z), p(z), p(f), None, p(f)) == \
         isam.ISAM_ERR_UNSUPPORTED
@@ -184,7 +183,11 @@ def test_gru_stack_wide_batch(L, T, batch, H, rb):
         assert nmax_err(got[l], ref[l]) <= TOL, (l, nmax_err(got[l], ref[l]))
 
 
-@pytest.mark.parametrize("L,T,batch,H,rb", [(2, 4, 9, 96, False), (3, 3, 32, 352, True)])
+@pytest.mark.parametrize("L,T,batch,H,rb", [(2, 4, 9, 96, False), (3, 3, 32, 352, True),
+                                            # per-layer chain with uneven K ranges: 2 splits
+                                            # (480, 832) and 4 splits (960, 992)
+                                            (2, 3, 7, 480, False), (2, 3, 5, 832, True),
+                                            (2, 3, 6, 960, False), (2, 2, 32, 992, True)])
 def test_gru_stack_hidden_odd_multiple_of_32(L, T, batch, H, rb):
     x, W, U, b, h0 = synth.gru_stack_operands(L, T, batch, H, seed=L + T + batch + H)
     got = run_stack(x, W, U, b, h0, rb)

@@ -33,7 +33,7 @@ def lib():
     return isam.load()
 
 
-@pytest.mark.parametrize("T,batch,H", [(128, 32, 1024), (9, 5, 192)])
+@pytest.mark.parametrize("T,batch,H", [(128, 32, 1024), (9, 5, 192), (6, 7, 96), (5, 32, 960)])
 def test_noalloc_matches_regular_entry_twice(lib, T, batch, H):
     import torch
     x, W, U, b, _ = synth.gru_operands(T, batch, H, seed=9000 + H)
