@@ -260,22 +260,46 @@ def time_grouped(isam, probs, steps, warmup):
 
 
 def time_e2e(isam, probs, steps, warmup):
-    """The sweep through host buffers: per step, pinned host -> device copies of
-    every operand, one isam_gemm_grouped launch, device -> host copies of every
-    result.  Steps alternate between two device operand sets so that the input
-    copies of step k + 1 (copy stream) overlap the GEMM and the result copies
-    of step k; events order each set's copies, GEMM and read-back, and every
-    step still moves its own inputs in and its result out."""
+    """The sweep through host buffers: per step, the pinned host -> device copy
+    of every operand, one isam_gemm_grouped launch, the device -> host copy of
+    every result.  Each step's operands sit back to back in one pinned host
+    buffer and one device buffer (likewise the results), so a step moves them
+    in one copy each way.  Steps alternate between two device operand sets so
+    that the input copy of step k + 1 (copy stream) overlaps the GEMM and the
+    result copy of step k; events order each set's copies, GEMM and read-back,
+    and every step still moves its own inputs in and its result out."""
     import torch
-    host = []
+
+    def layout(sizes):
+        offs, at = [], 0
+        for n in sizes:
+            offs.append(at)
+            at += (n + 255) // 256 * 256
+        return offs, at
+
+    in_sizes = []
     for p in probs:
-        host.append({"A": p["A"].cpu().pin_memory(), "B": p["B"].cpu().pin_memory(),
-                     "C": torch.empty(p["M"] * p["N"], dtype=torch.float32).pin_memory()})
-    h2d = sum(h["A"].numel() * 2 + h["B"].numel() * 2 for h in host)
-    d2h = sum(h["C"].numel() * 4 for h in host)
-    sets = [[{"A": p["A"], "B": p["B"], "C": p["C"]} for p in probs],
-            [{"A": torch.empty_like(p["A"]), "B": torch.empty_like(p["B"]), "C": torch.empty_like(p["C"])}
-             for p in probs]]
+        in_sizes += [p["A"].numel() * 2, p["B"].numel() * 2]
+    in_offs, in_total = layout(in_sizes)
+    out_offs, out_total = layout([p["M"] * p["N"] * 4 for p in probs])
+    host_in = torch.empty(in_total, dtype=torch.uint8).pin_memory()
+    host_out = torch.empty(out_total, dtype=torch.uint8).pin_memory()
+    for j, p in enumerate(probs):
+        for t, name in ((2 * j, "A"), (2 * j + 1, "B")):
+            host_in[in_offs[t]:in_offs[t] + in_sizes[t]].copy_(p[name].cpu().view(torch.uint8))
+    h2d, d2h = in_total, out_total  # the bytes each step's two copies move
+    dev_in = [torch.empty(in_total, dtype=torch.uint8, device=probs[0]["A"].device) for _ in range(2)]
+    dev_out = [torch.empty(out_total, dtype=torch.uint8, device=probs[0]["A"].device) for _ in range(2)]
+
+    def views(buf_in, buf_out):
+        out = []
+        for j, p in enumerate(probs):
+            a0, b0 = in_offs[2 * j], in_offs[2 * j + 1]
+            out.append({"A": buf_in[a0:a0 + in_sizes[2 * j]].view(torch.bfloat16),
+                        "B": buf_in[b0:b0 + in_sizes[2 * j + 1]].view(torch.bfloat16),
+                        "C": buf_out[out_offs[j]:out_offs[j] + p["M"] * p["N"] * 4].view(torch.float32)})
+        return out
+    sets = [views(dev_in[i], dev_out[i]) for i in range(2)]
     calls = [isam.GroupedGemm([(p["M"], p["N"], p["K"], p["tA"], 0, 1.0, d["A"], d["B"], 0.0, d["C"])
                                for p, d in zip(probs, ds)]) for ds in sets]
     s_in, s_run, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
@@ -287,9 +311,7 @@ def time_e2e(isam, probs, steps, warmup):
         with torch.cuda.stream(s_in):
             if not first[i]:
                 s_in.wait_event(ev["run"][i])  # set i's operands are no longer read
-            for p, h in zip(sets[i], host):
-                p["A"].copy_(h["A"], non_blocking=True)
-                p["B"].copy_(h["B"], non_blocking=True)
+            dev_in[i].copy_(host_in, non_blocking=True)
             ev["in"][i].record(s_in)
         with torch.cuda.stream(s_run):
             s_run.wait_event(ev["in"][i])
@@ -299,8 +321,7 @@ def time_e2e(isam, probs, steps, warmup):
             ev["run"][i].record(s_run)
         with torch.cuda.stream(s_out):
             s_out.wait_event(ev["run"][i])
-            for p, h in zip(sets[i], host):
-                h["C"].copy_(p["C"], non_blocking=True)
+            host_out.copy_(dev_out[i], non_blocking=True)
             ev["out"][i].record(s_out)
         first[i] = False
 
@@ -756,7 +777,7 @@ def main(argv=None):
                                    "timed-region CUDA events on the replay stream / steps"},
             "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-                    "what": "pinned host operands copied in, isam_gemm_grouped, results copied out; two device operand sets, step k+1 inputs copied while step k computes"},
+                    "what": "per step: every operand copied in from one pinned host buffer (one copy), isam_gemm_grouped, every result copied out to one pinned host buffer (one copy); two device operand sets, step k+1 inputs copied while step k computes"},
             "gpu_launches": launches,
             "clocks": sampler.summary(*window) if sampler else None,
             "per_call_sweep": {
