@@ -329,6 +329,41 @@ int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
  */
 int isam_dwsep_plan_info(int W, int Cin, int Cout, int *out);
 
+/*
+ * isam_dwsep_plan_info's plan for a device whose CTAs may opt in to
+ * smem_optin bytes of shared memory (232448 on sm_103a); host arithmetic
+ * only, no CUDA call, so it runs without a GPU.  ISAM_ERR_INVALID_ARG for
+ * sizes < 1 or a null out.
+ */
+int isam_dwsep_plan_for(int W, int Cin, int Cout, int smem_optin, int *out);
+
+/*
+ * The plan isam_gru_forward (layers = 1) or isam_gru_forward_stack takes for
+ * this batch and hidden size (it does not depend on T); nothing is launched.
+ * out[7]:
+ *   out[0]  K splits per group of 32 hidden units (cluster size: 1, 2 or 4)
+ *   out[1]  64-wide K atoms of U each CTA keeps resident
+ *   out[2]  padded batch of the recurrence (the MMA's N: 32, 64 or 128)
+ *   out[3]  CTAs of the recurrence (hidden / 32 x splits)
+ *   out[4]  shared memory of one recurrence CTA in bytes (the largest kernel
+ *           the call launches)
+ *   out[5]  how layers run: 0 one layer; 1 pairs of layers in one kernel;
+ *           2 one kernel per layer that also computes the next layer's input
+ *           projection; 3 layer by layer, the batch in chunks of out[2] rows
+ *   out[6]  recurrence launches per layer (batch chunks)
+ * Returns ISAM_ERR_UNSUPPORTED (with the reason) for shapes the call rejects,
+ * ISAM_ERR_INVALID_ARG for sizes < 1, reset_before not 0 or 1, or a null out.
+ */
+int isam_gru_plan_info(int layers, int batch, int hidden, int reset_before, int *out);
+
+/*
+ * isam_gru_plan_info's plan for a device with num_sms SMs (152 on a GB300)
+ * and smem_optin bytes of shared memory per CTA; host arithmetic only, no
+ * CUDA call.
+ */
+int isam_gru_plan_for(int layers, int batch, int hidden, int reset_before, int num_sms, int smem_optin,
+                      int *out);
+
 #ifdef __cplusplus
 }
 #endif

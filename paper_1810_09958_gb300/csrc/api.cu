@@ -423,7 +423,45 @@ int isam_dwsep_plan_info(int W, int Cin, int Cout, int *out) {
     int rc;
     DeviceState *ds = device_state(&rc);
     if (!ds) return rc;
-    return dwsep_plan(W, Cin, Cout, *ds, out);
+    return dwsep_plan(W, Cin, Cout, ds->max_smem_optin, out);
+}
+
+int isam_dwsep_plan_for(int W, int Cin, int Cout, int smem_optin, int *out) {
+    if (W < 1 || Cin < 1 || Cout < 1 || smem_optin < 1 || !out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_dwsep_plan_for: sizes must be >= 1, out non-null");
+    return dwsep_plan(W, Cin, Cout, smem_optin, out);
+}
+
+namespace {
+int gru_plan_out(int layers, int batch, int hidden, int reset_before, int num_sms, int smem_optin, int *out) {
+    GruPlan g;
+    const int rc = gru_plan(layers, batch, hidden, reset_before, num_sms, smem_optin, &g);
+    if (rc != ISAM_OK) return rc;
+    out[0] = g.ks;
+    out[1] = g.ka;
+    out[2] = g.bp;
+    out[3] = g.n_cta;
+    out[4] = g.smem;
+    out[5] = g.path;
+    out[6] = g.chunks;
+    return ISAM_OK;
+}
+}  // namespace
+
+int isam_gru_plan_info(int layers, int batch, int hidden, int reset_before, int *out) {
+    if (layers < 1 || batch < 1 || hidden < 1 || (reset_before != 0 && reset_before != 1) || !out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_plan_info: sizes must be >= 1, reset_before 0 or 1");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gru_plan_out(layers, batch, hidden, reset_before, ds->num_sms, ds->max_smem_optin, out);
+}
+
+int isam_gru_plan_for(int layers, int batch, int hidden, int reset_before, int num_sms, int smem_optin, int *out) {
+    if (layers < 1 || batch < 1 || hidden < 1 || (reset_before != 0 && reset_before != 1) || num_sms < 1 ||
+        smem_optin < 1 || !out)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gru_plan_for: sizes must be >= 1, reset_before 0 or 1");
+    return gru_plan_out(layers, batch, hidden, reset_before, num_sms, smem_optin, out);
 }
 
 }  // extern "C"

@@ -891,15 +891,15 @@ __global__ void __launch_bounds__(kRThreads, 1)
 // channels, or 0 where that kernel does not apply (an image wider than one
 // MMA block, a channel count its thread mapping does not divide, or no ring
 // that fits shared memory beside the block's weights).
-int dw_rows_per_tile(int W, int Cin, int pc, const DeviceState &ds) {
+int dw_rows_per_tile(int W, int Cin, int pc, int smem_optin) {
     int rt = (W <= kBM && kRProd % (Cin / 4) == 0) ? kBM / W : 0;
     if (rt > (kRingMax - 2) / 2) rt = (kRingMax - 2) / 2;
-    while (rt > 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total > ds.max_smem_optin) --rt;
-    return (rt >= 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total <= ds.max_smem_optin) ? rt : 0;
+    while (rt > 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total > smem_optin) --rt;
+    return (rt >= 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total <= smem_optin) ? rt : 0;
 }
 
-bool dw_block_fits(int W, int Cin, int pc, const DeviceState &ds) {
-    return dw_rows_per_tile(W, Cin, pc, ds) > 0 || dw_layout(Cin, pc).total <= ds.max_smem_optin;
+bool dw_block_fits(int W, int Cin, int pc, int smem_optin) {
+    return dw_rows_per_tile(W, Cin, pc, smem_optin) > 0 || dw_layout(Cin, pc).total <= smem_optin;
 }
 
 // One launch for output channels c0 .. c0 + pc - 1 of a layer with Cout
@@ -911,7 +911,7 @@ int dwsep_block(int N, int H, int W, int Cin, int Cout, int c0, int pc, const ui
     const uint16_t *pwb = pw + c0;
     float *outb = out + c0;
     int rc;
-    const int rt = dw_rows_per_tile(W, Cin, pc, ds);
+    const int rt = dw_rows_per_tile(W, Cin, pc, ds.max_smem_optin);
     if (rt > 0) {
         // Row-ring path: rt image rows per tile, 2 * rt + 2 rows resident.
         const DwRowLayout RL = dw_row_layout(W, Cin, pc, 2 * rt + 2);
@@ -1004,20 +1004,20 @@ int dwsep_block(int N, int H, int W, int Cin, int Cout, int c0, int pc, const ui
 // Output channels in blocks of pc (a multiple of 16): the widest block whose
 // resident pointwise weights fit shared memory beside the A tiles, the input
 // ring and the epilogue staging.  Returns the block width, 0 if none fits.
-int dw_block_width(int W, int Cin, int Cout, const DeviceState &ds) {
+int dw_block_width(int W, int Cin, int Cout, int smem_optin) {
     for (int blocks = 1; blocks <= Cout / 16; ++blocks) {
         const int pc = ((Cout + blocks - 1) / blocks + 15) / 16 * 16;
-        if (dw_block_fits(W, Cin, pc, ds)) return pc;
+        if (dw_block_fits(W, Cin, pc, smem_optin)) return pc;
     }
     return 0;
 }
 
-int dwsep_plan(int W, int Cin, int Cout, const DeviceState &ds, int *out) {
+int dwsep_plan(int W, int Cin, int Cout, int smem_optin, int *out) {
     if (Cin % 16 != 0 || Cin < 16 || Cin > 256 || Cout % 16 != 0 || Cout < 16 || Cout > 256)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_plan_info: needs Cin and Cout multiples of 16 in [16, 256]");
-    const int pc = dw_block_width(W, Cin, Cout, ds);
+    const int pc = dw_block_width(W, Cin, Cout, smem_optin);
     if (pc < 1) return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_plan_info: Cin=%d does not fit shared memory", Cin);
-    const int rt = dw_rows_per_tile(W, Cin, pc, ds);
+    const int rt = dw_rows_per_tile(W, Cin, pc, smem_optin);
     out[0] = rt > 0 ? 0 : 1;
     out[1] = rt;
     out[2] = (Cout + pc - 1) / pc;
@@ -1041,7 +1041,7 @@ int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, cons
     // One channel block at the benchmark layer; wide layers (Cin = Cout =
     // 256, say) take several launches, each of which recomputes the
     // depthwise stage for its block.
-    const int pc = dw_block_width(W, Cin, Cout, ds);
+    const int pc = dw_block_width(W, Cin, Cout, ds.max_smem_optin);
     if (pc < 1) return set_error(ISAM_ERR_UNSUPPORTED, "isam_dwsep_conv: Cin=%d does not fit shared memory", Cin);
     for (int c0 = 0; c0 < Cout; c0 += pc) {
         const int rc = dwsep_block(N, H, W, Cin, Cout, c0, std::min(pc, Cout - c0), x, dw, pw, out, ds, stream);

@@ -698,50 +698,81 @@ __global__ void __launch_bounds__(256) states_to_bf16_kernel(const float4 *in, u
 
 }  // namespace
 
-int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before, const uint16_t *x,
-                     const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
-                     DeviceState &ds, cudaStream_t stream) {
+int gru_plan(int layers, int batch, int hidden, int reset_before, int num_sms, int smem_optin, GruPlan *g) {
     const int H = hidden;
-    if (batch > kBatchMax || H % 32 != 0 || H > 1024 || H < 32)
+    if (layers < 1 || batch < 1 || batch > kBatchMax || H % 32 != 0 || H > 1024 || H < 32)
         return set_error(ISAM_ERR_UNSUPPORTED,
                          "isam_gru_forward: needs batch <= 256 and hidden a multiple of 32 in "
                          "[32, 1024] (batch=%d hidden=%d)",
                          batch, H);
-    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
-         reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |
-         reinterpret_cast<uintptr_t>(h0) | reinterpret_cast<uintptr_t>(h_out)) & 15u)
-        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: pointers must be 16-byte aligned");
-    const int n_cta = gru_cta_count(H);
-    if (n_cta > ds.num_sms)
-        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: %d CTAs cannot be co-resident", n_cta);
+    GruPlan q;
+    q.ks = gru_splits(H);
+    q.ka = gru_atoms(H);
+    q.n_cta = gru_cta_count(H);
+    if (q.n_cta > num_sms)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: %d CTAs cannot be co-resident", q.n_cta);
     // Padded batch of the recurrence (the MMA's N): 32 for batch <= 32, with
     // every feature; above that the narrowest of 64 and 128 that holds the
     // batch (else the widest that fits beside U), the batch running in chunks
     // of that many rows (one launch each; each chunk's rows are independent
     // sequences).  A step costs about the same whatever the width's fill.
     const bool chunked = batch > kBatchPad;
-    int bp = kBatchPad;
+    q.bp = kBatchPad;
     if (chunked) {
         auto fits = [&](int cand) {
-            return gru_bp_ok(gru_splits(H), cand) &&
-                   gru_smem_bytes(H, false, cand) <= static_cast<size_t>(ds.max_smem_optin);
+            return gru_bp_ok(q.ks, cand) && gru_smem_bytes(H, false, cand) <= static_cast<size_t>(smem_optin);
         };
         if (batch <= 64 && fits(64))
-            bp = 64;
+            q.bp = 64;
         else if (fits(128))
-            bp = 128;
+            q.bp = 128;
         else if (fits(64))
-            bp = 64;
+            q.bp = 64;
     }
-    const size_t smem_last = gru_smem_bytes(H, false, bp);
+    const size_t smem_last = gru_smem_bytes(H, false, q.bp);
     const size_t smem_next = gru_smem_bytes(H, true);
-    if (smem_last > static_cast<size_t>(ds.max_smem_optin))
+    if (smem_last > static_cast<size_t>(smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: hidden too large for shared memory");
-    if (layers > 1 && !chunked && smem_next > static_cast<size_t>(ds.max_smem_optin))
+    if (layers > 1 && !chunked && smem_next > static_cast<size_t>(smem_optin))
         return set_error(ISAM_ERR_UNSUPPORTED,
                          "isam_gru_forward_stack: hidden %d leaves no room for the next layer's "
                          "weights beside the recurrent ones (%zu bytes of shared memory)",
                          H, smem_next);
+    q.chunks = (batch + q.bp - 1) / q.bp;
+    q.smem = static_cast<int>(smem_last);
+    if (layers == 1) {
+        q.path = 0;
+    } else if (chunked) {
+        q.path = 3;
+    } else {
+        const char *nw = getenv("ISAM_NO_WAVE");
+        if (!reset_before && !(nw && nw[0] == '1') && gru_wave_fits(H, batch, num_sms, smem_optin)) {
+            q.path = 1;
+            q.smem = static_cast<int>(gru_wave_smem_bytes(H));
+        } else {
+            q.path = 2;
+            q.smem = static_cast<int>(smem_next);
+        }
+    }
+    *g = q;
+    return ISAM_OK;
+}
+
+int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before, const uint16_t *x,
+                     const uint16_t *W, const uint16_t *U, const float *b, const float *h0, float *h_out,
+                     DeviceState &ds, cudaStream_t stream) {
+    const int H = hidden;
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(W) |
+         reinterpret_cast<uintptr_t>(U) | reinterpret_cast<uintptr_t>(b) |
+         reinterpret_cast<uintptr_t>(h0) | reinterpret_cast<uintptr_t>(h_out)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gru_forward: pointers must be 16-byte aligned");
+    GruPlan plan;
+    int prc = gru_plan(layers, batch, H, reset_before, ds.num_sms, ds.max_smem_optin, &plan);
+    if (prc != ISAM_OK) return prc;
+    const bool chunked = batch > kBatchPad;  // path 3 when layers > 1
+    const int bp = plan.bp;
+    const size_t smem_last = gru_smem_bytes(H, false, bp);
+    const size_t smem_next = gru_smem_bytes(H, true);
 
     int rc;
     const size_t seq_rows = static_cast<size_t>(T) * batch;
@@ -858,8 +889,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
     // step behind layer l, its projection computed from the same h tiles.
     // Between pairs (and for an odd last layer) the layer below's states are
     // rounded to bf16 and projected by the GEMM.
-    const char *nw = getenv("ISAM_NO_WAVE");
-    if (layers >= 2 && !reset_before && !(nw && nw[0] == '1') && gru_wave_supported(H, batch, ds)) {
+    if (plan.path == 1) {
         if (layers > 2 && (rc = ensure_ws(reinterpret_cast<void **>(&ds.gru_xb), &ds.gru_xb_bytes,
                                           seq_rows * H * sizeof(uint16_t), "allocating the GRU layer-input buffer")))
             return rc;

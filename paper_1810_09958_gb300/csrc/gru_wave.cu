@@ -410,10 +410,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 size_t gru_wave_smem_bytes(int H) { return static_cast<size_t>(wave_layout(H / (kKS * 64)).total); }
 
-bool gru_wave_supported(int H, int batch, const DeviceState &ds) {
+bool gru_wave_fits(int H, int batch, int num_sms, int smem_optin) {
     if (H % 256 != 0 || H < 256 || H > 1024 || batch < 1 || batch > kBatchPad) return false;
-    if (H / kGroup * kKS > ds.num_sms) return false;
-    return gru_wave_smem_bytes(H) <= static_cast<size_t>(ds.max_smem_optin);
+    if (H / kGroup * kKS > num_sms) return false;
+    return gru_wave_smem_bytes(H) <= static_cast<size_t>(smem_optin);
+}
+
+bool gru_wave_supported(int H, int batch, const DeviceState &ds) {
+    return gru_wave_fits(H, batch, ds.num_sms, ds.max_smem_optin);
 }
 
 namespace {

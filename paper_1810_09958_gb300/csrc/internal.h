@@ -98,6 +98,21 @@ int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *
 // product, hidden a multiple of 256): layer a's projection gx_a is given,
 // layer b's comes from W_b and layer a's states inside the kernel.
 bool gru_wave_supported(int H, int batch, const DeviceState &ds);
+bool gru_wave_fits(int H, int batch, int num_sms, int smem_optin);
+size_t gru_wave_smem_bytes(int H);
+
+// How a GRU call runs on a device with num_sms SMs and smem_optin bytes of
+// shared memory per CTA (host arithmetic only, no CUDA call).
+struct GruPlan {
+    int ks = 0;       // K splits per group of 32 units (cluster size)
+    int ka = 0;       // 64-wide K atoms per CTA
+    int bp = 0;       // padded batch (the MMA's N)
+    int n_cta = 0;    // CTAs of the recurrence
+    int smem = 0;     // shared memory of one recurrence CTA (the largest launched)
+    int path = 0;     // 0 one layer, 1 layer pairs in one kernel, 2 per-layer chain, 3 layer by layer in batch chunks
+    int chunks = 0;   // recurrence launches per layer
+};
+int gru_plan(int layers, int batch, int hidden, int reset_before, int num_sms, int smem_optin, GruPlan *g);
 int gru_wave_launch(int T, int batch, int H, const float *gx_a, const uint16_t *U_a, const uint16_t *W_b,
                     const uint16_t *U_b, const float *b_a, const float *b_b, const float *h0_a,
                     const float *h0_b, float *out_a, float *out_b, uint16_t *hx_a, uint16_t *hx_b,
@@ -109,6 +124,6 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
 int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
                  const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t s);
 // out[4]: kernel (0 row ring, 1 per-pixel), image rows per tile, channel blocks, block width.
-int dwsep_plan(int W, int Cin, int Cout, const DeviceState &ds, int *out);
+int dwsep_plan(int W, int Cin, int Cout, int smem_optin, int *out);
 
 }  // namespace isam

@@ -65,11 +65,15 @@ def load():
         lib.isam_gru_forward_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         lib.isam_dwsep_plan_info.argtypes = [i, i, i, P]
+        lib.isam_dwsep_plan_for.argtypes = [i, i, i, i, P]
+        lib.isam_gru_plan_info.argtypes = [i, i, i, i, P]
+        lib.isam_gru_plan_for.argtypes = [i, i, i, i, i, i, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
                      "isam_gemm_plan_info", "isam_gemm_plan_info2", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
                      "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_gru_forward_stack",
-                     "isam_dwsep_conv", "isam_dwsep_plan_info"):
+                     "isam_dwsep_conv", "isam_dwsep_plan_info", "isam_dwsep_plan_for",
+                     "isam_gru_plan_info", "isam_gru_plan_for"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
         return lib
@@ -253,10 +257,31 @@ def dwsep_conv(N, H, W, Cin, Cout, x, dw_w, pw_w, out) -> None:
     check(lib.isam_dwsep_conv(N, H, W, Cin, Cout, _ptr(x), _ptr(dw_w), _ptr(pw_w), _ptr(out)))
 
 
-def dwsep_plan(W, Cin, Cout) -> dict:
+_DWSEP_PLAN_KEYS = ("kernel", "rows_per_tile", "blocks", "block_cout")
+_GRU_PLAN_KEYS = ("splits", "atoms", "batch_pad", "ctas", "smem", "path", "chunks")
+
+
+def dwsep_plan(W, Cin, Cout, smem_optin=None) -> dict:
     """isam_dwsep_plan_info: the kernel, tile rows and output-channel blocks
-    isam_dwsep_conv takes for this width and channel counts (nothing is launched)."""
+    isam_dwsep_conv takes for this width and channel counts (nothing is
+    launched); with smem_optin, isam_dwsep_plan_for on those limits (no GPU)."""
     lib = load()
     out = (ctypes.c_int * 4)()
-    check(lib.isam_dwsep_plan_info(W, Cin, Cout, out))
-    return dict(zip(("kernel", "rows_per_tile", "blocks", "block_cout"), list(out)))
+    if smem_optin is None:
+        check(lib.isam_dwsep_plan_info(W, Cin, Cout, out))
+    else:
+        check(lib.isam_dwsep_plan_for(W, Cin, Cout, smem_optin, out))
+    return dict(zip(_DWSEP_PLAN_KEYS, list(out)))
+
+
+def gru_plan(layers, batch, hidden, reset_before=False, num_sms=None, smem_optin=None) -> dict:
+    """isam_gru_plan_info: K splits, padded batch, CTAs, shared memory and the
+    layer schedule of a GRU call (nothing is launched); with num_sms and
+    smem_optin, isam_gru_plan_for on those limits (no GPU)."""
+    lib = load()
+    out = (ctypes.c_int * 7)()
+    if num_sms is None:
+        check(lib.isam_gru_plan_info(layers, batch, hidden, int(bool(reset_before)), out))
+    else:
+        check(lib.isam_gru_plan_for(layers, batch, hidden, int(bool(reset_before)), num_sms, smem_optin, out))
+    return dict(zip(_GRU_PLAN_KEYS, list(out)))

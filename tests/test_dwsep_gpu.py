@@ -141,3 +141,8 @@ def test_dwsep_unsupported_rejected():
     assert lib.isam_dwsep_conv(1, 4, 4, 272, 16, p(z), p(z), p(z), p(f)) == isam.ISAM_ERR_UNSUPPORTED
     out = (ctypes.c_int * 4)()
     assert lib.isam_dwsep_plan_info(4, 16, 8, out) == isam.ISAM_ERR_UNSUPPORTED
+
+
+def test_dwsep_plan_on_the_device_matches_the_host_plan():
+    for (W, cin, cout) in [(56, 128, 256), (56, 256, 256), (8, 256, 256), (130, 48, 16)]:
+        assert isam.dwsep_plan(W, cin, cout) == isam.dwsep_plan(W, cin, cout, smem_optin=232448)

@@ -270,3 +270,14 @@ def test_gru_uneven_k_splits(T, batch, H, rb):
     got = run_gru(x, W, U, b, h0, reset_before=rb)
     ref = oracle.gru_forward(x, W, U, b, h0, reset_before=rb)
     assert nmax_err(got, ref) <= TOL, nmax_err(got, ref)
+
+
+def test_gru_plan_on_the_device_matches_the_host_plan():
+    """isam_gru_plan_info (this device's limits) equals isam_gru_plan_for with
+    the limits the host-side planner tests assume (152 SMs, 232448 bytes)."""
+    import torch
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    for (layers, batch, H, rb) in [(1, 32, 1024, False), (2, 32, 1024, False), (2, 32, 1024, True),
+                                   (1, 200, 960, False), (3, 8, 864, True)]:
+        assert isam.gru_plan(layers, batch, H, rb) == isam.gru_plan(layers, batch, H, rb, num_sms=sms,
+                                                                     smem_optin=232448)

@@ -1,0 +1,139 @@
+"""The GRU and depthwise-separable planners, run on the host through the C ABI
+(isam_gru_plan_for, isam_dwsep_plan_for: host arithmetic, no CUDA call) with
+a GB300's limits: 152 SMs, 232448 bytes of opt-in shared memory per CTA.
+Every shape inside the boundary's support limits (GRU: batch <= 256, hidden
+any multiple of 32 up to 1024; dwsep: Cin and Cout multiples of 16 up to 256,
+any width) must get a plan that fits the device, and the plans must keep the
+invariants the kernels rely on."""
+import math
+
+import pytest
+
+from paper_1810_09958_gb300 import build, isam
+
+SMS = 152
+SMEM = 232448
+HIDDEN = list(range(32, 1025, 32))
+BATCH = [1, 7, 32, 33, 64, 65, 100, 128, 129, 256]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    isam.load()
+
+
+def gru_plan(layers, batch, hidden, rb=False):
+    return isam.gru_plan(layers, batch, hidden, rb, num_sms=SMS, smem_optin=SMEM)
+
+
+@pytest.mark.parametrize("layers", [1, 2, 3])
+def test_gru_every_supported_shape_has_a_plan_that_fits(layers, monkeypatch):
+    monkeypatch.delenv("ISAM_NO_WAVE", raising=False)
+    for H in HIDDEN:
+        for batch in BATCH:
+            for rb in (False, True):
+                p = gru_plan(layers, batch, H, rb)
+                ks, ka = p["splits"], p["atoms"]
+                atoms = math.ceil(H / 64)
+                assert ks in (1, 2, 4) and ka == math.ceil(atoms / ks), (H, p)
+                # K ranges of whole atoms cover the hidden size, and the last
+                # CTA of a cluster still holds part of it.
+                assert (ks - 1) * ka * 64 < H <= ks * ka * 64, (H, p)
+                assert p["ctas"] == H // 32 * ks <= SMS
+                assert 0 < p["smem"] <= SMEM, (H, batch, layers, rb, p)
+                bp = p["batch_pad"]
+                if batch <= 32:
+                    assert bp == 32
+                else:
+                    assert bp in (64, 128) and (bp == 64 or ks == 4)
+                assert p["chunks"] == math.ceil(batch / bp)
+                if layers == 1:
+                    assert p["path"] == 0
+                elif batch > 32:
+                    assert p["path"] == 3
+                elif not rb and H % 256 == 0:
+                    assert p["path"] == 1
+                else:
+                    assert p["path"] == 2
+
+
+def test_gru_benchmark_plans():
+    """Hidden 1024, batch 32: 32 clusters of 4 CTAs (128), 4 K atoms of U
+    each; two stacked layers run as one kernel, the reset-before form as the
+    per-layer chain."""
+    assert gru_plan(1, 32, 1024) == {"splits": 4, "atoms": 4, "batch_pad": 32, "ctas": 128,
+                                     "smem": gru_plan(1, 32, 1024)["smem"], "path": 0, "chunks": 1}
+    assert gru_plan(2, 32, 1024)["path"] == 1
+    assert gru_plan(2, 32, 1024, rb=True)["path"] == 2
+    assert gru_plan(1, 200, 1024)["batch_pad"] == 128 and gru_plan(1, 200, 1024)["chunks"] == 2
+    assert gru_plan(1, 64, 1024)["batch_pad"] == 64
+
+
+def test_gru_uneven_k_ranges():
+    """Hidden sizes whose atoms do not divide evenly among the splits."""
+    assert (gru_plan(1, 8, 960)["splits"], gru_plan(1, 8, 960)["atoms"]) == (4, 4)   # 15 atoms
+    assert (gru_plan(1, 8, 864)["splits"], gru_plan(1, 8, 864)["atoms"]) == (2, 7)   # 13.5 atoms
+    assert (gru_plan(1, 8, 448)["splits"], gru_plan(1, 8, 448)["atoms"]) == (1, 7)
+    assert (gru_plan(1, 8, 480)["splits"], gru_plan(1, 8, 480)["atoms"]) == (2, 4)
+
+
+def test_gru_no_wave_switch_selects_the_chain(monkeypatch):
+    monkeypatch.setenv("ISAM_NO_WAVE", "1")
+    assert gru_plan(2, 32, 1024)["path"] == 2
+
+
+def test_gru_rejects_shapes_outside_the_limits():
+    for (layers, batch, H) in [(1, 257, 64), (1, 1, 80), (1, 1, 1056), (1, 1, 16), (2, 300, 256)]:
+        with pytest.raises(isam.IsamError) as e:
+            gru_plan(layers, batch, H)
+        assert e.value.code == isam.ISAM_ERR_UNSUPPORTED
+    # Too few SMs for the co-resident recurrence of hidden 1024 (128 CTAs).
+    with pytest.raises(isam.IsamError) as e:
+        isam.gru_plan(1, 32, 1024, num_sms=100, smem_optin=SMEM)
+    assert e.value.code == isam.ISAM_ERR_UNSUPPORTED
+    lib = isam.load()
+    import ctypes
+    out = (ctypes.c_int * 7)()
+    assert lib.isam_gru_plan_for(0, 1, 64, 0, SMS, SMEM, out) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gru_plan_for(1, 1, 64, 2, SMS, SMEM, out) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gru_plan_for(1, 1, 64, 0, SMS, SMEM, None) == isam.ISAM_ERR_INVALID_ARG
+
+
+WIDTHS = [1, 2, 3, 7, 8, 13, 28, 56, 64, 100, 112, 128, 129, 200]
+
+
+def test_dwsep_every_supported_shape_has_a_plan():
+    for W in WIDTHS:
+        for cin in range(16, 257, 16):
+            for cout in range(16, 257, 16):
+                p = isam.dwsep_plan(W, cin, cout, smem_optin=SMEM)
+                pc, blocks = p["block_cout"], p["blocks"]
+                assert pc % 16 == 0 and 16 <= pc <= cout, (W, cin, cout, p)
+                assert blocks == math.ceil(cout / pc) and (blocks - 1) * pc < cout
+                if p["kernel"] == 0:
+                    rt = p["rows_per_tile"]
+                    assert W <= 128 and rt >= 1 and rt * W <= 128, (W, cin, cout, p)
+                else:
+                    assert p["kernel"] == 1 and p["rows_per_tile"] == 0
+
+
+def test_dwsep_benchmark_and_wide_layer_plans():
+    assert isam.dwsep_plan(56, 128, 256, smem_optin=SMEM) == {"kernel": 0, "rows_per_tile": 2, "blocks": 1,
+                                                              "block_cout": 256}
+    assert isam.dwsep_plan(56, 256, 256, smem_optin=SMEM) == {"kernel": 1, "rows_per_tile": 0, "blocks": 4,
+                                                              "block_cout": 64}
+    # More shared memory, fewer blocks: the planner follows the limit it is given.
+    assert isam.dwsep_plan(56, 256, 256, smem_optin=400 * 1024)["blocks"] < 4
+
+
+def test_dwsep_plan_rejects_unsupported_channels():
+    for (cin, cout) in [(24, 16), (16, 272), (272, 16), (8, 16)]:
+        with pytest.raises(isam.IsamError) as e:
+            isam.dwsep_plan(8, cin, cout, smem_optin=SMEM)
+        assert e.value.code == isam.ISAM_ERR_UNSUPPORTED
+    lib = isam.load()
+    import ctypes
+    out = (ctypes.c_int * 4)()
+    assert lib.isam_dwsep_plan_for(0, 16, 16, SMEM, out) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_dwsep_plan_for(8, 16, 16, SMEM, None) == isam.ISAM_ERR_INVALID_ARG
