@@ -160,6 +160,17 @@ int isam_gemm_plan_info(int M, int N, int K, int transA, int transB, float beta,
 int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta, int *out);
 
 /*
+ * isam_gemm_plan_info2's plan for a device with num_sms SMs, smem_optin
+ * bytes of opt-in shared memory per CTA and cluster_caps[3] clusters of 2, 4
+ * and 8 CTAs resident at once (host array); host arithmetic only, no CUDA
+ * call, so it runs without a GPU.  out: 8 ints as isam_gemm_plan_info2.
+ * ISAM_ERR_INVALID_ARG for a null out or cluster_caps or limits < 1, and the
+ * argument checks of isam_gemm.
+ */
+int isam_gemm_plan_for(int M, int N, int K, int transA, int transB, float beta, int num_sms, int smem_optin,
+                       const int *cluster_caps, int *out);
+
+/*
  * GRU forward inference over T steps (input size == hidden).
  *
  * The recurrent model the paper schedules with a priming, a recursive and a

@@ -365,6 +365,35 @@ int isam_gemm_plan_info2(int M, int N, int K, int transA, int transB, float beta
     return ISAM_OK;
 }
 
+int isam_gemm_plan_for(int M, int N, int K, int transA, int transB, float beta, int num_sms, int smem_optin,
+                       const int *cluster_caps, int *out) {
+    if (!out || !cluster_caps || num_sms < 1 || smem_optin < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_plan_for: null output or limits < 1");
+    GemmDesc g{M, N, K, transA, transB, 1.0f, beta, reinterpret_cast<const uint16_t *>(16),
+               reinterpret_cast<const uint16_t *>(16), reinterpret_cast<float *>(16), nullptr};
+    int rc = gemm_validate(g);
+    if (rc) return rc;
+    DeviceState ds;  // no device: the limits come from the arguments
+    ds.num_sms = num_sms;
+    ds.max_smem_optin = smem_optin;
+    for (int i = 0; i < 3; ++i) {
+        if (cluster_caps[i] < 1)
+            return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_plan_for: cluster capacities must be >= 1");
+        ds.cluster_cap[i] = cluster_caps[i];
+    }
+    GemmPlan plan;
+    if ((rc = gemm_plan(g, ds, &plan))) return rc;
+    out[0] = plan.BN;
+    out[1] = plan.split;
+    out[2] = plan.stages;
+    out[3] = plan.group_m;
+    out[4] = plan.grid;
+    out[5] = static_cast<int>(plan.smem);
+    out[6] = plan.pair ? 256 : 128;
+    out[7] = plan.pair ? 2 : 1;
+    return ISAM_OK;
+}
+
 int isam_gru_forward(int T, int batch, int hidden, const isam_bf16 *x, const isam_bf16 *W,
                      const isam_bf16 *U, const float *b, const float *h0, float *h_out) {
     if (T < 1 || batch < 1 || hidden < 1)

@@ -677,6 +677,7 @@ int ensure_smem_attr(KernelFn fn, size_t smem);
 int gemm_cluster_capacity(const DeviceState &ds, int size) {
     if (size <= 1) return ds.num_sms;
     const int idx = size == 2 ? 0 : size == 4 ? 1 : size == 8 ? 2 : -1;
+    if (idx >= 0 && ds.cluster_cap[idx] > 0) return ds.cluster_cap[idx];
     if (idx < 0 || ds.device < 0 || ds.device >= 64) return std::max(1, ds.num_sms / size);
     static std::mutex mu;
     static int cache[64][3] = {};

@@ -20,6 +20,9 @@ struct DeviceState {
     int device = -1;
     int num_sms = 0;
     int max_smem_optin = 0;
+    // Clusters of 2, 4 and 8 CTAs resident at once; 0 = ask the device (a
+    // host-side plan for given limits fills them in).
+    int cluster_cap[3] = {0, 0, 0};
     uint32_t *err_word = nullptr;  // 4 x uint32 on the device
     // GRU workspaces (grown on demand).
     float *gru_gx = nullptr;       // [T*batch][3H] fp32 input projection

@@ -66,6 +66,7 @@ def load():
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
         lib.isam_dwsep_plan_info.argtypes = [i, i, i, P]
         lib.isam_dwsep_plan_for.argtypes = [i, i, i, i, P]
+        lib.isam_gemm_plan_for.argtypes = [i, i, i, i, i, f, i, i, P, P]
         lib.isam_gru_plan_info.argtypes = [i, i, i, i, P]
         lib.isam_gru_plan_for.argtypes = [i, i, i, i, i, i, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
@@ -73,7 +74,7 @@ def load():
                      "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_gru_forward_stack",
                      "isam_dwsep_conv", "isam_dwsep_plan_info", "isam_dwsep_plan_for",
-                     "isam_gru_plan_info", "isam_gru_plan_for"):
+                     "isam_gru_plan_info", "isam_gru_plan_for", "isam_gemm_plan_for"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
         return lib
@@ -201,11 +202,17 @@ def gemm_grouped(problems) -> None:
     GroupedGemm(problems)()
 
 
-def gemm_plan(M, N, K, transA, transB, beta=0.0) -> dict:
-    """The tile plan the library's cost model picks (nothing is launched)."""
+def gemm_plan(M, N, K, transA, transB, beta=0.0, num_sms=None, smem_optin=None, cluster_caps=None) -> dict:
+    """The tile plan the library's cost model picks (nothing is launched);
+    with num_sms, smem_optin and cluster_caps (resident clusters of 2, 4, 8
+    CTAs), isam_gemm_plan_for on those limits (no GPU)."""
     lib = load()
     out = (ctypes.c_int * 8)()
-    check(lib.isam_gemm_plan_info2(M, N, K, int(transA), int(transB), float(beta), out))
+    if num_sms is None:
+        check(lib.isam_gemm_plan_info2(M, N, K, int(transA), int(transB), float(beta), out))
+    else:
+        caps = (ctypes.c_int * 3)(*cluster_caps)
+        check(lib.isam_gemm_plan_for(M, N, K, int(transA), int(transB), float(beta), num_sms, smem_optin, caps, out))
     return dict(zip(("BN", "split", "stages", "group_m", "grid", "smem", "tile_m", "cta_pair"), list(out)))
 
 

@@ -1,10 +1,12 @@
-"""The GRU and depthwise-separable planners, run on the host through the C ABI
-(isam_gru_plan_for, isam_dwsep_plan_for: host arithmetic, no CUDA call) with
-a GB300's limits: 152 SMs, 232448 bytes of opt-in shared memory per CTA.
-Every shape inside the boundary's support limits (GRU: batch <= 256, hidden
-any multiple of 32 up to 1024; dwsep: Cin and Cout multiples of 16 up to 256,
-any width) must get a plan that fits the device, and the plans must keep the
-invariants the kernels rely on."""
+"""The GEMM, GRU and depthwise-separable planners, run on the host through
+the C ABI (isam_gemm_plan_for, isam_gru_plan_for, isam_dwsep_plan_for: host
+arithmetic, no CUDA call) with a GB300's limits: 152 SMs, 232448 bytes of
+opt-in shared memory per CTA.  Every shape inside the boundary's support
+limits (GRU: batch <= 256, hidden any multiple of 32 up to 1024; dwsep: Cin
+and Cout multiples of 16 up to 256, any width; GEMM: the benchmark shapes and
+a grid of small, ragged and large ones in all four layouts) must get a plan
+that fits the device, and the plans must keep the invariants the kernels rely
+on."""
 import math
 
 import pytest
@@ -137,3 +139,66 @@ def test_dwsep_plan_rejects_unsupported_channels():
     out = (ctypes.c_int * 4)()
     assert lib.isam_dwsep_plan_for(0, 16, 16, SMEM, out) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_dwsep_plan_for(8, 16, 16, SMEM, None) == isam.ISAM_ERR_INVALID_ARG
+
+
+# ---- the GEMM planner (isam_gemm_plan_for): cluster capacities of 2, 4 and 8
+# CTAs as if every SM could hold one CTA of any cluster (the device query can
+# only lower them, which the invariants below do not depend on).
+CAPS = [SMS // 2, SMS // 4, SMS // 8]
+
+
+def gemm_plan(M, N, K, tA, tB, beta=0.0, caps=CAPS):
+    return isam.gemm_plan(M, N, K, tA, tB, beta, num_sms=SMS, smem_optin=SMEM, cluster_caps=caps)
+
+
+def check_gemm_plan(M, N, K, tA, tB, p):
+    assert p["BN"] in (16, 32, 64, 128, 256), p
+    assert p["split"] in (1, 2, 4, 8) and p["cta_pair"] in (1, 2), p
+    assert 0 < p["smem"] <= SMEM and 1 <= p["grid"] <= SMS, p
+    # Clusters (split-K groups or CTA pairs) fill the grid whole.
+    assert p["grid"] % (p["split"] * p["cta_pair"]) == 0, p
+    if p["cta_pair"] == 2:
+        assert p["tile_m"] == 256 and p["split"] == 1 and tA == 0 and N % 4 == 0 and K >= 256, p
+    else:
+        assert p["tile_m"] == 128
+    # A split never leaves a CTA without K atoms.
+    assert p["split"] <= max(1, math.ceil(K / 64)), p
+
+
+def test_gemm_plans_of_the_benchmark_shapes():
+    for (M, K) in [(1760, 1760), (2560, 2560), (4096, 4096), (7680, 2560)]:
+        for N in (16, 32, 64, 128):
+            for tA in (0, 1):
+                check_gemm_plan(M, N, K, tA, 0, gemm_plan(M, N, K, tA, 0))
+    p = gemm_plan(8192, 8192, 8192, 0, 0, 1.0)
+    check_gemm_plan(8192, 8192, 8192, 0, 0, p)
+    assert (p["tile_m"], p["cta_pair"], p["BN"], p["split"]) == (256, 2, 256, 1)
+    check_gemm_plan(512, 512, 512, 0, 0, gemm_plan(512, 512, 512, 0, 0))
+
+
+def test_gemm_plans_over_a_grid_of_shapes():
+    sizes = [8, 16, 24, 120, 128, 136, 1000, 2048, 4104]
+    for M in sizes:
+        for N in sizes:
+            for K in sizes:
+                for tA in (0, 1):
+                    for tB in (0, 1):
+                        check_gemm_plan(M, N, K, tA, tB, gemm_plan(M, N, K, tA, tB))
+
+
+def test_gemm_plans_with_few_resident_clusters():
+    for (M, N, K) in [(4096, 16, 4096), (8192, 8192, 8192), (512, 512, 512)]:
+        check_gemm_plan(M, N, K, 0, 0, gemm_plan(M, N, K, 0, 0, caps=[1, 1, 1]))
+
+
+def test_gemm_plan_for_rejects_bad_arguments():
+    import ctypes
+    lib = isam.load()
+    out = (ctypes.c_int * 8)()
+    caps = (ctypes.c_int * 3)(*CAPS)
+    assert lib.isam_gemm_plan_for(0, 16, 16, 0, 0, 0.0, SMS, SMEM, caps, out) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_gemm_plan_for(16, 16, 16, 0, 0, 0.0, SMS, SMEM, None, out) == isam.ISAM_ERR_INVALID_ARG
+    zero = (ctypes.c_int * 3)(0, 1, 1)
+    assert lib.isam_gemm_plan_for(16, 16, 16, 0, 0, 0.0, SMS, SMEM, zero, out) == isam.ISAM_ERR_INVALID_ARG
+    # K = 12: a K-major A row is not 16-byte aligned.
+    assert lib.isam_gemm_plan_for(16, 16, 12, 0, 0, 0.0, SMS, SMEM, caps, out) == isam.ISAM_ERR_UNSUPPORTED
