@@ -58,6 +58,10 @@ def _load():
             lib.oracle_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
             lib.oracle_gru_forward_reset_before.restype = ctypes.c_int
             lib.oracle_gemm_fp8.restype = ctypes.c_int
+            lib.oracle_e8m0.argtypes = [ctypes.c_uint8]
+            lib.oracle_e8m0.restype = ctypes.c_double
+            lib.oracle_gemm_mxfp8.argtypes = [i, i, i, d, P, P, P, P, d, P, P]
+            lib.oracle_gemm_mxfp8.restype = ctypes.c_int
             lib.oracle_gru_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
             lib.oracle_gru_stack.restype = ctypes.c_int
             for f in (lib.oracle_gemm_rows, lib.oracle_gemm, lib.oracle_gru_forward,
@@ -121,6 +125,33 @@ def gemm_fp8(M, N, K, alpha, A, B, beta=0.0, C_in=None):
     rc = _load().oracle_gemm_fp8(M, N, K, float(alpha), _p(A), _p(B), float(beta), _p(C_in), _p(out))
     if rc != 0:
         raise ValueError("oracle_gemm_fp8: invalid argument")
+    return out
+
+
+def e8m0(byte: int) -> float:
+    """The value of one OCP MX E8M0 scale byte: 2^(byte - 127), NaN for 255."""
+    return _load().oracle_e8m0(int(byte) & 0xFF)
+
+
+def gemm_mxfp8(M, N, K, alpha, A, SA, B, SB, beta=0.0, C_in=None):
+    """Block-scaled E4M3 GEMM (OCP MX): C = alpha * (SA . A) @ (SB . B)^T +
+    beta * C_in, A (M x K) and B (N x K) E4M3 bytes, SA (M x ceil(K/32)) and
+    SB (N x ceil(K/32)) E8M0 scale bytes, one per 32 consecutive K elements;
+    returns [M, N] float64."""
+    kb = (K + 31) // 32
+    A = np.ascontiguousarray(A, dtype=np.uint8)
+    B = np.ascontiguousarray(B, dtype=np.uint8)
+    SA = np.ascontiguousarray(SA, dtype=np.uint8)
+    SB = np.ascontiguousarray(SB, dtype=np.uint8)
+    assert A.size == M * K and B.size == N * K and SA.size == M * kb and SB.size == N * kb
+    if C_in is not None:
+        C_in = np.ascontiguousarray(C_in, dtype=np.float32)
+        assert C_in.size == M * N
+    out = np.empty((M, N), dtype=np.float64)
+    rc = _load().oracle_gemm_mxfp8(M, N, K, float(alpha), _p(A), _p(SA), _p(B), _p(SB), float(beta), _p(C_in),
+                                   _p(out))
+    if rc != 0:
+        raise ValueError("oracle_gemm_mxfp8: invalid argument")
     return out
 
 

@@ -134,6 +134,50 @@ int oracle_gemm_fp8(int M, int N, int K, double alpha, const uint8_t *A, const u
     return 0;
 }
 
+/*
+ * OCP Microscaling (MX) shared scale byte, E8M0: the value 2^(e - 127) for e
+ * in 0..254; e == 255 is NaN.  No sign, no mantissa.
+ */
+double oracle_e8m0(uint8_t e) {
+    if (e == 255) return NAN;
+    return ldexp(1.0, (int)e - 127);
+}
+
+/*
+ * Block-scaled E4M3 GEMM (OCP MX, MXFP8): each run of 32 consecutive K
+ * elements of a row of A, and of a row of B (stored N x K), shares one E8M0
+ * scale, so element k of row i of A stands for SA[i][k / 32] * A[i][k]:
+ *
+ *   C_out[i][j] = alpha * sum_k (SA[i][k/32] A[i][k]) (SB[j][k/32] B[j][k])
+ *                 + beta * C_in[i][j]
+ *
+ * SA is M x ceil(K / 32) and SB N x ceil(K / 32) scale bytes, row-major; a
+ * last block shorter than 32 (K not a multiple of 32) has a scale of its
+ * own.  Each dot product is summed in increasing k in double precision (every
+ * product is exact there: a power-of-two scale times an E4M3 value).
+ */
+int oracle_gemm_mxfp8(int M, int N, int K, double alpha, const uint8_t *A, const uint8_t *SA,
+                      const uint8_t *B, const uint8_t *SB, double beta, const float *C_in, double *C_out) {
+    if (M < 1 || N < 1 || K < 1 || !A || !SA || !B || !SB || !C_out) return 1;
+    if (beta != 0.0 && !C_in) return 1;
+    const int KB = (K + 31) / 32;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int i = 0; i < M; ++i) {
+        for (int j = 0; j < N; ++j) {
+            double acc = 0.0;
+            for (int k = 0; k < K; ++k) {
+                const double a = oracle_e8m0(SA[(size_t)i * KB + k / 32]) * oracle_e4m3(A[(size_t)i * K + k]);
+                const double bv = oracle_e8m0(SB[(size_t)j * KB + k / 32]) * oracle_e4m3(B[(size_t)j * K + k]);
+                acc += a * bv;
+            }
+            double v = alpha * acc;
+            if (beta != 0.0) v += beta * (double)C_in[(size_t)i * N + j];
+            C_out[(size_t)i * N + j] = v;
+        }
+    }
+    return 0;
+}
+
 int oracle_gemm(int M, int N, int K, int transA, int transB, double alpha,
                 const uint16_t *A, const uint16_t *B, double beta,
                 const float *C_in, double *C_out) {

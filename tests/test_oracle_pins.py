@@ -384,6 +384,75 @@ def test_e4m3_rounding_of_inputs(oracle_lib):
     assert np.array_equal(synth.to_e4m3_bits(vals), codes)
 
 
+# --------------------------------------------------------------------------- MX block-scaled E4M3 GEMM
+
+def test_e8m0_decode_known_values(oracle_lib):
+    """Values fixed by the OCP MX E8M0 scale format: 2^(e - 127), 255 is NaN."""
+    known = {127: 1.0, 128: 2.0, 126: 0.5, 0: 2.0 ** -127, 254: 2.0 ** 127, 137: 1024.0}
+    for byte, v in known.items():
+        assert oracle_lib.e8m0(byte) == v, byte
+    assert math.isnan(oracle_lib.e8m0(255))
+
+
+def _scales(seed, rows, kb, lo, hi):
+    return synth.integers(seed, rows * kb, lo, hi).astype(np.uint8).reshape(rows, kb)
+
+
+def test_mxfp8_unit_scales_are_the_e4m3_gemm(oracle_lib):
+    """Every scale 2^0 (byte 127): exactly the unscaled E4M3 GEMM, with a
+    ragged last block (K = 80: blocks of 32, 32, 16)."""
+    M, N, K = 11, 6, 80
+    A = synth.e4m3_uniform(41, (M, K))
+    B = synth.e4m3_uniform(42, (N, K))
+    C0 = synth.f32_uniform(43, (M, N))
+    ones_a = np.full((M, 3), 127, np.uint8)
+    ones_b = np.full((N, 3), 127, np.uint8)
+    got = oracle_lib.gemm_mxfp8(M, N, K, 1.5, A, ones_a, B, ones_b, -0.5, C0)
+    assert np.array_equal(got, oracle_lib.gemm_fp8(M, N, K, 1.5, A, B, -0.5, C0))
+
+
+def test_mxfp8_is_the_sum_of_scaled_block_products(oracle_lib):
+    """With integer E4M3 data and power-of-two scales every term is exact, so
+    the block-scaled GEMM equals the sum over K blocks of
+    diag(2^(SA-127)) (A_blk B_blk^T) diag(2^(SB-127)), each block product
+    taken by the (separately pinned) unscaled E4M3 GEMM."""
+    M, N, K = 9, 7, 112  # blocks of 32, 32, 32, 16
+    kb = (K + 31) // 32
+    A = synth.e4m3_integers(51, (M, K), -6, 6)
+    B = synth.e4m3_integers(52, (N, K), -6, 6)
+    SA = _scales(53, M, kb, 120, 134)
+    SB = _scales(54, N, kb, 121, 133)
+    got = oracle_lib.gemm_mxfp8(M, N, K, 1.0, A, SA, B, SB)
+    want = np.zeros((M, N))
+    for blk in range(kb):
+        k0, k1 = 32 * blk, min(K, 32 * blk + 32)
+        part = oracle_lib.gemm_fp8(M, N, k1 - k0, 1.0, np.ascontiguousarray(A[:, k0:k1]),
+                                   np.ascontiguousarray(B[:, k0:k1]))
+        sa = np.ldexp(1.0, SA[:, blk].astype(int) - 127)
+        sb = np.ldexp(1.0, SB[:, blk].astype(int) - 127)
+        want += sa[:, None] * part * sb[None, :]
+    assert np.array_equal(got, want)
+    # A scale one step up doubles exactly that block's share of its row.
+    SA2 = SA.copy()
+    SA2[4, 1] += 1
+    got2 = oracle_lib.gemm_mxfp8(M, N, K, 1.0, A, SA2, B, SB)
+    part1 = oracle_lib.gemm_fp8(M, N, 32, 1.0, np.ascontiguousarray(A[:, 32:64]), np.ascontiguousarray(B[:, 32:64]))
+    delta = np.ldexp(1.0, int(SA[4, 1]) - 127) * part1[4] * np.ldexp(1.0, SB[:, 1].astype(int) - 127)
+    assert np.array_equal(got2[4] - got[4], delta)
+    assert np.array_equal(np.delete(got2, 4, axis=0), np.delete(got, 4, axis=0))
+
+
+def test_mxfp8_nan_scale_poisons_only_its_row(oracle_lib):
+    M, N, K = 5, 4, 64
+    A = synth.e4m3_integers(61, (M, K), -3, 3)
+    B = synth.e4m3_integers(62, (N, K), -3, 3)
+    SA = np.full((M, 2), 127, np.uint8)
+    SB = np.full((N, 2), 127, np.uint8)
+    SA[2, 0] = 255
+    got = oracle_lib.gemm_mxfp8(M, N, K, 1.0, A, SA, B, SB)
+    assert np.isnan(got[2]).all() and np.isfinite(np.delete(got, 2, axis=0)).all()
+
+
 # --------------------------------------------------------------------------- GRU, reset before the product
 
 def _gru_rb_python(x, W, U, b, h0):
