@@ -49,9 +49,10 @@ METRIC = "GEMM TFLOP/s (tall-skinny sweep) and GRU timesteps/s on 1 GB300; % of 
 WORKLOAD = ("tall-skinny GEMM sweep: (M,K) in {(1760,1760),(2560,2560),(4096,4096),(7680,2560)} "
             "x N in {16,32,64,128} x {NN,TN}; bf16 U[-1,1]; fp32 accumulate/output; beta=0")
 # dram__bytes_read.sum + dram__bytes_write.sum of one gemm_group_kernel launch
-# over the sweep, from the ncu capture summarised in
-# profiles/gemm_group_kernel_skinny_sweep.md (None until taken for the current kernel).
-TRAFFIC_PER_STEP = 749125376 + 26610176
+# over the sweep, from an ncu capture of the current kernel; None until one is
+# taken (profiles/gemm_group_kernel_skinny_sweep.md holds 749125376 + 26610176
+# bytes, captured before the kernel gained its per-problem E4M3 path).
+TRAFFIC_PER_STEP = None
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
