@@ -295,7 +295,7 @@ int isam_gemm_grouped(int count, const int *M, const int *N, const int *K, const
         g[i] = GemmDesc{M[i], N[i], K[i], transA[i], transB[i], alpha[i], beta[i], A[i], B[i], C[i], nullptr};
         int rc = gemm_validate(g[i]);
         if (rc) {
-            char msg[512];
+            char msg[640];  // prefix + the 512-byte error text
             snprintf(msg, sizeof msg, "isam_gemm_grouped: problem %d: %s", i, isam_last_error_string());
             return set_error(rc, "%s", msg);
         }
@@ -318,7 +318,7 @@ int isam_gemm_grouped_fp8(int count, const int *M, const int *N, const int *K, c
                         reinterpret_cast<const uint16_t *>(B[i]), C[i], nullptr, 1};
         int rc = gemm_validate(g[i]);
         if (rc) {
-            char msg[512];
+            char msg[640];  // prefix + the 512-byte error text
             snprintf(msg, sizeof msg, "isam_gemm_grouped_fp8: problem %d: %s", i, isam_last_error_string());
             return set_error(rc, "%s", msg);
         }
