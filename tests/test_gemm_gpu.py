@@ -102,6 +102,17 @@ def test_gemm_small_and_ragged(shape, tA):
     assert nmax_err(got, ref) <= TOL
 
 
+@pytest.mark.parametrize("tA", [0, 1], ids=["NT", "TT"])
+def test_gemm_odd_n_c_rows_not_16_byte_aligned(tA):
+    """N = 13 and 77 with K-major B (transB = 1): a row of C is not 16-byte
+    aligned, so C moves by plain stores; integer inputs must match exactly."""
+    for (M, N, K) in [(200, 13, 136), (136, 77, 520)]:
+        A, B, C0 = synth.gemm_operands(M, N, K, tA, 1, seed=M + N + K + tA, dist="int4", beta_c=True)
+        got = run_gemm(M, N, K, tA, 1, 2.0, -1.0, A, B, C0=C0)
+        ref = oracle.gemm(M, N, K, tA, 1, 2.0, A, B, -1.0, C0)
+        assert np.array_equal(got.astype(np.float64), ref), (M, N, K)
+
+
 def test_gemm_beta_zero_does_not_read_c():
     M, N, K = 384, 128, 256
     A, B, _ = synth.gemm_operands(M, N, K, 0, 0, seed=5)
