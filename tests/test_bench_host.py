@@ -1,6 +1,7 @@
 """Host logic of bench.py that needs no GPU: the sweep definition, whole-job
 aggregation, the max-over-ranks reduction on two gloo ranks, the reference
-arm's rank handling, and the oracle's row sample of the sweep operands."""
+arm's rank handling and its JSON line, and the oracle's row sample of the
+sweep operands."""
 import json
 import os
 import socket
@@ -81,6 +82,29 @@ def test_reference_arm_other_ranks_exit_silently():
                        timeout=120)
     assert r.returncode == 0
     assert r.stdout.strip() == ""
+
+
+def test_reference_arm_prints_the_contract_line():
+    """Rank 0 of the reference arm (the fp64 oracle on the host cores) prints
+    one JSON line with the contract's keys; its end-to-end figure is its own
+    value with no host-device copies."""
+    env = {k: v for k, v in os.environ.items() if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK")}
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--steps", "1", "--warmup", "3"], env=env, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config"):
+        assert key in d, key
+    assert d["impl"] == "reference" and d["warmup"] >= 3 and d["steps"] == 1
+    assert d["value"] > 0 and d["unit"] == "TFLOP/s" and d["higher_is_better"] is True
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert "workload" in d["config"]
 
 
 def test_oracle_row_sample_draws_the_same_rows():
