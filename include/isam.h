@@ -23,6 +23,10 @@
  *     after the launch.  Argument errors are reported at once and nothing is
  *     launched.  Device-side failures (a bounded wait that ran out) are
  *     reported by the next isam_sync().
+ *   - One device per process: each kernel opts in to its dynamic shared
+ *     memory once, in the context of the first device that launches it, and
+ *     the attribute belongs to that device's context.  A process that drives
+ *     several GPUs through this library is not supported yet.
  *   - Every spin-wait inside the kernels is bounded in time (default 2 s,
  *     ISAM_WAIT_TIMEOUT_MS in the environment overrides); a wait that runs out
  *     sets the device error word and the kernel returns.
