@@ -72,3 +72,25 @@ def test_grouped_rejects_bad_count_without_cuda(lib):
     assert lib.isam_gemm_grouped(0, p, p, p, p, p, p, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_gemm_grouped(65, p, p, p, p, p, p, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_gemm_grouped(2, None, p, p, p, p, p, p, p, p, p) == isam.ISAM_ERR_INVALID_ARG
+
+
+def test_product_path_never_references_the_oracle():
+    """The library and its binding are independent of the oracle: no source
+    under the package, its CUDA directory or the public header imports, loads
+    or names it (synth.py, the input generators both sides share, only says
+    so in its docstring)."""
+    import os
+    import re
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    pkg = os.path.join(root, "paper_1810_09958_gb300")
+    files = [os.path.join(pkg, f) for f in os.listdir(pkg) if f.endswith(".py") and f != "synth.py"]
+    csrc = os.path.join(pkg, "csrc")
+    files += [os.path.join(csrc, f) for f in os.listdir(csrc) if f.endswith((".cu", ".cuh", ".h", ".cpp"))]
+    files += [os.path.join(root, "include", f) for f in os.listdir(os.path.join(root, "include"))]
+    pattern = re.compile(r"oracle", re.IGNORECASE)
+    for path in files:
+        with open(path) as f:
+            assert not pattern.search(f.read()), path
+    with open(os.path.join(pkg, "synth.py")) as f:
+        src = f.read()
+    assert not re.search(r"^\s*(import|from)\s+oracle", src, re.MULTILINE)
