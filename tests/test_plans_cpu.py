@@ -202,3 +202,31 @@ def test_gemm_plan_for_rejects_bad_arguments():
     assert lib.isam_gemm_plan_for(16, 16, 16, 0, 0, 0.0, SMS, SMEM, zero, out) == isam.ISAM_ERR_INVALID_ARG
     # K = 12: a K-major A row is not 16-byte aligned.
     assert lib.isam_gemm_plan_for(16, 16, 12, 0, 0, 0.0, SMS, SMEM, caps, out) == isam.ISAM_ERR_UNSUPPORTED
+
+
+def test_gemm_argument_rules_on_the_host():
+    """The boundary's GEMM support limits, checked before any CUDA call: sizes
+    >= 1, flags 0 or 1, and 16-byte rows of the stored operands (the row pitch
+    of A is K when A is M x K, M when it is K x M; of B, N when B is K x N, K
+    when it is N x K)."""
+    import ctypes
+    lib = isam.load()
+    out = (ctypes.c_int * 8)()
+    caps = (ctypes.c_int * 3)(*CAPS)
+    cases = [
+        ((16, 16, 16, 0, 0), isam.ISAM_OK),
+        ((16, 16, 16, 1, 1), isam.ISAM_OK),
+        ((13, 16, 16, 0, 0), isam.ISAM_OK),                 # M free when A is M x K
+        ((13, 16, 16, 1, 0), isam.ISAM_ERR_UNSUPPORTED),    # A stored K x 13: 26-byte rows
+        ((16, 13, 16, 0, 1), isam.ISAM_OK),                 # N free when B is N x K
+        ((16, 13, 16, 0, 0), isam.ISAM_ERR_UNSUPPORTED),    # B stored K x 13
+        ((16, 16, 12, 0, 1), isam.ISAM_ERR_UNSUPPORTED),    # K-major rows of 24 bytes
+        ((16, 16, 12, 1, 0), isam.ISAM_OK),                 # K is only a row count here
+        ((1, 1, 8, 0, 1), isam.ISAM_OK),
+        ((0, 16, 16, 0, 0), isam.ISAM_ERR_INVALID_ARG),
+        ((16, 16, 16, 2, 0), isam.ISAM_ERR_INVALID_ARG),
+        ((16, 16, 16, 0, -1), isam.ISAM_ERR_INVALID_ARG),
+    ]
+    for (M, N, K, tA, tB), want in cases:
+        got = lib.isam_gemm_plan_for(M, N, K, tA, tB, 0.0, SMS, SMEM, caps, out)
+        assert got == want, ((M, N, K, tA, tB), got, isam.last_error())
