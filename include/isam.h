@@ -23,10 +23,11 @@
  *     after the launch.  Argument errors are reported at once and nothing is
  *     launched.  Device-side failures (a bounded wait that ran out) are
  *     reported by the next isam_sync().
- *   - One device per process: each kernel opts in to its dynamic shared
- *     memory once, in the context of the first device that launches it, and
- *     the attribute belongs to that device's context.  A process that drives
- *     several GPUs through this library is not supported yet.
+ *   - Calls run on the caller's current device.  Workspaces, the error word
+ *     and each kernel's dynamic shared-memory opt-in are kept per device (the
+ *     opt-in belongs to each device's context), so one process may drive
+ *     several GPUs; the stream given to isam_set_stream() must belong to the
+ *     device that is current at each call.
  *   - Every spin-wait inside the kernels is bounded in time (default 2 s,
  *     ISAM_WAIT_TIMEOUT_MS in the environment overrides); a wait that runs out
  *     sets the device error word and the kernel returns.
@@ -203,8 +204,8 @@ int isam_gemm_plan_for(int M, int N, int K, int transA, int transB, float beta, 
  * Batches above 32 run with the batch padded to 64 or 128 rows (the MMA's N;
  * 128 only with 4 K splits), in chunks of that many rows, one launch per
  * chunk; the rows are independent sequences.  The recurrence runs on
- * hidden / 32 clusters of K-split CTAs, launched cooperatively so they are
- * co-resident: 4 splits when hidden is a multiple of 256, 2 for the other
+ * hidden / 32 clusters of K-split CTAs, launched only after the device
+ * reports that every cluster fits at once (they must all be resident): 4 splits when hidden is a multiple of 256, 2 for the other
  * multiples of 128, otherwise 1 up to hidden 448, 2 up to 896 and 4 above.
  * Each CTA keeps a 96-row slice of U over ceil(atoms / splits) 64-wide K
  * atoms in shared memory; where the last CTA's range ends past the matrix (a
@@ -292,13 +293,15 @@ int isam_gru_forward_stack(int layers, int T, int batch, int hidden, int reset_b
  * allocating routine is called.
  *
  *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture.
+ *     (cudaGetSymbolAddress) with that device current.
  *   - Every call shares the one array: calls that overlap on the GPU (other
  *     streams, other host threads) race and corrupt each other.  The call
  *     clears the parts that must start at zero (error word, step counter).
- *   - Unlike the other calls it waits for its own work on the stream before
- *     returning, so that it can report a device-side timeout itself:
+ *   - Unlike the other calls it synchronises its stream before returning
+ *     (it reads the device error word back on that stream, then waits for
+ *     that stream alone), so that it can report a device-side timeout
+ *     itself; it must therefore not be called while the stream is being
+ *     captured into a CUDA graph.  Results:
  *     ISAM_OK, ISAM_ERR_TIMEOUT (h_out undefined), ISAM_ERR_CUDA,
  *     ISAM_ERR_INVALID_ARG or ISAM_ERR_UNSUPPORTED (sizes beyond the limits
  *     above, misaligned pointers, a device other than sm_103a).

@@ -105,6 +105,34 @@ unsigned long long wait_timeout_ns() {
     return v;
 }
 
+namespace {
+struct SmemOptin {
+    int device;
+    const void *fn;
+    int bytes;
+};
+constexpr int kOptinCap = 256;
+SmemOptin g_optin[kOptinCap];
+int g_optin_n = 0;
+std::mutex g_optin_mu;
+}  // namespace
+
+int ensure_smem_optin(const void *fn, int bytes, int device, const char *what) {
+    std::lock_guard<std::mutex> lk(g_optin_mu);
+    int slot = -1;
+    for (int i = 0; i < g_optin_n; ++i)
+        if (g_optin[i].device == device && g_optin[i].fn == fn) {
+            if (g_optin[i].bytes >= bytes) return ISAM_OK;
+            slot = i;
+            break;
+        }
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e != cudaSuccess) return cuda_error(e, what);
+    if (slot < 0 && g_optin_n < kOptinCap) slot = g_optin_n++;
+    if (slot >= 0) g_optin[slot] = SmemOptin{device, fn, bytes};
+    return ISAM_OK;
+}
+
 DeviceState *device_state(int *status) {
     int dev = -1;
     cudaError_t e = cudaGetDevice(&dev);

@@ -944,13 +944,9 @@ int dwsep_block(int N, int H, int W, int Cin, int Cout, int c0, int pc, const ui
         q.ldo = Cout;
         q.timeout_ns = wait_timeout_ns();
         q.err = ds.err_word;
-        static bool rattr = false;
-        if (!rattr) {
-            cudaError_t e = cudaFuncSetAttribute(dwsep_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 ds.max_smem_optin);
-            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(dwsep rows)");
-            rattr = true;
-        }
+        if ((rc = ensure_smem_optin(reinterpret_cast<const void *>(dwsep_rows_kernel), ds.max_smem_optin, ds.device,
+                                    "cudaFuncSetAttribute(dwsep rows)")))
+            return rc;
         const int grid = q.tiles < ds.num_sms ? q.tiles : ds.num_sms;
         dwsep_rows_kernel<<<grid, kRThreads, RL.total, stream>>>(tmW, tmOut, tmOut16, tmOut8, q);
         cudaError_t e = cudaGetLastError();
@@ -984,14 +980,9 @@ int dwsep_block(int N, int H, int W, int Cin, int Cout, int c0, int pc, const ui
     p.dw = dw;
     p.timeout_ns = wait_timeout_ns();
     p.err = ds.err_word;
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(dwsep_fused_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             ds.max_smem_optin);
-        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(dwsep)");
-        attr_set = true;
-    }
+    if ((rc = ensure_smem_optin(reinterpret_cast<const void *>(dwsep_fused_kernel), ds.max_smem_optin, ds.device,
+                                "cudaFuncSetAttribute(dwsep)")))
+        return rc;
     const int grid = p.tiles < ds.num_sms ? p.tiles : ds.num_sms;
     dwsep_fused_kernel<<<grid, kThreads, L.total, stream>>>(tmW, tmOut, p);
     cudaError_t e = cudaGetLastError();

@@ -667,7 +667,6 @@ double estimate_us(const GemmDesc &g, int BN, int S, int num_sms, int cluster_ca
     return kFirstDataUs + std::max({t_steady, t_hbm, t_flops}) + tail + kLaunchGapUs;
 }
 
-int ensure_smem_attr(KernelFn fn, size_t smem);
 
 }  // namespace
 
@@ -686,7 +685,7 @@ int gemm_cluster_capacity(const DeviceState &ds, int size) {
     if (c > 0) return c;
     int n = 0;
     KernelFn fn = pick_kernel(128, false, false);
-    if (ensure_smem_attr(fn, static_cast<size_t>(ds.max_smem_optin)) == ISAM_OK) {
+    if (ensure_smem_optin(reinterpret_cast<const void *>(fn), ds.max_smem_optin, ds.device, "cudaFuncSetAttribute(gemm)") == ISAM_OK) {
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -708,39 +707,6 @@ int gemm_cluster_capacity(const DeviceState &ds, int size) {
     c = n > 0 ? std::min(n, ds.num_sms / size) : std::max(1, ds.num_sms / size);
     return c;
 }
-
-namespace {
-
-struct AttrCache {
-    std::mutex mu;
-    KernelFn fn[64] = {};
-    int smem[64] = {};
-    int n = 0;
-} g_attr;
-
-int ensure_smem_attr(KernelFn fn, size_t smem) {
-    std::lock_guard<std::mutex> lk(g_attr.mu);
-    for (int i = 0; i < g_attr.n; ++i)
-        if (g_attr.fn[i] == fn) {
-            if (g_attr.smem[i] >= static_cast<int>(smem)) return ISAM_OK;
-            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 static_cast<int>(smem));
-            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
-            g_attr.smem[i] = static_cast<int>(smem);
-            return ISAM_OK;
-        }
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm)");
-    if (g_attr.n < 64) {
-        g_attr.fn[g_attr.n] = fn;
-        g_attr.smem[g_attr.n] = static_cast<int>(smem);
-        ++g_attr.n;
-    }
-    return ISAM_OK;
-}
-
-}  // namespace
 
 int gemm_validate(const GemmDesc &g) {
     if (g.M < 1 || g.N < 1 || g.K < 1)
@@ -876,7 +842,9 @@ int gemm_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, cudaSt
 
     KernelFn fn = g.fp8 ? pick_kernel_f8(plan.BN) : pick_kernel(plan.BN, a_mn, b_mn);
     if (!fn) return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm: no kernel for BN=%d", plan.BN);
-    if ((rc = ensure_smem_attr(fn, plan.smem))) return rc;
+    if ((rc = ensure_smem_optin(reinterpret_cast<const void *>(fn), static_cast<int>(plan.smem), ds.device,
+                                "cudaFuncSetAttribute(gemm)")))
+        return rc;
 
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];

@@ -368,7 +368,6 @@ size_t group_smem_bytes(int stages) {
 }
 
 std::mutex g_group_mu;
-bool g_group_attr = false;
 
 }  // namespace
 
@@ -437,12 +436,9 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
     p.timeout_ns = wait_timeout_ns();
     p.err = ds.err_word;
     const size_t smem = group_smem_bytes(st);
-    if (!g_group_attr) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             ds.max_smem_optin);
-        if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(grouped gemm)");
-        g_group_attr = true;
-    }
+    if (const int rc = ensure_smem_optin(reinterpret_cast<const void *>(gemm_group_kernel), ds.max_smem_optin,
+                                         ds.device, "cudaFuncSetAttribute(grouped gemm)"))
+        return rc;
     const int grid = std::min(tiles, ds.num_sms);
     gemm_group_kernel<<<grid, kThreads, smem, stream>>>(p);
     cudaError_t e = cudaGetLastError();

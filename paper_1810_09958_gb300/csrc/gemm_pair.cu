@@ -367,8 +367,6 @@ size_t pair_smem_bytes(int stages) {
     return 1024 + static_cast<size_t>(stages) * (kAStage + kBStage) + kEpiBytes + (2 * stages + 15) * 8 + 16;
 }
 
-std::mutex g_pair_mu;
-bool g_pair_attr[2] = {false, false};
 
 }  // namespace
 
@@ -424,12 +422,9 @@ int gemm_pair_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, c
 
     const PairKernel fn = b_mn ? gemm_pair_kernel<true> : gemm_pair_kernel<false>;
     {
-        std::lock_guard<std::mutex> lk(g_pair_mu);
-        if (!g_pair_attr[b_mn ? 1 : 0]) {
-            cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, ds.max_smem_optin);
-            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gemm pair)");
-            g_pair_attr[b_mn ? 1 : 0] = true;
-        }
+        const int rc = ensure_smem_optin(reinterpret_cast<const void *>(fn), ds.max_smem_optin, ds.device,
+                                         "cudaFuncSetAttribute(gemm pair)");
+        if (rc) return rc;
     }
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];

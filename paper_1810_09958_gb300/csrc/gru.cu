@@ -555,21 +555,17 @@ GruKernel gru_kernel_for(int ks, int bp = kBatchPad) {
     return bp == 64 ? gru_kernel_for_bp<64>(ks) : gru_kernel_for_bp<32>(ks);
 }
 
-// Opts every instantiation in to `bytes` of dynamic shared memory (once per process).
-int gru_smem_attr(int bytes) {
-    static std::mutex mu;
-    static bool done = false;
-    std::lock_guard<std::mutex> lk(mu);
-    if (done) return ISAM_OK;
+// Opts every instantiation in to `bytes` of dynamic shared memory on the
+// current device (ordinal `device`; the record is kept per device).
+int gru_smem_attr(int bytes, int device) {
     const int ks[3] = {1, 2, 4}, bps[3] = {32, 64, 128};
     for (int k : ks)
         for (int bp : bps) {
             if (!gru_bp_ok(k, bp)) continue;
-            cudaError_t e =
-                cudaFuncSetAttribute(gru_kernel_for(k, bp), cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru)");
+            const int rc = ensure_smem_optin(reinterpret_cast<const void *>(gru_kernel_for(k, bp)), bytes, device,
+                                             "cudaFuncSetAttribute(gru)");
+            if (rc) return rc;
         }
-    done = true;
     return ISAM_OK;
 }
 
@@ -636,9 +632,11 @@ int recurrent_maps(const uint16_t *U, const uint16_t *hx, int H, CUtensorMap *tm
 }
 
 // Fills the shape fields of p and launches the recurrence: one cluster of KS
-// CTAs per group of 32 units; cooperative (guaranteed co-residency) when the
-// driver accepts it with clusters, otherwise after checking that every
-// cluster fits at once (the step counter needs every CTA resident).
+// CTAs per group of 32 units, as a plain cluster launch after checking that
+// every cluster fits on the device at once (the step counter needs every CTA
+// resident).  No cooperative attribute: a launch that carries both it and the
+// cluster shape can lose the cluster shape when a tool re-issues it, and the
+// bounded waits already turn a CTA that never runs into ISAM_ERR_TIMEOUT.
 int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tmH0,
                      const CUtensorMap &tmH1, const CUtensorMap &tmR0, const CUtensorMap &tmR1,
                      const CUtensorMap &tmWn, size_t smem, cudaStream_t stream, int bp = kBatchPad) {
@@ -651,26 +649,20 @@ int launch_recurrent(GruParams &p, const CUtensorMap &tmU, const CUtensorMap &tm
     p.nq = (p.ka % 4 == 0) ? 4 : (p.ka % 3 == 0) ? 3 : (p.ka % 2 == 0) ? 2 : 1;
     p.qk = p.ka / p.nq;
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[2];
+    cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = static_cast<unsigned>(p.ks);
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeCooperative;
-    attr[1].val.cooperative = 1;
     cfg.gridDim = dim3(static_cast<unsigned>(p.n_cta), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    const GruKernel kern = gru_kernel_for(p.ks, bp);
-    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmU, tmH0, tmH1, tmR0, tmR1, tmWn, p);
-    if (e == cudaSuccess) return ISAM_OK;
-    (void)cudaGetLastError();
     cfg.numAttrs = 1;
+    const GruKernel kern = gru_kernel_for(p.ks, bp);
     int max_clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+    cudaError_t e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
     if (e != cudaSuccess) return cuda_error(e, "cudaOccupancyMaxActiveClusters(gru)");
     if (max_clusters * p.ks < p.n_cta)
         return set_error(ISAM_ERR_UNSUPPORTED,
@@ -802,7 +794,7 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
         cudaError_t e = cudaMalloc(&ds.gru_counter, 256);
         if (e != cudaSuccess) return cuda_error(e, "allocating the GRU step counter");
     }
-    if ((rc = gru_smem_attr(ds.max_smem_optin))) return rc;
+    if ((rc = gru_smem_attr(ds.max_smem_optin, ds.device))) return rc;
 
     const size_t wsz = static_cast<size_t>(3) * H * H;
     uint16_t *rhx = ds.gru_hx + static_cast<size_t>(2) * bp * H;
@@ -1044,7 +1036,7 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
             if (rc) return rc;
         }
         nd = g_noalloc[dev];
-        int rc0 = gru_smem_attr(nd.smem_optin);
+        int rc0 = gru_smem_attr(nd.smem_optin, dev);
         if (rc0) return rc0;
     }
     const int n_cta = gru_cta_count(H);
@@ -1106,12 +1098,14 @@ extern "C" int isam_gru_forward_noalloc(int T, int batch, int hidden, const isam
         p.gxp_out = nullptr;
         if ((rc = launch_recurrent(p, tmU, tmH0, tmH1, tmH0, tmH1, tmU, smem, stream))) return rc;
     }
-    // Report device-side timeouts of this call before returning.
+    // Report device-side timeouts of this call before returning: the error
+    // word is read back on the call's own stream (no wait on other streams),
+    // then that stream alone is synchronised.
+    uint32_t w[4] = {0, 0, 0, 0};
+    if ((e = cudaMemcpyAsync(w, err, sizeof w, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+        return cuda_error(e, "isam_gru_forward_noalloc: reading the scratch error word");
     if ((e = cudaStreamSynchronize(stream)) != cudaSuccess)
         return cuda_error(e, "isam_gru_forward_noalloc: cudaStreamSynchronize");
-    uint32_t w[4] = {0, 0, 0, 0};
-    if ((e = cudaMemcpy(w, err, sizeof w, cudaMemcpyDeviceToHost)) != cudaSuccess)
-        return cuda_error(e, "isam_gru_forward_noalloc: reading the scratch error word");
     if (w[0] & DEV_ERR_LAUNCH_SHAPE)
         return set_error(ISAM_ERR_CUDA,
                          "isam_gru_forward_noalloc: the recurrent kernel found clusters of %u CTAs, "

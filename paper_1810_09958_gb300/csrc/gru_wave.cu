@@ -440,8 +440,6 @@ int wave_exchange_map(const uint16_t *slot, int H, int qk, CUtensorMap *tm) {
     return make_tmap_3d_bf16(tm, slot, dims, strides, box);
 }
 
-std::mutex g_wave_mu;
-bool g_wave_attr = false;
 
 }  // namespace
 
@@ -483,37 +481,27 @@ int gru_wave_launch(int T, int batch, int H, const float *gx_a, const uint16_t *
         (rc = wave_exchange_map(hx_a + slot, H, p.qk, &tmHa1)) || (rc = wave_exchange_map(hx_b, H, p.qk, &tmHb0)) ||
         (rc = wave_exchange_map(hx_b + slot, H, p.qk, &tmHb1)))
         return rc;
-    {
-        std::lock_guard<std::mutex> lk(g_wave_mu);
-        if (!g_wave_attr) {
-            cudaError_t e = cudaFuncSetAttribute(gru_wave_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 ds.max_smem_optin);
-            if (e != cudaSuccess) return cuda_error(e, "cudaFuncSetAttribute(gru wave)");
-            g_wave_attr = true;
-        }
-    }
+    if ((rc = ensure_smem_optin(reinterpret_cast<const void *>(gru_wave_kernel), ds.max_smem_optin, ds.device,
+                                "cudaFuncSetAttribute(gru wave)")))
+        return rc;
     cudaError_t e = cudaMemsetAsync(counter, 0, sizeof(uint32_t), stream);
     if (e != cudaSuccess) return cuda_error(e, "clearing the GRU round counter");
     const size_t smem = gru_wave_smem_bytes(H);
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[2];
+    // A plain cluster launch, once every cluster is known to fit at the same
+    // time (the round counter needs every CTA resident); no cooperative
+    // attribute, whose combination with the cluster shape a tool's re-issue
+    // of the launch can drop.
+    cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = kKS;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeCooperative;
-    attr[1].val.cooperative = 1;
     cfg.gridDim = dim3(static_cast<unsigned>(p.n_cta), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cfg.attrs = attr;
-    cfg.numAttrs = 2;
-    e = cudaLaunchKernelEx(&cfg, gru_wave_kernel, tmUa, tmWb, tmUb, tmHa0, tmHa1, tmHb0, tmHb1, p);
-    if (e == cudaSuccess) return ISAM_OK;
-    (void)cudaGetLastError();
-    // Without the cooperative attribute: only if every cluster fits at once
-    // (the round counter needs every CTA resident).
     cfg.numAttrs = 1;
     int max_clusters = 0;
     e = cudaOccupancyMaxActiveClusters(&max_clusters, gru_wave_kernel, &cfg);

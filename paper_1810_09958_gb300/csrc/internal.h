@@ -43,6 +43,11 @@ unsigned long long wait_timeout_ns();
 int set_error(int code, const char *fmt, ...);
 int cuda_error(cudaError_t e, const char *what);
 
+// Raises kernel fn's dynamic shared-memory limit to at least `bytes` on the
+// current device, whose ordinal is `device`.  The attribute belongs to each
+// device's context, so the record of what was set is kept per (device, kernel).
+int ensure_smem_optin(const void *fn, int bytes, int device, const char *what);
+
 // cuTensorMapEncodeTiled through the runtime's driver entry point, with a
 // small cache keyed on every encoded field.
 int make_tmap_2d_bf16(CUtensorMap *out, const void *base, uint64_t inner, uint64_t outer,

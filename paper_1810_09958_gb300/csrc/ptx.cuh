@@ -152,18 +152,6 @@ __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t b
         : "memory");
 }
 
-// 3-D tensor box multicast to every CTA of the cluster in cta_mask: the data
-// lands at the same shared offset in each, and each CTA's mbarrier at the same
-// offset receives the complete_tx.
-__device__ __forceinline__ void tma_load_3d_mc(const void *map, uint64_t *bar, void *dst, int32_t c0,
-                                               int32_t c1, int32_t c2, uint16_t cta_mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(smem_u32(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "h"(cta_mask)
-        : "memory");
-}
-
 // Bulk tensor store shared -> global (rows/cols outside the tensor are clipped).
 __device__ __forceinline__ void tma_store_2d(const void *map, const void *src, int32_t c0, int32_t c1) {
     asm volatile(

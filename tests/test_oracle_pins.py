@@ -588,3 +588,156 @@ def test_gru_stack_lower_layers_ignore_upper_weights(oracle_lib, reset_before):
     c = oracle_lib.gru_stack(x, W2, U2, b, h0, reset_before=reset_before)
     assert np.array_equal(a[:-1], c[:-1])
     assert np.max(np.abs(a[-1] - c[-1])) > 1e-3
+
+
+# ---- reset-before candidate: where the reset gate sits relative to U_n
+
+def _masked_reset(b, H, mask):
+    """b with b_ir = +30 on the units where mask is 1 and -30 elsewhere."""
+    b = b.copy()
+    b[:H] = np.where(mask, 30.0, -30.0).astype(np.float32)
+    return b
+
+
+def _masked_reset_case(seed, T=4, B=3, H=16):
+    """Operands whose reset gate is a fixed 0/1 mask per unit: the r rows of W
+    and U are zero, so r_j = sigmoid(b_ir_j + b_hr_j) with b_ir = +-30."""
+    x, W, U, b, _ = synth.gru_operands(T, B, H, seed=seed)
+    h0 = synth.f32_uniform(seed + 1, (B, H))
+    W = W.copy()
+    U = U.copy()
+    W[:H] = 0
+    U[:H] = 0
+    mask = (np.arange(H) % 3 != 1)          # mixed pattern, both values present
+    return x, W, U, b, h0, mask
+
+
+def _masked_reset_expected(oracle_gru, x, W, U, b, h0, mask, H):
+    """With r = mask, U_n (r * h) = (U_n with the columns of the masked-off
+    units zeroed) h, which the reset-after form computes exactly when its own
+    reset gate is 1 everywhere (b_ir = +30, r = 1 to 1e-13)."""
+    Um = U.copy()
+    Um[2 * H:, ~mask] = 0
+    b1 = _masked_reset(b, H, np.ones(H, dtype=bool))
+    return oracle_gru(x, W, Um, b1, h0)
+
+
+def test_gru_reset_before_masked_reset_gate(oracle_lib):
+    """A per-unit 0/1 reset gate selects COLUMNS of U_n in the reset-before
+    form (r multiplies h before the product), never rows of the product:
+    the slips r * (U_n h) + b_hn and r * (U_n h + b_hn) both fail here."""
+    T, B, H = 4, 3, 16
+    x, W, U, b, h0, mask = _masked_reset_case(90, T, B, H)
+    got = oracle_lib.gru_forward(x, W, U, _masked_reset(b, H, mask), h0, reset_before=True)
+    want = _masked_reset_expected(oracle_lib.gru_forward, x, W, U, b, h0, mask, H)
+    assert np.max(np.abs(got - want)) < 1e-10
+    # the row-selecting reading gives a clearly different answer on these inputs
+    Ur = U.copy()
+    Ur[2 * H:][~mask] = 0
+    wrong = oracle_lib.gru_forward(x, W, Ur, _masked_reset(b, H, np.ones(H, dtype=bool)), h0)
+    assert np.max(np.abs(wrong - want)) > 1e-3
+
+
+@pytest.mark.parametrize("layers", [1, 2])
+def test_gru_stack_reset_before_masked_reset_gate(oracle_lib, layers):
+    """The same pin through the stacked oracle's reset-before branch: every
+    layer's reset gate is a mask, so each layer equals the reset-after stack
+    with its U_n columns zeroed."""
+    T, B, H = 4, 3, 16
+    x, W1, U1, b1, h01, mask = _masked_reset_case(91, T, B, H)
+    Ws, Us, bs, bref, Uref = [], [], [], [], []
+    for l in range(layers):
+        _, Wl, Ul, bl, _, _ = _masked_reset_case(92 + 5 * l, T, B, H)
+        Ws.append(Wl)
+        Us.append(Ul)
+        bs.append(_masked_reset(bl, H, mask))
+        bref.append(_masked_reset(bl, H, np.ones(H, dtype=bool)))
+        Um = Ul.copy()
+        Um[2 * H:, ~mask] = 0
+        Uref.append(Um)
+    h0 = synth.f32_uniform(93, (layers, B, H))
+    got = oracle_lib.gru_stack(x, np.stack(Ws), np.stack(Us), np.stack(bs), h0, reset_before=True)
+    want = oracle_lib.gru_stack(x, np.stack(Ws), np.stack(Uref), np.stack(bref), h0)
+    assert np.max(np.abs(got - want)) < 1e-10
+
+
+def _build_mutant(tmp_path, replacements):
+    """Compiles a copy of the oracle's C source with the given text edits (a
+    planted mistake) into a library of its own under tmp_path."""
+    import ctypes
+    import os
+    import subprocess
+    import oracle
+    src = open(os.path.join(os.path.dirname(oracle.__file__), "isam_oracle.c")).read()
+    for old, new in replacements:
+        assert src.count(old) == 1, old
+        src = src.replace(old, new)
+    c = tmp_path / "mutant.c"
+    c.write_text(src)
+    so = tmp_path / "libmutant.so"
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+                    "-o", str(so), str(c), "-lm"], check=True)
+    lib = ctypes.CDLL(str(so))
+    P, i = ctypes.c_void_p, ctypes.c_int
+    lib.oracle_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
+    lib.oracle_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
+    lib.oracle_gru_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
+    return lib
+
+
+def _call_gru(fn, x, W, U, b, h0):
+    import ctypes
+    T, B, H = x.shape
+    out = np.empty((T, B, H))
+    arrs = [np.ascontiguousarray(a) for a in (x, W, U, b.astype(np.float32), h0.astype(np.float32))]
+    ptr = [a.ctypes.data_as(ctypes.c_void_p) for a in arrs]
+    assert fn(T, B, H, *ptr, out.ctypes.data_as(ctypes.c_void_p)) == 0
+    return out
+
+
+def test_masked_reset_pin_catches_a_planted_slip(tmp_path, oracle_lib):
+    """Plants r * (U_n h) + b_hn into a copy of the reset-before oracle (CPU
+    only).  The copy still passes the saturated-gate pins (r = 1, and r = 0
+    with b_hn = 0), and the masked-reset pin fails it."""
+    mut = _build_mutant(tmp_path, [
+        ("rh[j] = r * h[j];", "rh[j] = r;"),
+        ("for (int k = 0; k < H; ++k) an += bf(un[k]) * rh[k];",
+         "for (int k = 0; k < H; ++k) an += bf(un[k]) * h[k];"),
+        ("const double n = tanh(gx[2 * H + j] + an + (double)b[G + 2 * H + j]);",
+         "const double n = tanh(gx[2 * H + j] + rh[j] * an + (double)b[G + 2 * H + j]);"),
+    ])
+    T, B, H = 4, 3, 16
+    # r = 1 everywhere: the slip agrees with the true form
+    x, W, U, b, _ = synth.gru_operands(T, B, H, seed=46)
+    h0 = synth.f32_uniform(47, (B, H))
+    b1 = b.copy()
+    b1[:H] = 30.0
+    np.testing.assert_allclose(_call_gru(mut.oracle_gru_forward_reset_before, x, W, U, b1, h0),
+                               oracle_lib.gru_forward(x, W, U, b1, h0, reset_before=True), rtol=0, atol=1e-10)
+    # the masked reset gate separates them
+    x, W, U, b, h0, mask = _masked_reset_case(90, T, B, H)
+    got = _call_gru(mut.oracle_gru_forward_reset_before, x, W, U, _masked_reset(b, H, mask), h0)
+    want = _masked_reset_expected(oracle_lib.gru_forward, x, W, U, b, h0, mask, H)
+    assert np.max(np.abs(got - want)) > 1e-3
+
+
+def test_masked_reset_pin_catches_a_planted_slip_in_the_stack(tmp_path, oracle_lib):
+    """The same slip planted in the stacked oracle's layer loop."""
+    import ctypes
+    mut = _build_mutant(tmp_path, [
+        ("rh[j] = reset_before ? r * h[j] : h[j];", "rh[j] = h[j];"),
+        ("const double n = reset_before ? tanh(gx[2 * H + j] + gh[2 * H + j])",
+         "const double n = reset_before ? tanh(gx[2 * H + j] + r * (gh[2 * H + j] - (double)b[G + 2 * H + j])"
+         " + (double)b[G + 2 * H + j])"),
+    ])
+    T, B, H = 4, 3, 16
+    x, W, U, b, h0, mask = _masked_reset_case(91, T, B, H)
+    bm = _masked_reset(b, H, mask)
+    out = np.empty((1, T, B, H))
+    arrs = [np.ascontiguousarray(a) for a in (x, W[None], U[None], bm[None], h0[None].astype(np.float32))]
+    ptr = [a.ctypes.data_as(ctypes.c_void_p) for a in arrs]
+    assert mut.oracle_gru_stack(1, T, B, H, 1, *ptr, out.ctypes.data_as(ctypes.c_void_p)) == 0
+    want = _masked_reset_expected(oracle_lib.gru_forward, x, W, U, b, h0, mask, H)
+    assert np.max(np.abs(out[0] - want)) > 1e-3
+    good = oracle_lib.gru_stack(x, W[None], U[None], bm[None], h0[None], reset_before=True)
+    assert np.max(np.abs(good[0] - want)) < 1e-10
