@@ -18,7 +18,13 @@ from gpu_util import Guarded, dev_bf16, nmax_err
 
 pytestmark = pytest.mark.gpu
 TOL = 1e-2    # the GRU parity tolerance against the fp64 oracle
-TIGHT = 1e-4  # against the regular entry point: the same kernels, projection in chunks
+# Against the regular entry point.  Both run the same recurrent kernel, but the
+# chunked projection GEMM has a different M, hence another tile plan and
+# summation order; last-bit differences in G_x flip a few bf16 roundings of h
+# for the tensor cores, which measured 1.6e-4 after 128 steps.  An error at a
+# chunk boundary (h carried from the wrong step) is of the order of a step's
+# change in h, above 1e-1.
+TIGHT = 1e-3
 
 
 def _ptr(t):
