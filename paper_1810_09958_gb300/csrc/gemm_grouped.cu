@@ -66,8 +66,11 @@ struct GroupParams {
     CUtensorMap tmC[kMaxGroup];
 };
 
-__device__ __forceinline__ int find_problem(const GroupParams &p, int tile) {
-    int i = 0;
+// The problem that owns `tile`, searched forward from `i` (a CTA visits its
+// tiles in increasing order, so each role keeps its index and the search
+// advances by at most a few entries per tile instead of rescanning the table
+// in parameter space).
+__device__ __forceinline__ int find_problem(const GroupParams &p, int tile, int i) {
     while (i + 1 < p.count && p.prob[i + 1].tile_start <= tile) ++i;
     return i;
 }
@@ -122,11 +125,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
-            int stage = 0, issued = 0;
+            int stage = 0, issued = 0, pi = 0;
             uint32_t phase = 0;
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < p.total_tiles; tile += gridDim.x) {
-                const int pi = find_problem(p, tile);
+                pi = find_problem(p, tile, pi);
                 const GroupProblem &pr = p.prob[pi];
                 const int local = tile - pr.tile_start;
                 const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
@@ -177,11 +180,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
-            int stage = 0, acc = 0;
+            int stage = 0, acc = 0, pi = 0;
             uint32_t phase = 0, acc_phase = 0;
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < p.total_tiles; tile += gridDim.x) {
-                const GroupProblem &pr = p.prob[find_problem(p, tile)];
+                pi = find_problem(p, tile, pi);
+                const GroupProblem &pr = p.prob[pi];
                 const bool f8 = pr.fp8 != 0;
                 const uint32_t idesc =
                     f8 ? idesc_e4m3_f32(kBM, pr.bn) : idesc_bf16_f32(kBM, pr.bn, pr.a_mn != 0, pr.b_mn != 0);
@@ -230,10 +234,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
         uint64_t *cb = cbar + ew * 2;
         uint32_t cpar[2] = {0u, 0u};
         bool cpend[2] = {false, false};
-        int gbuf = 0, acc = 0;
+        int gbuf = 0, acc = 0, pi = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < p.total_tiles; tile += gridDim.x) {
-            const int pi = find_problem(p, tile);
+            pi = find_problem(p, tile, pi);
             const GroupProblem &pr = p.prob[pi];
             const int local = tile - pr.tile_start;
             const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
