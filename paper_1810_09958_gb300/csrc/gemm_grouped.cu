@@ -14,6 +14,7 @@
 // 16-byte aligned).  Layout (NN/TN/NT/TT) and tile width are per problem; a
 // problem's tensor maps travel in the kernel parameters.
 #include <algorithm>
+#include <cstdlib>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -49,6 +50,7 @@ struct GroupProblem {
     int M, N, K;
     int m_tiles, n_tiles, kb_total;
     int a_mn, b_mn, bn;
+    int panels;       // 128-row A panels per tile: 1, or 2 (256-row tiles for the heavy problems)
     int fp8;          // E4M3 operands (both K-major): 128-element K atoms
     int tma_c;        // C rows 16-byte aligned: TMA epilogue
     int tile_start;   // first global tile index of this problem
@@ -95,7 +97,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    constexpr uint32_t kTmemCols = 2 * kBNMax;
+    constexpr uint32_t kTmemCols = 4 * kBNMax;  // two accumulators of two 128-row panels
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < ST; ++i) {
@@ -133,9 +135,44 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                 const GroupProblem &pr = p.prob[pi];
                 const int local = tile - pr.tile_start;
                 const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
+                const int panels = pr.panels;
                 const uint32_t bbytes = pr.b_mn ? static_cast<uint32_t>((pr.bn + 63) / 64) * 8192u
                                                 : static_cast<uint32_t>(pr.bn) * 128u;
+                if (panels == 1) {
+                    for (int kb = 0; kb < pr.kb_total; ++kb) {
+                        if (!bounded_wait(&empty[stage], phase ^ 1u, w, SITE_G_EMPTY)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(kAStage) + bbytes);
+                        uint8_t *a = sA + static_cast<size_t>(stage) * kAStage;
+                        uint8_t *b = sB + static_cast<size_t>(stage) * kBStage;
+                        const int k0 = kb * (pr.fp8 ? 2 * kBK : kBK);  // in elements
+                        if (pr.a_mn) {
+                            tma_load_2d(&p.tmA[pi], &full[stage], a, mt * kBM, k0);
+                            tma_load_2d(&p.tmA[pi], &full[stage], a + 8192, mt * kBM + 64, k0);
+                        } else {
+                            tma_load_2d(&p.tmA[pi], &full[stage], a, k0, mt * kBM);
+                        }
+                        if (pr.b_mn) {
+                            for (int c = 0; c < (pr.bn + 63) / 64; ++c)
+                                tma_load_2d(&p.tmB[pi], &full[stage], b + c * 8192, nt * pr.bn + c * 64, k0);
+                        } else {
+                            tma_load_2d(&p.tmB[pi], &full[stage], b, k0, nt * pr.bn);
+                        }
+                        ++issued;
+                        if (++stage == ST) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                    }
+                    continue;
+                }
+                // A k-block of a 256-row tile takes two consecutive stages:
+                // panel 0 and the B block in the first, panel 1 in the second.
+                const int r0 = mt * 2 * kBM, r1 = r0 + kBM;
                 for (int kb = 0; kb < pr.kb_total; ++kb) {
+                    const int k0 = kb * (pr.fp8 ? 2 * kBK : kBK);  // in elements
                     if (!bounded_wait(&empty[stage], phase ^ 1u, w, SITE_G_EMPTY)) {
                         ok = false;
                         break;
@@ -143,18 +180,34 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                     mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(kAStage) + bbytes);
                     uint8_t *a = sA + static_cast<size_t>(stage) * kAStage;
                     uint8_t *b = sB + static_cast<size_t>(stage) * kBStage;
-                    const int k0 = kb * (pr.fp8 ? 2 * kBK : kBK);  // in elements
                     if (pr.a_mn) {
-                        tma_load_2d(&p.tmA[pi], &full[stage], a, mt * kBM, k0);
-                        tma_load_2d(&p.tmA[pi], &full[stage], a + 8192, mt * kBM + 64, k0);
+                        tma_load_2d(&p.tmA[pi], &full[stage], a, r0, k0);
+                        tma_load_2d(&p.tmA[pi], &full[stage], a + 8192, r0 + 64, k0);
                     } else {
-                        tma_load_2d(&p.tmA[pi], &full[stage], a, k0, mt * kBM);
+                        tma_load_2d(&p.tmA[pi], &full[stage], a, k0, r0);
                     }
                     if (pr.b_mn) {
                         for (int c = 0; c < (pr.bn + 63) / 64; ++c)
                             tma_load_2d(&p.tmB[pi], &full[stage], b + c * 8192, nt * pr.bn + c * 64, k0);
                     } else {
                         tma_load_2d(&p.tmB[pi], &full[stage], b, k0, nt * pr.bn);
+                    }
+                    ++issued;
+                    if (++stage == ST) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                    if (!bounded_wait(&empty[stage], phase ^ 1u, w, SITE_G_EMPTY)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[stage], static_cast<uint32_t>(kAStage));
+                    a = sA + static_cast<size_t>(stage) * kAStage;
+                    if (pr.a_mn) {
+                        tma_load_2d(&p.tmA[pi], &full[stage], a, r1, k0);
+                        tma_load_2d(&p.tmA[pi], &full[stage], a + 8192, r1 + 64, k0);
+                    } else {
+                        tma_load_2d(&p.tmA[pi], &full[stage], a, k0, r1);
                     }
                     ++issued;
                     if (++stage == ST) {
@@ -191,30 +244,86 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                     f8 ? idesc_e4m3_f32(kBM, pr.bn) : idesc_bf16_f32(kBM, pr.bn, pr.a_mn != 0, pr.b_mn != 0);
                 if (!bounded_wait(&tempty[acc], acc_phase ^ 1u, w, SITE_G_TEMPTY)) break;
                 tc_fence_after();
-                const uint32_t d = tmem_base + static_cast<uint32_t>(acc * kBNMax);
-                for (int kb = 0; kb < pr.kb_total; ++kb) {
-                    if (!bounded_wait(&full[stage], phase, w, SITE_G_FULL)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t a0 = smem_u32(sA + static_cast<size_t>(stage) * kAStage);
-                    const uint32_t b0 = smem_u32(sB + static_cast<size_t>(stage) * kBStage);
+                const uint32_t d = tmem_base + static_cast<uint32_t>(acc * 2 * kBNMax);
+                if (pr.panels == 1) {
+                    for (int kb = 0; kb < pr.kb_total; ++kb) {
+                        if (!bounded_wait(&full[stage], phase, w, SITE_G_FULL)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a0 = smem_u32(sA + static_cast<size_t>(stage) * kAStage);
+                        const uint32_t b0 = smem_u32(sB + static_cast<size_t>(stage) * kBStage);
 #pragma unroll
-                    for (int k = 0; k < kBK / 16; ++k) {
-                        const uint64_t ad = pr.a_mn ? sdesc_sw128(a0 + k * 2048, 8192, 1024)
-                                                    : sdesc_sw128(a0 + k * 32, 16, 1024);
-                        const uint64_t bd = pr.b_mn ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
-                                                    : sdesc_sw128(b0 + k * 32, 16, 1024);
-                        if (f8)
-                            umma_f8(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
-                        else
-                            umma_bf16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint64_t ad = pr.a_mn ? sdesc_sw128(a0 + k * 2048, 8192, 1024)
+                                                        : sdesc_sw128(a0 + k * 32, 16, 1024);
+                            const uint64_t bd = pr.b_mn ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
+                                                        : sdesc_sw128(b0 + k * 32, 16, 1024);
+                            if (f8)
+                                umma_f8(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                            else
+                                umma_bf16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                        }
+                        umma_commit(&empty[stage]);
+                        if (++stage == ST) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
                     }
-                    umma_commit(&empty[stage]);
-                    if (++stage == ST) {
-                        stage = 0;
-                        phase ^= 1u;
+                } else {
+                    // 256-row tile: each k-block spans two stages, panel 0
+                    // with the B block, then panel 1; both panels multiply
+                    // the first stage's B, so both stages are freed after
+                    // the k-block's last MMA.
+                    for (int kb = 0; kb < pr.kb_total; ++kb) {
+                        const int s0 = stage;
+                        if (!bounded_wait(&full[s0], phase, w, SITE_G_FULL)) {
+                            ok = false;
+                            break;
+                        }
+                        if (++stage == ST) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                        tc_fence_after();
+                        const uint32_t a0 = smem_u32(sA + static_cast<size_t>(s0) * kAStage);
+                        const uint32_t b0 = smem_u32(sB + static_cast<size_t>(s0) * kBStage);
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint64_t ad = pr.a_mn ? sdesc_sw128(a0 + k * 2048, 8192, 1024)
+                                                        : sdesc_sw128(a0 + k * 32, 16, 1024);
+                            const uint64_t bd = pr.b_mn ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
+                                                        : sdesc_sw128(b0 + k * 32, 16, 1024);
+                            if (f8)
+                                umma_f8(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                            else
+                                umma_bf16(d, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                        }
+                        const int s1 = stage;
+                        if (!bounded_wait(&full[s1], phase, w, SITE_G_FULL)) {
+                            ok = false;
+                            break;
+                        }
+                        if (++stage == ST) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                        tc_fence_after();
+                        const uint32_t a1 = smem_u32(sA + static_cast<size_t>(s1) * kAStage);
+#pragma unroll
+                        for (int k = 0; k < kBK / 16; ++k) {
+                            const uint64_t ad = pr.a_mn ? sdesc_sw128(a1 + k * 2048, 8192, 1024)
+                                                        : sdesc_sw128(a1 + k * 32, 16, 1024);
+                            const uint64_t bd = pr.b_mn ? sdesc_sw128(b0 + k * 2048, 8192, 1024)
+                                                        : sdesc_sw128(b0 + k * 32, 16, 1024);
+                            if (f8)
+                                umma_f8(d + kBNMax, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                            else
+                                umma_bf16(d + kBNMax, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                        }
+                        umma_commit(&empty[s0]);
+                        umma_commit(&empty[s1]);
                     }
                 }
                 if (!ok) break;
@@ -241,10 +350,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
             const GroupProblem &pr = p.prob[pi];
             const int local = tile - pr.tile_start;
             const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
-            const int row0 = mt * kBM + q * 32;
             const int col0 = nt * pr.bn;
             const bool load_c = pr.tma_c && pr.beta != 0.0f;
             const int nch = (pr.bn + 31) / 32;
+            bool ok = true;
+            for (int pn = 0; ok && pn < pr.panels; ++pn) {
+            const int row0 = (mt * pr.panels + pn) * kBM + q * 32;
+            if ((mt * pr.panels + pn) * kBM >= pr.M) {
+                // a second panel wholly below the matrix: nothing to store
+                continue;
+            }
             if (load_c) {
                 if (lane == 0) {
                     bulk_wait_read<0>();
@@ -255,11 +370,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                 cpend[gbuf & 1] = true;
                 __syncwarp();
             }
-            if (!warp_wait(&tfull[acc], acc_phase, w, SITE_G_TFULL)) break;
-            tc_fence_after();
+            if (pn == 0) {
+                if (!warp_wait(&tfull[acc], acc_phase, w, SITE_G_TFULL)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+            }
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
-                                   static_cast<uint32_t>(acc * kBNMax);
-            bool ok = true;
+                                   static_cast<uint32_t>(acc * 2 * kBNMax + pn * kBNMax);
             for (int j = 0; j < nch; ++j) {
                 const int b = gbuf & 1;
                 if (load_c && j + 1 < nch) {
@@ -338,6 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                 }
                 ++gbuf;
             }
+            }
             if (!ok) break;
             tc_fence_before();
             __syncwarp();
@@ -378,12 +498,36 @@ std::mutex g_group_mu;
 int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStream_t stream) {
     if (count < 1 || count > kMaxGroup)
         return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped: count must be in [1, %d]", kMaxGroup);
+    auto atoms = [&](int i) { return (g[i].K + (g[i].fp8 ? 2 * kBK : kBK) - 1) / (g[i].fp8 ? 2 * kBK : kBK); };
+    // Tile height: 256 rows (two 128-row panels sharing each B block) for
+    // problems whose 128-row panel of A is 640 KB or more, which halves the
+    // tile starts a CTA pays on them; kept at 128 rows when that would leave
+    // fewer than two tiles per SM.
+    int panels[kMaxGroup];
+    {
+        long long tall_tiles = 0;
+        for (int i = 0; i < count; ++i) {
+            const long long eb = g[i].fp8 ? 1 : 2;
+            panels[i] = (g[i].M > kBM && static_cast<long long>(kBM) * g[i].K * eb >= 640 * 1024) ? 2 : 1;
+            const int bn = std::min(kBNMax, (g[i].N + 15) / 16 * 16);
+            tall_tiles += static_cast<long long>((g[i].M + kBM * panels[i] - 1) / (kBM * panels[i])) *
+                          ((g[i].N + bn - 1) / bn);
+        }
+        if (tall_tiles < 2LL * ds.num_sms)
+            for (int i = 0; i < count; ++i) panels[i] = 1;
+        // ISAM_GROUP_PANELS=1 or 2 forces the tile height (2: every problem
+        // taller than one panel), for tests and measurements.
+        const char *fe = getenv("ISAM_GROUP_PANELS");
+        const int forced = fe ? atoi(fe) : 0;
+        if (forced == 1 || forced == 2)
+            for (int i = 0; i < count; ++i) panels[i] = (forced == 2 && g[i].M > kBM) ? 2 : 1;
+    }
     // Host-side order: problems with the costliest tiles first, so the
     // round-robin walk over tiles ends with the cheap ones.
     int order[kMaxGroup];
     std::iota(order, order + count, 0);
-    auto atoms = [&](int i) { return (g[i].K + (g[i].fp8 ? 2 * kBK : kBK) - 1) / (g[i].fp8 ? 2 * kBK : kBK); };
-    std::stable_sort(order, order + count, [&](int a, int b) { return atoms(a) > atoms(b); });
+    std::stable_sort(order, order + count,
+                     [&](int a, int b) { return atoms(a) * panels[a] > atoms(b) * panels[b]; });
 
     static GroupParams p;  // ~29 KB: built under the lock, copied into the launch
     std::lock_guard<std::mutex> lk(g_group_mu);
@@ -400,7 +544,8 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
         pr.a_mn = d.fp8 ? 0 : d.transA;
         pr.b_mn = (d.fp8 || d.transB == 1) ? 0 : 1;
         pr.bn = std::min(kBNMax, (d.N + 15) / 16 * 16);
-        pr.m_tiles = (d.M + kBM - 1) / kBM;
+        pr.panels = panels[order[s]];
+        pr.m_tiles = (d.M + kBM * pr.panels - 1) / (kBM * pr.panels);
         pr.n_tiles = (d.N + pr.bn - 1) / pr.bn;
         pr.kb_total = atoms(order[s]);
         pr.tma_c = (d.N % 4 == 0) ? 1 : 0;

@@ -129,3 +129,42 @@ def test_grouped_fp8_integer_bit_exact_ragged():
              (1, 8, 16, 1.0, 0.0), (257, 129, 1008, 1.0, -2.0)]
     for (got, ref), spec in zip(run_group_fp8(specs, dist="int"), specs):
         assert np.array_equal(got.astype(np.float64), ref), spec
+
+
+# 256-row tiles (two 128-row panels sharing each B block) forced on every
+# problem taller than one panel: last tiles whose second panel is partial,
+# a single row, or wholly below the matrix; all four layouts; beta and plain
+# stores (N % 4 != 0).
+TALL_SPECS = [(328, 200, 584, 0, 0, 2.0, -1.0), (200, 13, 136, 0, 1, 1.0, 0.5), (136, 48, 72, 1, 0, 1.0, 0.0),
+              (384, 160, 264, 1, 1, -1.0, 1.0), (257, 129, 1000, 0, 1, 1.0, -2.0), (640, 16, 2560, 0, 0, 1.0, 0.0),
+              (512, 64, 128, 1, 0, 1.0, 0.0), (1, 8, 8, 0, 0, 1.0, 0.0)]
+
+
+def test_grouped_tall_tiles_integer_bit_exact(monkeypatch):
+    monkeypatch.setenv("ISAM_GROUP_PANELS", "2")
+    for (got, ref), spec in zip(run_group(TALL_SPECS, dist="int4", seed0=1300), TALL_SPECS):
+        assert np.array_equal(got.astype(np.float64), ref), spec
+
+
+def test_grouped_tall_tiles_uniform(monkeypatch):
+    monkeypatch.setenv("ISAM_GROUP_PANELS", "2")
+    for (got, ref), spec in zip(run_group(TALL_SPECS, seed0=1400), TALL_SPECS):
+        assert nmax_err(got, ref) <= TOL, spec
+
+
+def test_grouped_one_panel_tiles_on_the_sweep(monkeypatch):
+    """The skinny sweep with every tile 128 rows high (the heavy problems
+    take 256-row tiles by default)."""
+    monkeypatch.setenv("ISAM_GROUP_PANELS", "1")
+    specs = [(M, N, K, tA, 0, 1.0, 0.0) for tA in (0, 1)
+             for (M, K) in [(2560, 2560), (4096, 4096)] for N in (16, 128)]
+    for (got, ref), spec in zip(run_group(specs, seed0=1500), specs):
+        assert nmax_err(got, ref) <= TOL, spec
+
+
+def test_grouped_fp8_tall_tiles_integer_bit_exact(monkeypatch):
+    monkeypatch.setenv("ISAM_GROUP_PANELS", "2")
+    specs = [(328, 200, 1168, 2.0, -1.0), (200, 13, 144, 1.0, 0.5), (384, 48, 80, 1.0, 0.0),
+             (257, 129, 1008, 1.0, -2.0), (1, 8, 16, 1.0, 0.0)]
+    for (got, ref), spec in zip(run_group_fp8(specs, dist="int", seed0=1600), specs):
+        assert np.array_equal(got.astype(np.float64), ref), spec
