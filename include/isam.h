@@ -114,6 +114,40 @@ int isam_gemm_fp8(int M, int N, int K, float alpha, const uint8_t *A, const uint
                   float *C);
 
 /*
+ * Block-scaled E4M3 GEMM in the OCP Microscaling (MX) form: every 32
+ * consecutive K elements of a row of A, and of a row of B, share one E8M0
+ * scale byte e meaning 2^(e - 127) (e = 255 is NaN):
+ *   C[i][j] <- alpha * sum_k (2^(SA[i][k/32]-127) A[i][k]) (2^(SB[j][k/32]-127) B[j][k])
+ *              + beta * C[i][j].
+ * The paper's instruction selection (Section 2.4) picks the instruction whose
+ * semantics cover the computation; here the tensor cores' block-scaled
+ * operand kind applies the scales inside the product.
+ *   A  M x K, B  N x K: E4M3 bytes, row-major (K-major), device pointers,
+ *      16-byte aligned; K a multiple of 16 (16-byte rows).
+ *   SA [M][ceil(K/32)], SB [N][ceil(K/32)]: E8M0 bytes, row-major, device
+ *      pointers, any alignment.  A last block shorter than 32 (K % 32 != 0)
+ *      has a scale of its own.
+ *   C  M x N fp32 row-major, 16-byte aligned; beta == 0 does not read C.
+ * Products of the scaled operands are exact and accumulate in fp32.  One
+ * persistent launch over 128 x min(128, N rounded up to 16) tiles (no
+ * split-K); asynchronous on the stream set by isam_set_stream.
+ * ISAM_ERR_INVALID_ARG for sizes < 1 or null pointers, ISAM_ERR_UNSUPPORTED
+ * for misaligned pointers or K % 16 != 0.
+ */
+int isam_gemm_mxfp8(int M, int N, int K, float alpha, const uint8_t *A, const uint8_t *SA,
+                    const uint8_t *B, const uint8_t *SB, float beta, float *C);
+
+/*
+ * isam_gemm_mxfp8 for 1 <= count <= 64 independent problems in one launch
+ * (host arrays of count entries; the rules of isam_gemm_grouped: no C[i] may
+ * overlap another problem's operands or result).  Errors name the problem.
+ */
+int isam_gemm_grouped_mxfp8(int count, const int *M, const int *N, const int *K, const float *alpha,
+                            const uint8_t *const *A, const uint8_t *const *SA,
+                            const uint8_t *const *B, const uint8_t *const *SB,
+                            const float *beta, float *const *C);
+
+/*
  * Several independent GEMMs in one launch: problem i computes
  * C[i] <- alpha[i] * op(A[i]) * op(B[i]) + beta[i] * C[i] exactly as isam_gemm
  * would, with the same per-problem argument rules.

@@ -357,6 +357,39 @@ int isam_gemm_grouped_fp8(int count, const int *M, const int *N, const int *K, c
     return gemm_grouped_launch(count, g, *ds, current_stream());
 }
 
+int isam_gemm_mxfp8(int M, int N, int K, float alpha, const uint8_t *A, const uint8_t *SA, const uint8_t *B,
+                    const uint8_t *SB, float beta, float *C) {
+    MxDesc g{M, N, K, alpha, beta, A, SA, B, SB, C};
+    int rc = gemm_mx_validate(g);
+    if (rc) return rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gemm_mx_launch(1, &g, *ds, current_stream());
+}
+
+int isam_gemm_grouped_mxfp8(int count, const int *M, const int *N, const int *K, const float *alpha,
+                            const uint8_t *const *A, const uint8_t *const *SA, const uint8_t *const *B,
+                            const uint8_t *const *SB, const float *beta, float *const *C) {
+    if (count < 1 || count > 64)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped_mxfp8: count must be in [1, 64]");
+    if (!M || !N || !K || !alpha || !A || !SA || !B || !SB || !beta || !C)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_gemm_grouped_mxfp8: null array");
+    MxDesc g[64];
+    for (int i = 0; i < count; ++i) {
+        g[i] = MxDesc{M[i], N[i], K[i], alpha[i], beta[i], A[i], SA[i], B[i], SB[i], C[i]};
+        int rc = gemm_mx_validate(g[i]);
+        if (rc) {
+            char msg[640];  // prefix + the 512-byte error text
+            snprintf(msg, sizeof msg, "isam_gemm_grouped_mxfp8: problem %d: %s", i, isam_last_error_string());
+            return set_error(rc, "%s", msg);
+        }
+    }
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return gemm_mx_launch(count, g, *ds, current_stream());
+}
+
 // Reports the tile plan the cost model picks for a GEMM (for benchmarks and
 // tests; nothing is launched).  out[0..5] = BN, split, stages, group_m, grid,
 // shared-memory bytes.

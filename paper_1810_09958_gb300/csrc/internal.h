@@ -98,6 +98,22 @@ int gemm_pair_launch(const GemmDesc &g, const GemmPlan &plan, DeviceState &ds, c
 // Independent GEMMs in one persistent launch (1 <= count <= 64).
 int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStream_t s);
 
+// Block-scaled E4M3 GEMM (OCP MX): C = alpha (SA o A)(SB o B)^T + beta C with
+// A M x K and B N x K E4M3 bytes (K-major) and one E8M0 scale byte per 32 K
+// elements of each row, SA [M][ceil(K/32)], SB [N][ceil(K/32)].
+struct MxDesc {
+    int M, N, K;
+    float alpha, beta;
+    const uint8_t *A;
+    const uint8_t *SA;
+    const uint8_t *B;
+    const uint8_t *SB;
+    float *C;
+};
+int gemm_mx_validate(const MxDesc &g);
+// One persistent launch over the tiles of 1 <= count <= 64 problems.
+int gemm_mx_launch(int count, const MxDesc *g, DeviceState &ds, cudaStream_t s);
+
 // reset_before: the candidate's recurrent input is U_n (r * h) (two rounds per step).
 int gru_launch(int T, int batch, int hidden, const uint16_t *x, const uint16_t *W,
                const uint16_t *U, const float *b, const float *h0, float *h_out, DeviceState &ds,

@@ -245,6 +245,32 @@ __device__ __forceinline__ void umma_f8(uint32_t d_tmem, uint64_t a_desc, uint64
         : "memory");
 }
 
+// Block-scaled E4M3 MMA (kind::mxf8f6f4, one E8M0 scale per 32 K elements of
+// each row of A and of B): K = 32 per instruction; the scale factors are read
+// from tensor memory at sfa_tmem / sfb_tmem, the byte within each 32-bit cell
+// chosen by the scale-factor IDs of the instruction descriptor.
+__device__ __forceinline__ void umma_mx(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                        uint32_t sfa_tmem, uint32_t sfb_tmem, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %6, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%4], [%5], p;\n\t}" ::"r"(
+            d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(sfa_tmem), "r"(sfb_tmem), "r"(accumulate)
+        : "memory");
+}
+
+// 32 lanes x 32 bit, 4 consecutive columns from registers: thread t of the
+// warp writes columns [col, col + 4) of TMEM lane (lane field of taddr) + t.
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t (&v)[4]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(v[0]), "r"(v[1]),
+                 "r"(v[2]), "r"(v[3])
+                 : "memory");
+}
+
+// Waits until this thread's tcgen05.st have completed.
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
 // ---- the same for a CTA pair (cta_group::2): the two CTAs of a cluster
 // allocate TMEM together and the first one issues MMAs whose A rows and B
 // columns come from both CTAs' shared memory (same offsets in each).  A kernel
@@ -379,6 +405,16 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool a_mn, b
 // code 0 in bits 7-9 and 10-12), both K-major.
 __host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
     return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// Instruction descriptor, kind::mxf8f6f4 with E8M0 scales: E4M3 A and B (format
+// code 0), both K-major, fp32 accumulator (implied by the kind).
+//   bits 4-5 scale-factor ID of B (which byte of its 32-bit TMEM cell),
+//   17-22 N >> 3, 23 scale type (1 = UE8M0), 24-28 M >> 4 (M = 128 only),
+//   29-30 scale-factor ID of A.
+__host__ __device__ constexpr uint32_t idesc_mx_e4m3(int M, int N, uint32_t sfa_id, uint32_t sfb_id) {
+    return ((sfb_id & 3u) << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (1u << 23) |
+           (static_cast<uint32_t>(M >> 4) << 24) | ((sfa_id & 3u) << 29);
 }
 
 // ---------------------------------------------------------------- dependent launch

@@ -60,6 +60,8 @@ def load():
         lib.isam_gemm_grouped.argtypes = [i, P, P, P, P, P, P, P, P, P, P]
         lib.isam_gemm_fp8.argtypes = [i, i, i, f, P, P, f, P]
         lib.isam_gemm_grouped_fp8.argtypes = [i, P, P, P, P, P, P, P, P]
+        lib.isam_gemm_mxfp8.argtypes = [i, i, i, f, P, P, P, P, f, P]
+        lib.isam_gemm_grouped_mxfp8.argtypes = [i, P, P, P, P, P, P, P, P, P, P]
         lib.isam_gru_forward.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_gru_forward_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
@@ -71,6 +73,7 @@ def load():
         lib.isam_gru_plan_for.argtypes = [i, i, i, i, i, i, P]
         for name in ("isam_version", "isam_set_stream", "isam_sync", "isam_shutdown", "isam_gemm",
                      "isam_gemm_plan_info", "isam_gemm_plan_info2", "isam_gemm_grouped", "isam_gemm_fp8", "isam_gemm_grouped_fp8",
+                     "isam_gemm_mxfp8", "isam_gemm_grouped_mxfp8",
                      "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_gru_forward_stack",
                      "isam_dwsep_conv", "isam_dwsep_plan_info", "isam_dwsep_plan_for",
@@ -144,6 +147,58 @@ def gemm_fp8(M, N, K, alpha, A, B, beta, C) -> None:
     _dev(C, torch.float32, M * N, "C")
     _use_current_stream(lib)
     check(lib.isam_gemm_fp8(M, N, K, float(alpha), _ptr(A), _ptr(B), float(beta), _ptr(C)))
+
+
+def _e4m3_dev(t, n, name):
+    import torch
+    if t.dtype not in (torch.uint8, getattr(torch, "float8_e4m3fn", torch.uint8)):
+        raise ValueError(f"{name} must hold E4M3 bytes (uint8 or float8_e4m3fn), got {t.dtype}")
+    _dev(t, t.dtype, n, name)
+
+
+def gemm_mxfp8(M, N, K, alpha, A, SA, B, SB, beta, C) -> None:
+    """isam_gemm_mxfp8: C = alpha (SA o A)(SB o B)^T + beta C with A (M x K) and
+    B (N x K) E4M3 bytes, SA [M, ceil(K/32)] and SB [N, ceil(K/32)] E8M0 bytes
+    (torch.uint8), C fp32."""
+    import torch
+    lib = load()
+    kb = (K + 31) // 32
+    _e4m3_dev(A, M * K, "A")
+    _e4m3_dev(B, N * K, "B")
+    _dev(SA, torch.uint8, M * kb, "SA")
+    _dev(SB, torch.uint8, N * kb, "SB")
+    _dev(C, torch.float32, M * N, "C")
+    _use_current_stream(lib)
+    check(lib.isam_gemm_mxfp8(M, N, K, float(alpha), _ptr(A), _ptr(SA), _ptr(B), _ptr(SB), float(beta), _ptr(C)))
+
+
+class GroupedGemmMxfp8:
+    """Marshalled arguments of one isam_gemm_grouped_mxfp8 call over a list of
+    (M, N, K, alpha, A, SA, B, SB, beta, C)."""
+
+    def __init__(self, problems):
+        import torch
+        n = len(problems)
+        ia = lambda vals: (ctypes.c_int * n)(*vals)
+        fa = lambda vals: (ctypes.c_float * n)(*vals)
+        pa = lambda vals: (ctypes.c_void_p * n)(*vals)
+        for (M, N, K, alpha, A, SA, B, SB, beta, C) in problems:
+            kb = (K + 31) // 32
+            _e4m3_dev(A, M * K, "A")
+            _e4m3_dev(B, N * K, "B")
+            _dev(SA, torch.uint8, M * kb, "SA")
+            _dev(SB, torch.uint8, N * kb, "SB")
+            _dev(C, torch.float32, M * N, "C")
+        cols = list(zip(*problems))
+        self.n = n
+        ptrs = lambda col: pa([t.data_ptr() for t in col])
+        self.args = (ia(cols[0]), ia(cols[1]), ia(cols[2]), fa(cols[3]), ptrs(cols[4]), ptrs(cols[5]),
+                     ptrs(cols[6]), ptrs(cols[7]), fa(cols[8]), ptrs(cols[9]))
+
+    def __call__(self):
+        lib = load()
+        _use_current_stream(lib)
+        check(lib.isam_gemm_grouped_mxfp8(self.n, *self.args))
 
 
 class GroupedGemm:
