@@ -49,14 +49,23 @@ METRIC = "GEMM TFLOP/s (tall-skinny sweep) and GRU timesteps/s on 1 GB300; % of 
 WORKLOAD = ("tall-skinny GEMM sweep: (M,K) in {(1760,1760),(2560,2560),(4096,4096),(7680,2560)} "
             "x N in {16,32,64,128} x {NN,TN}; bf16 U[-1,1]; fp32 accumulate/output; beta=0")
 # dram__bytes_read.sum + dram__bytes_write.sum of one gemm_group_kernel launch
-# over the sweep, from an ncu capture of the current kernel; None until one is
-# taken (profiles/gemm_group_kernel_skinny_sweep.md holds 749125376 + 26610176
-# bytes, captured before the kernel gained its per-problem E4M3 path).
-TRAFFIC_PER_STEP = None
+# over the sweep (750249984 + 24287232 bytes), from an ncu capture of the kernel
+# with 256-row tiles for the heavy problems; None whenever the kernel changes
+# until the counters are taken again.
+TRAFFIC_PER_STEP = 774537216
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
 # --------------------------------------------------------------------------- host logic
+def sweep_config(world: int) -> dict:
+    """The workload description both arms print (identical keys and values)."""
+    bytes_step = sum(gemm_bytes(M, N, K) for (M, N, K, _t) in sweep_problems())
+    return {"workload": WORKLOAD, "gemms_per_step": 32,
+            "l2": "inputs larger than L2: each GEMM has its own operands, "
+                  f"{bytes_step / 1e9:.2f} GB per step",
+            "parallelism": f"replica x{world}"}
+
+
 def sweep_problems():
     """(M, N, K, transA) of the 32 GEMMs of one step, in launch order."""
     return [(M, N, K, tA) for tA in (0, 1) for (M, K) in SWEEP_MK for N in SWEEP_N]
@@ -117,7 +126,7 @@ def row_sample(M: int, stride: int):
 
 # --------------------------------------------------------------------------- clocks
 class ClockSampler:
-    """nvidia-smi sampled every 20 ms in the background."""
+    """nvidia-smi sampled every 5 ms in the background."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -133,7 +142,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "20"],
+                 "--format=csv,noheader,nounits", "-lms", "5"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
@@ -370,18 +379,75 @@ def time_call(fn, reps, warmup, flush=None):
     return statistics.median(ts)
 
 
+def per_shape_table(isam, dev, peaks, fp8=False):
+    """Each sweep shape through the per-call API (isam_gemm, or isam_gemm_fp8
+    on E4M3 operands for the 16 K-major shapes): a CUDA graph of back-to-back
+    calls, each on its own operand set, with enough sets that a replay moves
+    at least 256 MB (twice L2), so every call reads its operands from HBM.
+    Returns one row per shape: kernel time per call (CUDA events over the
+    replays / calls), GB/s and the fraction of the measured HBM peak."""
+    import torch
+    from paper_1810_09958_gb300 import synth
+    rows = []
+    shapes = ([(M, N, K, 0) for (M, K) in SWEEP_MK for N in SWEEP_N] if fp8 else sweep_problems())
+    for (M, N, K, tA) in shapes:
+        by = (M * K + N * K + 4 * M * N) if fp8 else gemm_bytes(M, N, K)
+        sets = max(2, min(64, int(256e6 // by) + 1))
+        ops = []
+        for i in range(sets):
+            seed = synth.stream_seed(synth.BASE_SEED, 9, M, K, N, tA, i)
+            if fp8:
+                A = synth.e4m3_uniform_torch(synth.stream_seed(seed, 1), M * K, dev)
+                B = synth.e4m3_uniform_torch(synth.stream_seed(seed, 2), N * K, dev)
+            else:
+                A = synth.bf16_uniform_torch(synth.stream_seed(seed, 1), M * K, dev)
+                B = synth.bf16_uniform_torch(synth.stream_seed(seed, 2), K * N, dev)
+            ops.append((A, B, torch.empty(M * N, dtype=torch.float32, device=dev)))
+        if fp8:
+            run = lambda: [isam.gemm_fp8(M, N, K, 1.0, A, B, 0.0, C) for (A, B, C) in ops]
+        else:
+            run = lambda: [isam.gemm(M, N, K, tA, 0, 1.0, A, B, 0.0, C) for (A, B, C) in ops]
+        for _ in range(2):
+            run()
+        isam.sync()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            run()
+        ms = time_call(g.replay, reps=10, warmup=3) / sets
+        del g, ops
+        gbs = by / ms / 1e6
+        plan = isam.gemm_plan(M, N, K, tA, 0, 0.0) if not fp8 else None
+        row = {"M": M, "N": N, "K": K, "layout": "TN" if tA else "NN", "us": round(ms * 1e3, 3),
+               "gbs": round(gbs, 1), "frac_hbm": round(gbs / peaks["hbm_gbs"], 4),
+               "roofline_us": round(by / peaks["hbm_gbs"] / 1e3, 3)}
+        if plan:
+            row["plan"] = {k: plan[k] for k in ("BN", "split", "grid", "stages")}
+        rows.append(row)
+    torch.cuda.empty_cache()
+    return rows
+
+
 def hot_path_rows(isam, dev, peaks):
     """The remaining rows of the hot path, each timed on its benchmark shape."""
     import torch
     from paper_1810_09958_gb300 import synth
     out = {}
+    windows = {}
+
+    def timed(name, fn, **kw):
+        # time_call, with the wall-clock window of its timed calls kept for
+        # the row's clock summary
+        t0 = time.time()
+        ms = time_call(fn, **kw)
+        windows[name] = (t0, time.time())
+        return ms
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)  # 256 MB > L2
     # 8192^3, beta = 1, N(0,1)*0.02 operands, C U[-1,1].
     n = 8192
     A = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 2, 1), n * n, dev, 0.0, 0.02)
     B = synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 2, 2), n * n, dev, 0.0, 0.02)
     C = synth.f32_uniform_torch(synth.stream_seed(synth.BASE_SEED, 2, 3), n * n, dev)
-    ms = time_call(lambda: isam.gemm(n, n, n, 0, 0, 1.0, A, B, 1.0, C), reps=10, warmup=3)
+    ms = timed("gemm_8192_beta1", lambda: isam.gemm(n, n, n, 0, 0, 1.0, A, B, 1.0, C), reps=10, warmup=3)
     tf = gemm_flops(n, n, n) / ms / 1e9
     out["gemm_8192_beta1"] = {"ms": round(ms, 4), "tflops": round(tf, 1),
                               "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4),
@@ -404,7 +470,7 @@ def hot_path_rows(isam, dev, peaks):
     g8 = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g8):
         run_f8()
-    ms = time_call(g8.replay, reps=50, warmup=3) / 1.0
+    ms = timed("gemm_fp8_sweep_16", g8.replay, reps=50, warmup=3) / 1.0
     fl = sum(gemm_flops(M, N_, K) for (M, N_, K, *_r) in f8)
     by = sum(M * K + N_ * K + 4 * M * N_ for (M, N_, K, *_r) in f8)
     out["gemm_fp8_sweep_16"] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
@@ -419,12 +485,37 @@ def hot_path_rows(isam, dev, peaks):
     gg = torch.cuda.CUDAGraph()
     with torch.cuda.graph(gg):
         gcall()
-    ms = time_call(gg.replay, reps=50, warmup=3)
+    ms = timed("gemm_fp8_grouped_16", gg.replay, reps=50, warmup=3)
     out["gemm_fp8_grouped_16"] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
                                   "gbs": round(by / ms / 1e6, 1),
                                   "frac_hbm": round(by / ms / 1e6 / peaks["hbm_gbs"], 4),
                                   "what": "the same 16 E4M3 problems in one isam_gemm_grouped_fp8 launch"}
-    del f8, g8, gg, gcall
+    # The same 16 shapes as block-scaled (MX) E4M3: one E8M0 scale per 32 K
+    # elements of every row of A and B, one isam_gemm_grouped_mxfp8 launch.
+    mx = []
+    for (M, N_, K, A_, B_, C_) in f8:
+        kb = (K + 31) // 32
+        seed = synth.stream_seed(synth.BASE_SEED, 8, M, K, N_)
+        SA = torch.randint(120, 135, (M * kb,), dtype=torch.uint8, device=dev,
+                           generator=torch.Generator(device=dev).manual_seed(seed & 0x7FFFFFFF))
+        SB = torch.randint(120, 135, (N_ * kb,), dtype=torch.uint8, device=dev,
+                           generator=torch.Generator(device=dev).manual_seed((seed >> 1) & 0x7FFFFFFF))
+        mx.append((M, N_, K, 1.0, A_, SA, B_, SB, 0.0, C_))
+    mcall = isam.GroupedGemmMxfp8(mx)
+    for _ in range(3):
+        mcall()
+    isam.sync()
+    gm = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gm):
+        mcall()
+    ms = timed("gemm_mx_grouped_16", gm.replay, reps=50, warmup=3)
+    bym = sum(M * K + N_ * K + (M + N_) * ((K + 31) // 32) + 4 * M * N_ for (M, N_, K, *_r) in mx)
+    out["gemm_mx_grouped_16"] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
+                                 "gbs": round(bym / ms / 1e6, 1),
+                                 "frac_hbm": round(bym / ms / 1e6 / peaks["hbm_gbs"], 4),
+                                 "what": "the 16 problems as block-scaled E4M3 (E8M0 scale per 32 K elements "
+                                         "of each row of A and B) in one isam_gemm_grouped_mxfp8 launch"}
+    del f8, g8, gg, gcall, mx, gm, mcall
     # GRU: hidden = input = 1024, batch 32, T = 128.
     T, batch, H = 128, 32, 1024
     s = 1.0 / 32.0
@@ -434,7 +525,7 @@ def hot_path_rows(isam, dev, peaks):
     b = synth.f32_uniform_torch(synth.stream_seed(synth.BASE_SEED, 3, 4), 6 * H, dev, -0.1, 0.1)
     h0 = torch.zeros(batch * H, dtype=torch.float32, device=dev)
     hout = torch.empty(T * batch * H, dtype=torch.float32, device=dev)
-    ms = time_call(lambda: isam.gru_forward(T, batch, H, x, W, U, b, h0, hout), reps=10, warmup=3,
+    ms = timed("gru_h1024_b32_t128", lambda: isam.gru_forward(T, batch, H, x, W, U, b, h0, hout), reps=10, warmup=3,
                    flush=flush)
     gflop = 2.0 * T * batch * 3 * H * (H + H) / 1e9
     tf = gflop / ms
@@ -443,7 +534,7 @@ def hot_path_rows(isam, dev, peaks):
                                  "frac_bf16_burst": round(tf / peaks["bf16_tflops"], 4)}
     # The same GRU with the reset gate applied before the candidate's product
     # (two exchange rounds per step).
-    ms = time_call(lambda: isam.gru_forward(T, batch, H, x, W, U, b, h0, hout, reset_before=True),
+    ms = timed("gru_reset_before_h1024_b32_t128", lambda: isam.gru_forward(T, batch, H, x, W, U, b, h0, hout, reset_before=True),
                    reps=10, warmup=3, flush=flush)
     tf = gflop / ms
     out["gru_reset_before_h1024_b32_t128"] = {
@@ -460,7 +551,7 @@ def hot_path_rows(isam, dev, peaks):
     U = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 5, 3), L * 3 * H * H, dev, -s, s)
     b = synth.f32_uniform_torch(synth.stream_seed(synth.BASE_SEED, 5, 4), L * 6 * H, dev, -0.1, 0.1)
     hout = torch.empty(L * T * batch * H, dtype=torch.float32, device=dev)
-    ms = time_call(lambda: isam.gru_forward_stack(L, T, batch, H, x, W, U, b, None, hout), reps=10,
+    ms = timed("gru_stack2_h1024_b32_t128", lambda: isam.gru_forward_stack(L, T, batch, H, x, W, U, b, None, hout), reps=10,
                    warmup=3, flush=flush)
     seq = T * batch * H
     x1 = torch.empty(seq, dtype=torch.bfloat16, device=dev)
@@ -469,7 +560,7 @@ def hot_path_rows(isam, dev, peaks):
         isam.gru_forward(T, batch, H, x, W[:3 * H * H], U[:3 * H * H], b[:6 * H], None, hout[:seq])
         x1.copy_(hout[:seq])
         isam.gru_forward(T, batch, H, x1, W[3 * H * H:], U[3 * H * H:], b[6 * H:], None, hout[seq:])
-    ms_pl = time_call(per_layer, reps=10, warmup=3, flush=flush)
+    ms_pl = timed("gru_stack2_per_layer", per_layer, reps=10, warmup=3, flush=flush)
     out["gru_stack2_h1024_b32_t128"] = {
         "ms": round(ms, 4), "layer_timesteps_per_s": round(L * T / (ms / 1e3), 1),
         "us_per_layer_step": round(ms * 1e3 / (L * T), 3),
@@ -484,7 +575,7 @@ def hot_path_rows(isam, dev, peaks):
     pw = synth.bf16_uniform_torch(synth.stream_seed(synth.BASE_SEED, 4, 3), Cin * Cout, dev,
                                   -Cin ** -0.5, Cin ** -0.5)
     od = torch.empty(N * Hh * Ww * Cout, dtype=torch.float32, device=dev)
-    ms = time_call(lambda: isam.dwsep_conv(N, Hh, Ww, Cin, Cout, xd, dw, pw, od), reps=20, warmup=3,
+    ms = timed("dwsep_32x56x56_128_256", lambda: isam.dwsep_conv(N, Hh, Ww, Cin, Cout, xd, dw, pw, od), reps=20, warmup=3,
                    flush=flush)
     byts = N * Hh * Ww * (Cin * 2 + Cout * 4) + 9 * Cin * 2 + Cin * Cout * 2
     gbs = byts / ms / 1e6
@@ -492,7 +583,7 @@ def hot_path_rows(isam, dev, peaks):
                                      "frac_hbm": round(gbs / peaks["hbm_gbs"], 4),
                                      "tflops": round(2.0 * N * Hh * Ww * Cin * (9 + Cout) / ms / 1e9, 2)}
     isam.sync()
-    return out
+    return out, windows
 
 
 # --------------------------------------------------------------------------- CPU (oracle) arm
@@ -584,7 +675,8 @@ def reference_arm(args):
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_all / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": WORKLOAD, "gemms_per_step": 32},
+            "data": "synthetic", "config": sweep_config(world),
+            "api": "the fp64 oracle (oracle_gemm) on a row sample of each sweep GEMM",
             "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": oracle.num_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -742,16 +834,26 @@ def main(argv=None):
     call_ms = reduce_max(call_ms, dev)
     call_value = whole_job_tflops(flops_step, args.steps, world, call_ms)
 
-    e2e_steps = max(3, args.steps // 20)
+    e2e_steps = max(20, args.steps // 20)
     e2e_ms, h2d, d2h = time_e2e(isam, probs, e2e_steps, args.warmup)
     e2e_ms = reduce_max(e2e_ms, dev)
     e2e_value = whole_job_tflops(flops_step, e2e_steps, world, e2e_ms)
 
-    hot = None
+    hot, hot_windows = None, {}
     if not args.no_hot_path:
-        hot = hot_path_rows(isam, dev, peaks)
+        hot, hot_windows = hot_path_rows(isam, dev, peaks)
+        t0 = time.time()
+        shape_rows = per_shape_table(isam, dev, peaks)
+        shape_rows_f8 = per_shape_table(isam, dev, peaks, fp8=True)
+        hot_windows["per_shape"] = (t0, time.time())
     if sampler:
         sampler.stop()
+        if hot is not None:
+            for name, win in hot_windows.items():
+                if name in hot:
+                    hot[name]["clocks"] = sampler.summary(*win)
+            hot["gru_stack2_h1024_b32_t128"]["per_layer_clocks"] = sampler.summary(
+                *hot_windows["gru_stack2_per_layer"])
     del probs
     torch.cuda.empty_cache()
 
@@ -763,11 +865,8 @@ def main(argv=None):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "gemms_per_step": 32,
-                       "api": "isam_gemm_grouped: the 32 GEMMs of a step in one call",
-                       "l2": "inputs larger than L2: each GEMM has its own operands, "
-                             f"{bytes_step / 1e9:.2f} GB per step",
-                       "parallelism": f"replica x{world}"},
+            "config": sweep_config(world),
+            "api": "isam_gemm_grouped: the 32 GEMMs of a step in one call",
             "roofline": {"kernel": "gemm_group_kernel", "bound": "hbm", "achieved": round(achieved, 1),
                          "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": round(achieved / peaks["hbm_gbs"], 4), "traffic": TRAFFIC_PER_STEP,
@@ -790,6 +889,11 @@ def main(argv=None):
         }
         if hot is not None:
             line["hot_path"] = hot
+            line["per_shape"] = {
+                "what": "each sweep shape alone through the per-call API, back-to-back calls on "
+                        "their own operand sets (>= 256 MB per replay), CUDA-event time per call",
+                "clocks": sampler.summary(*hot_windows["per_shape"]) if sampler else None,
+                "isam_gemm": shape_rows, "isam_gemm_fp8": shape_rows_f8}
         if not args.no_cpu_baseline and world == 1:
             import oracle
             oracle.build()
