@@ -494,11 +494,10 @@ def hot_path_rows(isam, dev, peaks):
     # elements of every row of A and B, one isam_gemm_grouped_mxfp8 launch.
     mx = []
     for (M, N_, K, A_, B_, C_) in f8:
-        kb = (K + 31) // 32
         seed = synth.stream_seed(synth.BASE_SEED, 8, M, K, N_)
-        SA = torch.randint(120, 135, (M * kb,), dtype=torch.uint8, device=dev,
+        SA = torch.randint(120, 135, (isam.mx_scale_bytes(M, K),), dtype=torch.uint8, device=dev,
                            generator=torch.Generator(device=dev).manual_seed(seed & 0x7FFFFFFF))
-        SB = torch.randint(120, 135, (N_ * kb,), dtype=torch.uint8, device=dev,
+        SB = torch.randint(120, 135, (isam.mx_scale_bytes(N_, K),), dtype=torch.uint8, device=dev,
                            generator=torch.Generator(device=dev).manual_seed((seed >> 1) & 0x7FFFFFFF))
         mx.append((M, N_, K, 1.0, A_, SA, B_, SB, 0.0, C_))
     mcall = isam.GroupedGemmMxfp8(mx)
@@ -509,7 +508,7 @@ def hot_path_rows(isam, dev, peaks):
     with torch.cuda.graph(gm):
         mcall()
     ms = timed("gemm_mx_grouped_16", gm.replay, reps=50, warmup=3)
-    bym = sum(M * K + N_ * K + (M + N_) * ((K + 31) // 32) + 4 * M * N_ for (M, N_, K, *_r) in mx)
+    bym = sum(M * K + N_ * K + isam.mx_scale_bytes(M + N_, K) + 4 * M * N_ for (M, N_, K, *_r) in mx)
     out["gemm_mx_grouped_16"] = {"ms": round(ms, 4), "tflops": round(fl / ms / 1e9, 1),
                                  "gbs": round(bym / ms / 1e6, 1),
                                  "frac_hbm": round(bym / ms / 1e6 / peaks["hbm_gbs"], 4),
@@ -687,7 +686,8 @@ def reference_arm(args):
 # --------------------------------------------------------------------------- single case
 def run_case(args):
     """Times one hot-path call on its own (for profiling and sweeps):
-    sweep (the 32 sweep GEMMs in one grouped call) | gemm:M,N,K,transA,transB,beta |
+    sweep (the 32 sweep GEMMs in one grouped call) | fp8 | mx (the 16 K-major sweep shapes as
+    E4M3 / block-scaled E4M3 in one grouped call) | gemm:M,N,K,transA,transB,beta |
     gru[:T,batch,hidden] | gru_rb[:T,batch,hidden] (reset gate before the candidate's
     product) | gru_stack[:L,T,batch,hidden] | gru_stack_rb[:...] | gru_layers[:...] (the
     stack as one call per layer) | dwsep[:N,H,W,Cin,Cout]."""
@@ -717,6 +717,27 @@ def run_case(args):
         fn = call
         work = {"tflops": sum(p["flops"] for p in probs) / 1e12,
                 "gb": sum(p["bytes"] for p in probs) / 1e9}
+    elif kind in ("fp8", "mx"):
+        # the 16 K-major sweep shapes on E4M3 operands in one grouped call;
+        # "mx" adds one E8M0 scale per 32 K elements of each row of A and B
+        probs = []
+        by = 0
+        for (M, K) in SWEEP_MK:
+            for N_ in SWEEP_N:
+                seed = synth.stream_seed(synth.BASE_SEED, 7, M, K, N_)
+                A_ = synth.e4m3_uniform_torch(synth.stream_seed(seed, 1), M * K, dev)
+                B_ = synth.e4m3_uniform_torch(synth.stream_seed(seed, 2), N_ * K, dev)
+                C_ = torch.empty(M * N_, dtype=torch.float32, device=dev)
+                if kind == "mx":
+                    SA = torch.full((isam.mx_scale_bytes(M, K),), 127, dtype=torch.uint8, device=dev)
+                    SB = torch.full((isam.mx_scale_bytes(N_, K),), 127, dtype=torch.uint8, device=dev)
+                    probs.append((M, N_, K, 1.0, A_, SA, B_, SB, 0.0, C_))
+                    by += M * K + N_ * K + isam.mx_scale_bytes(M + N_, K) + 4 * M * N_
+                else:
+                    probs.append((M, N_, K, 1.0, A_, B_, 0.0, C_))
+                    by += M * K + N_ * K + 4 * M * N_
+        fn = isam.GroupedGemmMxfp8(probs) if kind == "mx" else isam.GroupedGemmFp8(probs)
+        work = {"tflops": sum(2.0 * q[0] * q[1] * q[2] for q in probs) / 1e12, "gb": by / 1e9}
     elif kind in ("gru", "gru_rb"):
         T, batch, H = (int(v) for v in vals) if vals else (128, 32, 1024)
         s = H ** -0.5

@@ -117,16 +117,22 @@ int isam_gemm_fp8(int M, int N, int K, float alpha, const uint8_t *A, const uint
  * Block-scaled E4M3 GEMM in the OCP Microscaling (MX) form: every 32
  * consecutive K elements of a row of A, and of a row of B, share one E8M0
  * scale byte e meaning 2^(e - 127) (e = 255 is NaN):
- *   C[i][j] <- alpha * sum_k (2^(SA[i][k/32]-127) A[i][k]) (2^(SB[j][k/32]-127) B[j][k])
- *              + beta * C[i][j].
+ *   C[i][j] <- alpha * sum_k (2^(sa(i,k)-127) A[i][k]) (2^(sb(j,k)-127) B[j][k])
+ *              + beta * C[i][j],
+ * sa(i, k), sb(j, k) the scale bytes of the 32-element K block holding k.
  * The paper's instruction selection (Section 2.4) picks the instruction whose
  * semantics cover the computation; here the tensor cores' block-scaled
  * operand kind applies the scales inside the product.
  *   A  M x K, B  N x K: E4M3 bytes, row-major (K-major), device pointers,
  *      16-byte aligned; K a multiple of 16 (16-byte rows).
- *   SA [M][ceil(K/32)], SB [N][ceil(K/32)]: E8M0 bytes, row-major, device
- *      pointers, any alignment.  A last block shorter than 32 (K % 32 != 0)
- *      has a scale of its own.
+ *   SA, SB: the E8M0 bytes, device pointers, 4-byte aligned, atom-major:
+ *      for each 128-element K atom a (ceil(K/128) of them) and each row,
+ *      four consecutive bytes, byte t the scale of K block 4a + t of that
+ *      row: SA[((a * M) + i) * 4 + t] scales A[i][k] for k in
+ *      [128a + 32t, 128a + 32t + 32), and SB likewise with N rows.  Bytes of
+ *      blocks past ceil(K/32) are ignored.  A last block shorter than 32
+ *      (K % 32 != 0) has a scale of its own.  (This layout puts the words one
+ *      K atom needs for consecutive rows next to each other.)
  *   C  M x N fp32 row-major, 16-byte aligned; beta == 0 does not read C.
  * Products of the scaled operands are exact and accumulate in fp32.  One
  * persistent launch over 128 x min(128, N rounded up to 16) tiles (no

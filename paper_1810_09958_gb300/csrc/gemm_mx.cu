@@ -25,6 +25,12 @@
 // own lanes.  For A, column 0 holds row m at lane m and columns 1..3 hold row
 // r + 32j at lane 32q + r, which serves a quarter reading either its own rows
 // at column 0 or column q.
+//
+// Scale bytes are taken atom-major: SA [ceil(K/128)][M][4], SB
+// [ceil(K/128)][N][4], the four E8M0 bytes of a row for one 128-element K
+// atom forming one 32-bit word (byte t = the atom's t-th 32-element block).
+// The words of one atom for consecutive rows are consecutive, so the scale
+// warps read them with coalesced 4-byte loads, one load per TMEM cell.
 #include <algorithm>
 #include <cstdio>
 #include <cstring>
@@ -65,14 +71,14 @@ enum : uint32_t {
 struct MxProblem {
     int M, N, K;
     int m_tiles, n_tiles, kb_total;  // kb_total: 128-element K atoms
-    int nblk;                        // scale bytes per row: ceil(K / 32)
+    int nblk;                        // 32-element K blocks: ceil(K / 32)
     int bn;
     int tma_c;                       // C rows 16-byte aligned: TMA epilogue
     int tile_start;
     float alpha, beta;
     float *C;
-    const uint8_t *SA;               // [M][nblk]
-    const uint8_t *SB;               // [N][nblk]
+    const uint32_t *SA;              // [ceil(K/128)][M] words of 4 scale bytes
+    const uint32_t *SB;              // [ceil(K/128)][N]
 };
 
 struct MxParams {
@@ -91,23 +97,22 @@ __device__ __forceinline__ int mx_find_problem(const MxParams &p, int tile, int 
     return i;
 }
 
-// Four scale bytes of `row` for K blocks 4*atom .. 4*atom + 3 packed into one
-// word (byte t = block 4*atom + t); rows past the matrix and blocks past K
-// read as 127 (a scale of 1: the operands there are zero-filled).
-__device__ __forceinline__ uint32_t load_scales4(const uint8_t *S, int rows, int nblk, int row, int atom) {
-    uint32_t v = 0x7F7F7F7Fu;
-    if (row < rows) {
-        const uint8_t *p = S + static_cast<size_t>(row) * nblk;
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-            const int b = atom * 4 + t;
-            if (b < nblk) {
-                const uint32_t e = __ldg(p + b);
-                v = (v & ~(0xFFu << (8 * t))) | (e << (8 * t));
-            }
-        }
-    }
-    return v;
+// The scale word of `row` for K atom `atom`, loaded into v only when the row
+// exists (v keeps 0x7F7F7F7F, a scale of 1 on zero-filled operands,
+// otherwise).  Nothing reads v here, so the load stays in flight while the
+// warp goes on; mask_past_k applies the last atom's mask where v is used.
+__device__ __forceinline__ void load_scale_word(uint32_t &v, const uint32_t *S, int rows, int row, int atom) {
+    v = 0x7F7F7F7Fu;
+    if (row < rows) v = __ldg(S + static_cast<size_t>(atom) * rows + row);
+}
+
+// The bytes of the last atom's blocks past K read as 127, whatever the caller
+// stored there.
+__device__ __forceinline__ uint32_t mask_past_k(uint32_t v, int nblk, int atom) {
+    const int past = 4 * atom + 4 - nblk;  // 0..3 on the last atom
+    if (past <= 0) return v;
+    const uint32_t keep = 0xFFFFFFFFu >> (8 * past);
+    return (v & keep) | (0x7F7F7F7Fu & ~keep);
 }
 
 __global__ void __launch_bounds__(kThreads, 1) gemm_mx_kernel(const __grid_constant__ MxParams p) {
@@ -267,34 +272,53 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_mx_kernel(const __grid_const
             const int local = tile - pr.tile_start;
             const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
             const int m0 = mt * kBM, n0 = nt * pr.bn;
-            for (int kb = 0; kb < pr.kb_total; ++kb) {
-                // The loads are issued before the wait for the slot, so their
-                // latency overlaps it.
-                uint32_t va[4], vb[4];
-                va[0] = load_scales4(pr.SA, pr.M, pr.nblk, m0 + q * 32 + lane, kb);
+            // Scale words of K atom kb: this lane's rows of A (column 0: row
+            // 32q + lane; columns 1..3: row lane + 32j) and of B (row lane + 32j).
+            auto load_atom = [&](int kb, uint32_t (&va)[4], uint32_t (&vb)[4]) {
+                load_scale_word(va[0], pr.SA, pr.M, m0 + q * 32 + lane, kb);
 #pragma unroll
-                for (int j = 1; j < 4; ++j) va[j] = load_scales4(pr.SA, pr.M, pr.nblk, m0 + lane + 32 * j, kb);
+                for (int j = 1; j < 4; ++j) load_scale_word(va[j], pr.SA, pr.M, m0 + lane + 32 * j, kb);
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const int n = lane + 32 * j;
-                    vb[j] = n < pr.bn ? load_scales4(pr.SB, pr.N, pr.nblk, n0 + n, kb) : 0x7F7F7F7Fu;
-                }
-                if (!warp_wait(&sempty[slot], sphase ^ 1u, w, SITE_X_SEMPTY)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t col = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + kSfCol0 +
-                                     static_cast<uint32_t>(slot * 8);
-                tmem_st4(col, va);
-                tmem_st4(col + 4, vb);
-                tmem_st_wait();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&sfull[slot]);
-                if (++slot == kSfSlots) {
-                    slot = 0;
-                    sphase ^= 1u;
+                for (int j = 0; j < 4; ++j)
+                    load_scale_word(vb[j], pr.SB, lane + 32 * j < pr.bn ? pr.N : 0, n0 + lane + 32 * j, kb);
+            };
+            // The loads run kPf atoms ahead of the stores (a register ring
+            // indexed at compile time), so their latency is paid once per tile.
+            constexpr int kPf = 4;
+            uint32_t pa[kPf][4], pb[kPf][4];
+#pragma unroll
+            for (int i = 0; i < kPf; ++i)
+                if (i < pr.kb_total) load_atom(i, pa[i], pb[i]);
+            for (int kb0 = 0; ok && kb0 < pr.kb_total; kb0 += kPf) {
+#pragma unroll
+                for (int i = 0; i < kPf; ++i) {
+                    const int kb = kb0 + i;
+                    if (kb >= pr.kb_total) break;
+                    if (!warp_wait(&sempty[slot], sphase ^ 1u, w, SITE_X_SEMPTY)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t col = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + kSfCol0 +
+                                         static_cast<uint32_t>(slot * 8);
+                    if (4 * kb + 4 > pr.nblk) {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            pa[i][j] = mask_past_k(pa[i][j], pr.nblk, kb);
+                            pb[i][j] = mask_past_k(pb[i][j], pr.nblk, kb);
+                        }
+                    }
+                    tmem_st4(col, pa[i]);
+                    tmem_st4(col + 4, pb[i]);
+                    tmem_st_wait();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&sfull[slot]);
+                    if (++slot == kSfSlots) {
+                        slot = 0;
+                        sphase ^= 1u;
+                    }
+                    if (kb + kPf < pr.kb_total) load_atom(kb + kPf, pa[i], pb[i]);
                 }
             }
         }
@@ -464,6 +488,8 @@ int gemm_mx_validate(const MxDesc &g) {
     if (g.K % 16 != 0)
         return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm_mxfp8: K (%d) must be a multiple of 16 (16-byte rows)",
                          g.K);
+    if ((reinterpret_cast<uintptr_t>(g.SA) | reinterpret_cast<uintptr_t>(g.SB)) & 3u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_gemm_mxfp8: SA and SB must be 4-byte aligned");
     return ISAM_OK;
 }
 
@@ -498,8 +524,8 @@ int gemm_mx_launch(int count, const MxDesc *g, DeviceState &ds, cudaStream_t str
         pr.alpha = d.alpha;
         pr.beta = d.beta;
         pr.C = d.C;
-        pr.SA = d.SA;
-        pr.SB = d.SB;
+        pr.SA = reinterpret_cast<const uint32_t *>(d.SA);
+        pr.SB = reinterpret_cast<const uint32_t *>(d.SB);
         tiles += pr.m_tiles * pr.n_tiles;
         int rc;
         if ((rc = make_tmap_2d_u8(&p.tmA[s], d.A, d.K, d.M, static_cast<uint64_t>(d.K), kAtom, kBM))) return rc;

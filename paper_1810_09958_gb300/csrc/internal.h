@@ -100,7 +100,8 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
 
 // Block-scaled E4M3 GEMM (OCP MX): C = alpha (SA o A)(SB o B)^T + beta C with
 // A M x K and B N x K E4M3 bytes (K-major) and one E8M0 scale byte per 32 K
-// elements of each row, SA [M][ceil(K/32)], SB [N][ceil(K/32)].
+// elements of each row, atom-major: SA [ceil(K/128)][M][4], SB
+// [ceil(K/128)][N][4] (4-byte aligned).
 struct MxDesc {
     int M, N, K;
     float alpha, beta;

@@ -156,17 +156,21 @@ def _e4m3_dev(t, n, name):
     _dev(t, t.dtype, n, name)
 
 
+def mx_scale_bytes(rows, K) -> int:
+    """Bytes of an atom-major scale array: ceil(K/128) x rows x 4."""
+    return (K + 127) // 128 * rows * 4
+
+
 def gemm_mxfp8(M, N, K, alpha, A, SA, B, SB, beta, C) -> None:
     """isam_gemm_mxfp8: C = alpha (SA o A)(SB o B)^T + beta C with A (M x K) and
-    B (N x K) E4M3 bytes, SA [M, ceil(K/32)] and SB [N, ceil(K/32)] E8M0 bytes
-    (torch.uint8), C fp32."""
+    B (N x K) E4M3 bytes, SA and SB E8M0 bytes (torch.uint8) in the atom-major
+    layout [ceil(K/128)][rows][4] (include/isam.h), C fp32."""
     import torch
     lib = load()
-    kb = (K + 31) // 32
     _e4m3_dev(A, M * K, "A")
     _e4m3_dev(B, N * K, "B")
-    _dev(SA, torch.uint8, M * kb, "SA")
-    _dev(SB, torch.uint8, N * kb, "SB")
+    _dev(SA, torch.uint8, mx_scale_bytes(M, K), "SA")
+    _dev(SB, torch.uint8, mx_scale_bytes(N, K), "SB")
     _dev(C, torch.float32, M * N, "C")
     _use_current_stream(lib)
     check(lib.isam_gemm_mxfp8(M, N, K, float(alpha), _ptr(A), _ptr(SA), _ptr(B), _ptr(SB), float(beta), _ptr(C)))
@@ -174,7 +178,7 @@ def gemm_mxfp8(M, N, K, alpha, A, SA, B, SB, beta, C) -> None:
 
 class GroupedGemmMxfp8:
     """Marshalled arguments of one isam_gemm_grouped_mxfp8 call over a list of
-    (M, N, K, alpha, A, SA, B, SB, beta, C)."""
+    (M, N, K, alpha, A, SA, B, SB, beta, C); SA, SB atom-major (mx_scale_bytes)."""
 
     def __init__(self, problems):
         import torch
@@ -183,11 +187,10 @@ class GroupedGemmMxfp8:
         fa = lambda vals: (ctypes.c_float * n)(*vals)
         pa = lambda vals: (ctypes.c_void_p * n)(*vals)
         for (M, N, K, alpha, A, SA, B, SB, beta, C) in problems:
-            kb = (K + 31) // 32
             _e4m3_dev(A, M * K, "A")
             _e4m3_dev(B, N * K, "B")
-            _dev(SA, torch.uint8, M * kb, "SA")
-            _dev(SB, torch.uint8, N * kb, "SB")
+            _dev(SA, torch.uint8, mx_scale_bytes(M, K), "SA")
+            _dev(SB, torch.uint8, mx_scale_bytes(N, K), "SB")
             _dev(C, torch.float32, M * N, "C")
         cols = list(zip(*problems))
         self.n = n

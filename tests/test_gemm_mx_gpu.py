@@ -1,5 +1,6 @@
 """isam_gemm_mxfp8 / isam_gemm_grouped_mxfp8 (block-scaled E4M3, one E8M0
-scale per 32 K elements) on the GPU against the fp64 oracle
+scale per 32 K elements, passed atom-major with NaN bytes in the padding past
+K, which the library must ignore) on the GPU against the fp64 oracle
 (oracle.gemm_mxfp8): unit scales reproduce the grouped E4M3 GEMM bit for bit;
 integer operands with power-of-two scales are exact; uniform operands with
 random scales are within the GEMM tolerance (5e-3)."""
@@ -30,6 +31,24 @@ def dev_u8(a):
     return torch.from_numpy(np.ascontiguousarray(a, dtype=np.uint8).reshape(-1)).to("cuda")
 
 
+def atom_major(S, K, pad=255):
+    """[rows][ceil(K/32)] scale bytes (the oracle's layout) rearranged into the
+    library's [ceil(K/128)][rows][4]; the bytes of blocks past ceil(K/32) are
+    `pad` (255 is an E8M0 NaN, which the library must ignore there)."""
+    rows, kb = S.shape
+    na = (K + 127) // 128
+    out = np.full((na, rows, 4), pad, np.uint8)
+    for a in range(na):
+        for t in range(4):
+            if 4 * a + t < kb:
+                out[a, :, t] = S[:, 4 * a + t]
+    return out
+
+
+def dev_scales(S, K):
+    return dev_u8(atom_major(S, K))
+
+
 def operands(M, N, K, seed, dist):
     kb = (K + 31) // 32
     if dist == "int":
@@ -49,7 +68,7 @@ def operands(M, N, K, seed, dist):
 
 def run_mx(M, N, K, alpha, beta, A, SA, B, SB, C0):
     out = Guarded(M * N, init=C0)
-    isam.gemm_mxfp8(M, N, K, alpha, dev_u8(A), dev_u8(SA), dev_u8(B), dev_u8(SB), beta, out.t)
+    isam.gemm_mxfp8(M, N, K, alpha, dev_u8(A), dev_scales(SA, K), dev_u8(B), dev_scales(SB, K), beta, out.t)
     isam.sync()
     assert out.guards_intact()
     return out.numpy().reshape(M, N)
@@ -131,7 +150,7 @@ def test_grouped_mixed_problems():
     for i, (M, N, K, alpha, beta) in enumerate(specs):
         A, SA, B, SB, C0 = operands(M, N, K, 3500 + 7 * i, "int")
         out = Guarded(M * N, init=C0)
-        probs.append((M, N, K, alpha, dev_u8(A), dev_u8(SA), dev_u8(B), dev_u8(SB), beta, out.t))
+        probs.append((M, N, K, alpha, dev_u8(A), dev_scales(SA, K), dev_u8(B), dev_scales(SB, K), beta, out.t))
         keep.append((A, SA, B, SB, C0, out))
     isam.GroupedGemmMxfp8(probs)()
     isam.sync()
@@ -152,3 +171,14 @@ def test_argument_errors():
     assert lib.isam_gemm_mxfp8(0, 8, 32, 1.0, p(z), p(z), p(z), p(z), 0.0, p(c)) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_gemm_mxfp8(8, 8, 32, 1.0, p(z), None, p(z), p(z), 0.0, p(c)) == isam.ISAM_ERR_INVALID_ARG
     assert lib.isam_gemm_mxfp8(8, 8, 32, 1.0, p(z[1:]), p(z), p(z), p(z), 0.0, p(c)) == isam.ISAM_ERR_UNSUPPORTED
+    # scale arrays hold 4-byte words
+    assert lib.isam_gemm_mxfp8(8, 8, 32, 1.0, p(z), p(z[2:]), p(z), p(z), 0.0, p(c)) == isam.ISAM_ERR_UNSUPPORTED
+
+
+def test_atom_major_layout_helper():
+    """The rearrangement the tests use: byte t of word (a, row) is block 4a + t."""
+    S = np.arange(3 * 5, dtype=np.uint8).reshape(3, 5)  # 3 rows, K = 160 -> 5 blocks, 2 atoms
+    out = atom_major(S, 160)
+    assert out.shape == (2, 3, 4)
+    assert np.array_equal(out[0], S[:, 0:4]) and np.array_equal(out[1, :, 0], S[:, 4])
+    assert (out[1, :, 1:] == 255).all()
