@@ -581,6 +581,26 @@ def hot_path_rows(isam, dev, peaks):
     out["dwsep_32x56x56_128_256"] = {"ms": round(ms, 4), "gbs": round(gbs, 1),
                                      "frac_hbm": round(gbs / peaks["hbm_gbs"], 4),
                                      "tflops": round(2.0 * N * Hh * Ww * Cin * (9 + Cout) / ms / 1e9, 2)}
+    # The same layer unfused: the depthwise factor to memory (bf16), then the
+    # pointwise factor through isam_gemm (M = N*H*W, N = Cout, K = Cin).
+    M = N * Hh * Ww
+    yb = torch.empty(M * Cin, dtype=torch.bfloat16, device=dev)
+    ms_dw = timed("dwsep_unfused_depthwise", lambda: isam.depthwise_conv3x3(N, Hh, Ww, Cin, xd, dw, yb), reps=20,
+                  warmup=3, flush=flush)
+    ms_pw = timed("dwsep_unfused_pointwise", lambda: isam.gemm(M, Cout, Cin, 0, 0, 1.0, yb, pw, 0.0, od), reps=20,
+                  warmup=3, flush=flush)
+
+    def unfused():
+        isam.depthwise_conv3x3(N, Hh, Ww, Cin, xd, dw, yb)
+        isam.gemm(M, Cout, Cin, 0, 0, 1.0, yb, pw, 0.0, od)
+    ms_u = timed("dwsep_unfused_32x56x56_128_256", unfused, reps=20, warmup=3, flush=flush)
+    bytes_u = byts + 2 * M * Cin * 2  # the intermediate written and read back
+    out["dwsep_unfused_32x56x56_128_256"] = {
+        "ms": round(ms_u, 4), "depthwise_ms": round(ms_dw, 4), "pointwise_ms": round(ms_pw, 4),
+        "gbs": round(bytes_u / ms_u / 1e6, 1), "frac_hbm": round(bytes_u / ms_u / 1e6 / peaks["hbm_gbs"], 4),
+        "layer_gbs": round(byts / ms_u / 1e6, 1),
+        "what": "isam_depthwise_conv3x3 (bf16 intermediate in HBM) then isam_gemm; gbs counts the intermediate's "
+                "round trip, layer_gbs the fused layer's algorithmic bytes"}
     isam.sync()
     return out, windows
 

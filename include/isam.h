@@ -376,6 +376,22 @@ int isam_dwsep_conv(int N, int H, int W, int Cin, int Cout, const isam_bf16 *x,
                     const isam_bf16 *dw_w, const isam_bf16 *pw_w, float *out);
 
 /*
+ * The first factor of Listing 3 alone: a 3x3 depthwise convolution over an
+ * NHWC tensor (stride 1, zero border of one pixel, channel multiplier 1),
+ *   y[n][i][j][c] = bf16( sum_{di,dj in 0..2} x[n][i+di-1][j+dj-1][c] * D[di][dj][c] ),
+ * summed in fp32 (taps in row-major order) and rounded once to bf16.
+ * Followed by isam_gemm(M = N*H*W, N = Cout, K = C, transA = 0, transB = 0,
+ * A = y, B = pw_w), it is the unfused schedule of the separable layer
+ * (Section 2.3), which writes the intermediate to memory; isam_dwsep_conv is
+ * the fused one.
+ *   x [N][H][W][C] bf16, dw_w [3][3][C] bf16, y [N][H][W][C] bf16; device
+ *   pointers, 16-byte aligned; C a multiple of 8.  Otherwise
+ *   ISAM_ERR_UNSUPPORTED; sizes < 1 or null pointers ISAM_ERR_INVALID_ARG.
+ */
+int isam_depthwise_conv3x3(int N, int H, int W, int C, const isam_bf16 *x, const isam_bf16 *dw_w,
+                           isam_bf16 *y);
+
+/*
  * The plan isam_dwsep_conv takes for an image W pixels wide with Cin -> Cout
  * channels (it does not depend on N or H); nothing is launched.  out[4]:
  *   out[0]  kernel: 0 = whole image rows per tile with an input-row ring in

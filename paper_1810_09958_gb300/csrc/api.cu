@@ -357,6 +357,21 @@ int isam_gemm_grouped_fp8(int count, const int *M, const int *N, const int *K, c
     return gemm_grouped_launch(count, g, *ds, current_stream());
 }
 
+int isam_depthwise_conv3x3(int N, int H, int W, int C, const isam_bf16 *x, const isam_bf16 *dw_w, isam_bf16 *y) {
+    if (N < 1 || H < 1 || W < 1 || C < 1)
+        return set_error(ISAM_ERR_INVALID_ARG, "isam_depthwise_conv3x3: sizes must be >= 1");
+    if (!x || !dw_w || !y) return set_error(ISAM_ERR_INVALID_ARG, "isam_depthwise_conv3x3: null pointer");
+    if (C % 8 != 0)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_depthwise_conv3x3: C (%d) must be a multiple of 8", C);
+    if ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(dw_w) | reinterpret_cast<uintptr_t>(y)) & 15u)
+        return set_error(ISAM_ERR_UNSUPPORTED, "isam_depthwise_conv3x3: pointers must be 16-byte aligned");
+    int rc;
+    DeviceState *ds = device_state(&rc);
+    if (!ds) return rc;
+    return depthwise_launch(N, H, W, C, reinterpret_cast<const uint16_t *>(x), reinterpret_cast<const uint16_t *>(dw_w),
+                            reinterpret_cast<uint16_t *>(y), *ds, current_stream());
+}
+
 int isam_gemm_mxfp8(int M, int N, int K, float alpha, const uint8_t *A, const uint8_t *SA, const uint8_t *B,
                     const uint8_t *SB, float beta, float *C) {
     MxDesc g{M, N, K, alpha, beta, A, SA, B, SB, C};

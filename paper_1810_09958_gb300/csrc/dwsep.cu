@@ -361,11 +361,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 // a shared-memory ring filled by one TMA copy per row.  Every input element
 // then leaves L2 about once per CTA, and the producers read the 3x3 taps from
 // shared memory.
-constexpr int kRProdWarps = 12;               // depthwise producer warps 0-11
+constexpr int kRProdWarps = 11;               // depthwise producer warps 0-10
 constexpr int kRProd = kRProdWarps * 32;
-constexpr int kRMmaWarp = kRProdWarps;         // warp 12: ring loader + MMA issuer
-constexpr int kREpiWarp0 = kRProdWarps + 1;    // warps 13-16: epilogue
-constexpr int kRThreads = (kRProdWarps + 5) * 32;
+constexpr int kRMmaWarp = kRProdWarps;         // warp 11: ring loader + MMA issuer
+constexpr int kREpiWarp0 = kRProdWarps + 1;    // warps 12-19: epilogue, two per TMEM lane quarter
+constexpr int kREpiWarps = 8;
+constexpr int kRThreads = (kRProdWarps + 1 + kREpiWarps) * 32;
 constexpr int kRingMax = 32;  // input rows resident per CTA: 2 * rt + 2 (this tile + halo + the next)
 
 enum : uint32_t { SITE_DW_RING = 0x306 };
@@ -487,7 +488,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         mbar_init(a_empty, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&tfull[i], 1);
-            mbar_init(&tempty[i], 4);
+            mbar_init(&tempty[i], kREpiWarps);
         }
         mbar_init(wbar, 1);
         *abort_flag = 0;
@@ -528,14 +529,17 @@ __global__ void __launch_bounds__(kRThreads, 1)
         // Tile, row and ring-slot positions advance incrementally: an integer
         // division by a run-time value costs hundreds of cycles of latency,
         // and here it would sit on the critical path of every tile.
-        const int groups = Cin / 4;  // divides kRProd (Cin is 16, 32, ..., 256)
+        const int groups = Cin / 4;  // at most 64 (Cin <= 256), fewer than kRProd
         const int g = tid % groups;
-        // Column segment of this thread: the kRProd / groups segments split
-        // the W columns evenly (lengths differ by at most one).
+        // Column segment of this thread: the kRProd / groups whole segments
+        // split the W columns evenly (lengths differ by at most one); threads
+        // past the last whole segment get an empty one (x from W to W: they
+        // read valid columns and store nothing) and only join the barriers.
         const int nseg = kRProd / groups;
         const int seg = tid / groups;
-        const int xs = (seg * W) / nseg;
-        const int xe = ((seg + 1) * W) / nseg;
+        const bool seg_live = seg < nseg;
+        const int xs = seg_live ? (seg * W) / nseg : W;
+        const int xe = seg_live ? ((seg + 1) * W) / nseg : W;
         const int seg_max = (W + nseg - 1) / nseg;
         uint32_t wb[9][2];  // bf16 weights of channels 4g..4g+3, two per word
 #pragma unroll
@@ -784,18 +788,23 @@ __global__ void __launch_bounds__(kRThreads, 1)
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------ epilogue (warps 13-16)
+        // ------------------------------------------------ epilogue (warps 12-19)
+        // Two warps per TMEM lane quarter q, taking alternate 32-column
+        // chunks: twice the TMEM loads in flight of one warp per quarter (a
+        // warp's chain tcgen05.ld -> staging -> TMA store sets the pace), with
+        // one 4 KB staging buffer each (the same 32 KB as two per warp).
         const int q = warp & 3;
         const int ew = warp - kREpiWarp0;
-        uint8_t *stg = sStage + ew * (2 * 4096);
-        int acc = 0, buf = 0;
+        const int c_first = (ew >> 2) * 32;  // this warp's first column chunk; it then takes every second
+        uint8_t *sb = sStage + ew * 4096;
+        int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = tb; tile < te; ++tile) {
             bool tok = true;
             if (lane == 0) tok = bounded_wait(&tfull[acc], acc_phase, w, SITE_DW_TFULL);
             __syncwarp();
-            // The 4 epilogue warps decide together and leave the wait joined.
-            if (!named_bar_and(3, 128, tok)) break;
+            // The epilogue warps decide together and leave the wait joined.
+            if (!named_bar_and(3, 32 * kREpiWarps, tok)) break;
             tc_fence_after();
             int n, y0, y1, lo, hi;
             tile_rows(p, tile, n, y0, y1, lo, hi);
@@ -804,31 +813,30 @@ __global__ void __launch_bounds__(kRThreads, 1)
             const long long row0 = (static_cast<long long>(n) * H + y0) * W + q * 32;
             const uint32_t tb_addr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                      static_cast<uint32_t>(acc * ncols);
-            // The TMEM load of chunk c + 32 is issued as soon as chunk c sits
-            // in the staging buffer, so its latency overlaps the store of c.
+            // The TMEM load of the next chunk is issued as soon as the current
+            // one sits in the staging buffer, so its latency overlaps the store.
             uint32_t r[32];
-            if (nv > 0) {
-                if (Cout >= 32)
-                    tmem_ld32(tb_addr, r);
+            if (nv > 0 && c_first < Cout) {
+                if (Cout - c_first >= 32)
+                    tmem_ld32(tb_addr + c_first, r);
                 else
-                    tmem_ld16(tb_addr, *reinterpret_cast<uint32_t (*)[16]>(&r[0]));
+                    tmem_ld16(tb_addr + c_first, *reinterpret_cast<uint32_t (*)[16]>(&r[0]));
             }
-            for (int c = 0; c < Cout && nv > 0; c += 32) {
+            for (int c = c_first; c < Cout && nv > 0; c += 64) {
                 tmem_ld_wait(r);
-                if (lane == 0) bulk_wait_read<1>();
+                if (lane == 0) bulk_wait_read<0>();  // the previous store has read the buffer
                 __syncwarp();
-                uint8_t *sb = stg + buf * 4096;
 #pragma unroll
                 for (int ch = 0; ch < 8; ++ch) {
                     const int pos = ch ^ (lane & 7);
                     *reinterpret_cast<uint4 *>(sb + lane * 128 + pos * 16) =
                         make_uint4(r[4 * ch], r[4 * ch + 1], r[4 * ch + 2], r[4 * ch + 3]);
                 }
-                if (c + 32 < Cout) {
-                    if (Cout - c - 32 >= 32)
-                        tmem_ld32(tb_addr + c + 32, r);
+                if (c + 64 < Cout) {
+                    if (Cout - c - 64 >= 32)
+                        tmem_ld32(tb_addr + c + 64, r);
                     else
-                        tmem_ld16(tb_addr + c + 32, *reinterpret_cast<uint32_t (*)[16]>(&r[0]));
+                        tmem_ld16(tb_addr + c + 64, *reinterpret_cast<uint32_t (*)[16]>(&r[0]));
                 }
                 if (nv == 32) {
                     fence_proxy_async_smem();
@@ -863,7 +871,6 @@ __global__ void __launch_bounds__(kRThreads, 1)
                     }
                     __syncwarp();
                 }
-                buf ^= 1;
                 __syncwarp();  // joined again before the next aligned tcgen05.ld
             }
             tc_fence_before();
@@ -892,7 +899,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
 // MMA block, a channel count its thread mapping does not divide, or no ring
 // that fits shared memory beside the block's weights).
 int dw_rows_per_tile(int W, int Cin, int pc, int smem_optin) {
-    int rt = (W <= kBM && kRProd % (Cin / 4) == 0) ? kBM / W : 0;
+    int rt = (W <= kBM && Cin / 4 <= kRProd) ? kBM / W : 0;
     if (rt > (kRingMax - 2) / 2) rt = (kRingMax - 2) / 2;
     while (rt > 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total > smem_optin) --rt;
     return (rt >= 1 && dw_row_layout(W, Cin, pc, 2 * rt + 2).total <= smem_optin) ? rt : 0;

@@ -148,6 +148,10 @@ int gru_stack_launch(int layers, int T, int batch, int hidden, int reset_before,
 
 int dwsep_launch(int N, int H, int W, int Cin, int Cout, const uint16_t *x, const uint16_t *dw,
                  const uint16_t *pw, float *out, DeviceState &ds, cudaStream_t s);
+// The 3x3 depthwise stage alone: y (NHWC bf16) from x (NHWC bf16) and dw
+// [3][3][C]; C a multiple of 8, pointers 16-byte aligned (checked by the caller).
+int depthwise_launch(int N, int H, int W, int C, const uint16_t *x, const uint16_t *dw, uint16_t *y,
+                     const DeviceState &ds, cudaStream_t s);
 // out[4]: kernel (0 row ring, 1 per-pixel), image rows per tile, channel blocks, block width.
 int dwsep_plan(int W, int Cin, int Cout, int smem_optin, int *out);
 

@@ -66,6 +66,7 @@ def load():
         lib.isam_gru_forward_reset_before.argtypes = [i, i, i, P, P, P, P, P, P]
         lib.isam_gru_forward_stack.argtypes = [i, i, i, i, i, P, P, P, P, P, P]
         lib.isam_dwsep_conv.argtypes = [i, i, i, i, i, P, P, P, P]
+        lib.isam_depthwise_conv3x3.argtypes = [i, i, i, i, P, P, P]
         lib.isam_dwsep_plan_info.argtypes = [i, i, i, P]
         lib.isam_dwsep_plan_for.argtypes = [i, i, i, i, P]
         lib.isam_gemm_plan_for.argtypes = [i, i, i, i, i, f, i, i, P, P]
@@ -76,7 +77,7 @@ def load():
                      "isam_gemm_mxfp8", "isam_gemm_grouped_mxfp8",
                      "isam_gru_forward", "isam_gru_forward_reset_before",
                      "isam_gru_forward_stack",
-                     "isam_dwsep_conv", "isam_dwsep_plan_info", "isam_dwsep_plan_for",
+                     "isam_dwsep_conv", "isam_dwsep_plan_info", "isam_dwsep_plan_for", "isam_depthwise_conv3x3",
                      "isam_gru_plan_info", "isam_gru_plan_for", "isam_gemm_plan_for"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
@@ -320,6 +321,17 @@ def dwsep_conv(N, H, W, Cin, Cout, x, dw_w, pw_w, out) -> None:
     _dev(out, torch.float32, N * H * W * Cout, "out")
     _use_current_stream(lib)
     check(lib.isam_dwsep_conv(N, H, W, Cin, Cout, _ptr(x), _ptr(dw_w), _ptr(pw_w), _ptr(out)))
+
+
+def depthwise_conv3x3(N, H, W, C, x, dw_w, y) -> None:
+    """isam_depthwise_conv3x3: NHWC 3x3 depthwise (pad 1), bf16 in and out."""
+    import torch
+    lib = load()
+    _dev(x, torch.bfloat16, N * H * W * C, "x")
+    _dev(dw_w, torch.bfloat16, 9 * C, "dw_w")
+    _dev(y, torch.bfloat16, N * H * W * C, "y")
+    _use_current_stream(lib)
+    check(lib.isam_depthwise_conv3x3(N, H, W, C, _ptr(x), _ptr(dw_w), _ptr(y)))
 
 
 _DWSEP_PLAN_KEYS = ("kernel", "rows_per_tile", "blocks", "block_cout")

@@ -100,8 +100,13 @@ BLOCKED = [
     ((1, 6, 56, 192, 256), (0, 1, 2, 128)),    # row ring, one row per tile, 2 blocks
     ((1, 4, 56, 256, 256), (1, 0, 4, 64)),     # per-pixel kernel, 4 blocks
     ((1, 3, 130, 256, 256), (1, 0, 4, 64)),    # wider than one MMA block
-    ((2, 3, 11, 208, 80), (1, 0, 2, 48)),      # 48-wide blocks (a 16-column TMEM tail)
-    ((2, 4, 33, 144, 208), (1, 0, 2, 112)),
+    ((2, 3, 130, 208, 80), (1, 0, 2, 48)),     # 48-wide blocks (a 16-column TMEM tail)
+    ((2, 4, 130, 144, 208), (1, 0, 2, 112)),
+    # the row ring with idle producer threads (52 and 36 channel groups do
+    # not divide the producers; the threads past the last whole segment only
+    # join the barriers)
+    ((2, 3, 11, 208, 80), (0, 5, 1, 80)),
+    ((2, 4, 33, 144, 208), (0, 1, 1, 208)),
     ((3, 2, 1, 256, 256), (0, 15, 2, 128)),    # one-pixel-wide images
 ]
 
@@ -146,3 +151,79 @@ def test_dwsep_unsupported_rejected():
 def test_dwsep_plan_on_the_device_matches_the_host_plan():
     for (W, cin, cout) in [(56, 128, 256), (56, 256, 256), (8, 256, 256), (130, 48, 16)]:
         assert isam.dwsep_plan(W, cin, cout) == isam.dwsep_plan(W, cin, cout, smem_optin=232448)
+
+
+# ---- the depthwise factor alone (isam_depthwise_conv3x3) and the unfused
+# schedule: depthwise to memory, then the pointwise factor through isam_gemm
+
+def run_depthwise(x, dw):
+    import torch
+    N, H, W, C = x.shape
+    y = torch.full((N * H * W * C + 2 * 64,), float("nan"), dtype=torch.bfloat16, device="cuda")
+    yv = y[64:64 + N * H * W * C]
+    isam.depthwise_conv3x3(N, H, W, C, dev_bf16(x), dev_bf16(dw), yv)
+    isam.sync()
+    guard = y.float().cpu().numpy()
+    assert np.isnan(guard[:64]).all() and np.isnan(guard[-64:]).all(), "write outside y"
+    return yv, yv.float().cpu().numpy().reshape(N, H, W, C)
+
+
+def identity_pw(C):
+    return synth.to_bf16_bits(np.eye(C))
+
+
+@pytest.mark.parametrize("shape", [(1, 1, 1, 8), (2, 5, 7, 16), (1, 9, 130, 24), (3, 4, 33, 64), (2, 13, 11, 128),
+                                   (32, 56, 56, 128)])
+def test_depthwise_alone_matches_oracle(shape):
+    """The oracle's separable layer with an identity pointwise factor is the
+    depthwise sum itself (each output channel picks one input channel, exactly
+    in fp64); the kernel sums in fp32 and rounds once to bf16 (8 significant
+    bits), so each element is within 2^-8 of its own magnitude and the
+    normalised error is at most 2^-8 (plus fp32 summation, far below)."""
+    N, H, W, C = shape
+    x, dw, _ = synth.dwsep_operands(N, H, W, C, C, seed=sum(shape) * 17 + C)
+    _, got = run_depthwise(x, dw)
+    ref = oracle.dwsep(x, dw, identity_pw(C))
+    assert nmax_err(got, ref) <= 2.0 ** -8 + 1e-6, shape
+
+
+def test_depthwise_alone_integer_exact():
+    """Integer data whose window sums fit bf16's 8-bit significand: exact."""
+    N, H, W, C = 2, 6, 9, 32
+    x = synth.to_bf16_bits(synth.integers(601, N * H * W * C, -3, 3).reshape(N, H, W, C))
+    dw = synth.to_bf16_bits(synth.integers(602, 9 * C, -2, 2).reshape(3, 3, C))
+    _, got = run_depthwise(x, dw)
+    ref = oracle.dwsep(x, dw, identity_pw(C))
+    assert np.array_equal(got.astype(np.float64), ref)
+
+
+def test_unfused_schedule_matches_oracle_and_fused_layer():
+    """Depthwise to memory, then isam_gemm(M = N*H*W, N = Cout, K = Cin,
+    A = y, B = pw_w): the separable layer within the tolerance, and equal to
+    the fused kernel up to summation order (both feed bf16 depthwise sums to
+    fp32-accumulating tensor cores)."""
+    import torch
+    N, H, W, Cin, Cout = 4, 14, 14, 128, 256
+    x, dw, pw = synth.dwsep_operands(N, H, W, Cin, Cout, seed=611)
+    yv, _ = run_depthwise(x, dw)
+    M = N * H * W
+    out = Guarded(M * Cout)
+    isam.gemm(M, Cout, Cin, 0, 0, 1.0, yv, dev_bf16(pw), 0.0, out.t)
+    isam.sync()
+    assert out.guards_intact()
+    unfused = out.numpy().reshape(N, H, W, Cout)
+    ref = oracle.dwsep(x, dw, pw)
+    assert nmax_err(unfused, ref) <= TOL
+    fused = run_dwsep(x, dw, pw)
+    assert nmax_err(unfused, fused) <= 1e-5
+
+
+def test_depthwise_rejects_bad_arguments():
+    import torch
+    lib = isam.load()
+    z = torch.zeros(4096, dtype=torch.bfloat16, device="cuda")
+    p = isam._ptr
+    assert lib.isam_depthwise_conv3x3(1, 2, 2, 12, p(z), p(z), p(z)) == isam.ISAM_ERR_UNSUPPORTED  # C % 8
+    assert lib.isam_depthwise_conv3x3(1, 2, 2, 16, p(z[1:]), p(z), p(z)) == isam.ISAM_ERR_UNSUPPORTED
+    assert lib.isam_depthwise_conv3x3(0, 2, 2, 16, p(z), p(z), p(z)) == isam.ISAM_ERR_INVALID_ARG
+    assert lib.isam_depthwise_conv3x3(1, 2, 2, 16, None, p(z), p(z)) == isam.ISAM_ERR_INVALID_ARG
