@@ -67,10 +67,18 @@ struct Cfg {
     static constexpr int kCW = BN < 32 ? BN : 32;  // epilogue column chunk
 };
 
-// Epilogue shared memory: split-K partial tile, or per-warp staging (TMA
+// Split-K partial rows of 128 columns go to their owner through a per-warp
+// transpose (whole row segments per remote store); narrower tiles push each
+// thread's row directly.
+__host__ __device__ constexpr bool xpose_push(int BN) { return BN >= 128; }
+
+// Epilogue shared memory: split-K partial tile (128 x BN fp32 received
+// slices; rows padded by 4 floats for the direct push, plus a 4 KB transpose
+// buffer per epilogue warp for the transposed one), or per-warp staging (TMA
 // path: 2 x 4 KB per epilogue warp; plain path: a 32 x 33 fp32 transpose).
 __host__ __device__ inline size_t epi_bytes(int BN, int split) {
-    if (split > 1) return static_cast<size_t>(kBM) * (BN + 4) * 4;
+    if (split > 1)
+        return xpose_push(BN) ? static_cast<size_t>(kBM) * BN * 4 + 4 * 4096 : static_cast<size_t>(kBM) * (BN + 4) * 4;
     return BN >= 32 ? static_cast<size_t>(4) * 2 * 4096 : static_cast<size_t>(4) * 32 * 33 * 4;
 }
 
@@ -132,7 +140,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&tfull[i], 1);
             mbar_init(&tempty[i], 4);
         }
-        mbar_init(red_full, kBM);
+        // Direct push: one arrival per partial row (S sources x 128 / S rows).
+        // Transposed push: one per (source CTA, epilogue warp) whose 32 rows
+        // meet this CTA's slice of the tile.
+        int red_arrivals = xpose_push(BN) ? 0 : kBM;
+        if (S > 1 && xpose_push(BN)) {
+            const int rp = kBM / S;
+            for (int q = 0; q < 4; ++q)
+                if (q * 32 < static_cast<int>(rank + 1) * rp && q * 32 + 32 > static_cast<int>(rank) * rp)
+                    red_arrivals += S;
+        }
+        mbar_init(red_full, red_arrivals > 0 ? red_arrivals : 1);
         mbar_init(red_free, S);
         for (int i = 0; i < 8; ++i) mbar_init(&cbar[i], 1);
         mbar_init(done, 4);
@@ -299,7 +317,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------ epilogue (warps 2-5)
         const int ew = warp - 2;          // 0..3
         const int q = warp & 3;           // TMEM lane quadrant this warp may read
-        const int row_local = q * 32 + lane;
         const bool use_tma = (S == 1) && (BN >= 32) && (p.tma_c != 0);
         const bool load_c = use_tma && (p.beta != 0.0f);
         uint8_t *stg = reinterpret_cast<uint8_t *>(ebuf) + ew * 8192;  // TMA path: 2 x 4 KB
@@ -438,12 +455,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             } else {
                 // Split-K, push style: row slice o (128 / S rows) of the tile is
-                // reduced by cluster rank o.  Every epilogue thread stores its
-                // partial row straight into the owner's shared memory and then
-                // release-arrives on the owner's red_full (128 arrivals per
-                // tile: S sources x 128 / S rows); each owner sums the S slices
-                // it received in rank order (deterministic) and stores its rows
-                // of C.
+                // reduced by cluster rank o.  Narrow tiles: every epilogue
+                // thread stores its partial row straight into the owner's
+                // shared memory and release-arrives on the owner's red_full
+                // (128 arrivals per tile: S sources x 128 / S rows).  128-column
+                // tiles: each epilogue warp transposes its 32 partial rows
+                // through a 4 KB shared-memory buffer, 32 columns at a time, so
+                // that every remote store instruction writes four 128-byte row
+                // segments of the owner's slot instead of one 16-byte piece of
+                // 32 rows, then release-arrives once on each owner of its rows.
+                // Each owner sums the S slices it received in rank order
+                // (deterministic) and stores its rows of C.
                 // A wait that runs out skips the work but still reaches the
                 // epilogue barrier below, which makes the decision to stop
                 // uniform across the four warps.
@@ -451,7 +473,52 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (iter > 0)
                     wok = warp_wait<true>(red_free, static_cast<uint32_t>((iter - 1) & 1), w, SITE_EPI_REDFREE);
                 const int rows_per = kBM / S;
-                if (wok) {
+                constexpr bool kXpose = xpose_push(BN);
+                constexpr int EP = kXpose ? BN : BN + 4;  // row pitch of the received slices
+                if (kXpose && wok) {
+                    uint8_t *sx = reinterpret_cast<uint8_t *>(ebuf) + static_cast<size_t>(kBM) * BN * 4 + ew * 4096;
+                    // Piece j (16 bytes) of row r sits at slot j ^ (r & 7) of
+                    // the row's 128 bytes: writes by row and reads by row
+                    // segment both take the minimum of four wavefronts.
+                    const int rr = lane >> 3;  // row segment of this lane in a read-back instruction
+                    const int jj = lane & 7;   // its 16-byte piece
+#pragma unroll 1
+                    for (int c = 0; c < BN; c += 32) {
+                        uint32_t r[32];
+                        tmem_ld32(tbase + c, r);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            *reinterpret_cast<uint4 *>(sx + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                                make_uint4(r[4 * j], r[4 * j + 1], r[4 * j + 2], r[4 * j + 3]);
+                        __syncwarp();
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int row = i * 4 + rr;  // 0..31 within this warp's rows
+                            const uint4 v = *reinterpret_cast<const uint4 *>(sx + row * 128 + ((jj ^ (row & 7)) << 4));
+                            const int rl = q * 32 + row;  // row of the tile
+                            const uint32_t owner = static_cast<uint32_t>(rl / rows_per);
+                            const int ro = rl - static_cast<int>(owner) * rows_per;
+                            const uint32_t dst = mapa_shared(
+                                smem_u32(ebuf + static_cast<size_t>(static_cast<int>(rank) * rows_per + ro) * EP + c +
+                                         jj * 4),
+                                owner);
+                            st_dsmem_f4(dst, make_float4(__uint_as_float(v.x), __uint_as_float(v.y),
+                                                         __uint_as_float(v.z), __uint_as_float(v.w)));
+                        }
+                        __syncwarp();  // the buffer is read back before the next chunk overwrites it
+                    }
+                    // The barrier orders every lane's remote stores before lane
+                    // 0's release-arrive on each owner of this warp's rows.
+                    if (lane == 0) {
+                        const int o_first = (q * 32) / rows_per;
+                        const int o_last = (q * 32 + 31) / rows_per;
+                        for (int o = o_first; o <= o_last; ++o) mbar_arrive_remote(red_full, static_cast<uint32_t>(o));
+                    }
+                    __syncwarp();
+                }
+                if (!kXpose && wok) {
+                    const int row_local = q * 32 + lane;
                     const uint32_t owner = static_cast<uint32_t>(row_local / rows_per);
                     const int rr = row_local - static_cast<int>(owner) * rows_per;
                     const uint32_t dst = mapa_shared(
@@ -501,7 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
                         for (int r = 0; r < S; ++r) {
                             const float4 v = *reinterpret_cast<const float4 *>(
-                                ebuf + static_cast<size_t>(r * rows_per + rr) * (BN + 4) + c4);
+                                ebuf + static_cast<size_t>(r * rows_per + rr) * EP + c4);
                             s.x += v.x;
                             s.y += v.y;
                             s.z += v.z;
