@@ -70,7 +70,7 @@ def test_gemm_8192_cube_beta1_sampled_rows():
     assert nmax_err(got[rows], ref) <= TOL
 
 
-FORCED = [(16, 1), (32, 2), (64, 4), (128, 8), (256, 1), (128, 1), (64, 2), (16, 8)]
+FORCED = [(16, 1), (32, 2), (64, 4), (128, 8), (256, 1), (128, 1), (64, 2), (16, 8), (128, 2), (128, 4)]
 
 
 @pytest.mark.parametrize("tA,tB", [(0, 0), (1, 0), (0, 1), (1, 1)], ids=["NN", "TN", "NT", "TT"])
@@ -119,6 +119,23 @@ def test_gemm_beta_zero_does_not_read_c():
     got = run_gemm(M, N, K, 0, 0, 1.0, 0.0, A, B, fill=np.nan)
     assert np.isfinite(got).all()
     assert nmax_err(got, oracle.gemm(M, N, K, 0, 0, 1.0, A, B)) <= TOL
+
+
+@pytest.mark.parametrize("split", [2, 4, 8])
+def test_gemm_split_k_several_tiles_per_cluster(split, monkeypatch):
+    """128-column split tiles (partial rows pushed through the per-warp
+    transpose) with more tiles than resident clusters, so every cluster runs
+    several tiles and reuses its reduction slots; ragged M, N and K, integer
+    data exact."""
+    monkeypatch.setenv("ISAM_FORCE_TILE", f"128,{split},0")
+    M, N, K = 5000, 136, 520
+    A, B, C0 = synth.gemm_operands(M, N, K, 0, 0, seed=300 + split, dist="int4", beta_c=True)
+    got = run_gemm(M, N, K, 0, 0, 2.0, -1.0, A, B, C0=C0)
+    ref = oracle.gemm(M, N, K, 0, 0, 2.0, A, B, -1.0, C0)
+    assert np.array_equal(got.astype(np.float64), ref)
+    plan = isam.gemm_plan(M, N, K, 0, 0, -1.0)
+    assert (plan["BN"], plan["split"]) == (128, split)
+    assert plan["grid"] // split < 40 * 2  # fewer resident clusters than tiles
 
 
 def test_gemm_split_k_deterministic(monkeypatch):
