@@ -23,8 +23,8 @@ hot_path: the other rows measured in the same run (not part of value): the
          depthwise layer (32x56x56, 128 -> 256: GB/s vs HBM).
 cpu_baseline: the fp64 oracle on the host cores, on a row sample of the sweep.
 
---impl reference times the oracle itself (the only reference this build has)
-on the same workload's row sample, K steps after W warm-up steps.
+--impl reference times the oracle itself (the paper publishes no code to run
+instead) on the same workload's row sample, K steps after W warm-up steps.
 Multi-GPU (torchrun): every rank runs the whole sweep on its own GPU with no
 collective on the data path (weak scaling); timing is the max over ranks.
 """
