@@ -176,31 +176,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int kg_end = static_cast<int>((static_cast<long long>(rank + 1) * p.kg_total) / S);
     const int num_tiles = p.m_tiles * p.n_tiles;
 
-    // Dependent launch: this grid may be resident while the previous kernel on
-    // the stream finishes.  Before waiting for it, pull this CTA's first
-    // stages into L2 (a prefetch only fills L2, the point of coherence, so it
-    // cannot observe stale data); every global load or store comes after.
+    // Dependent launch: this grid's CTAs may start (barriers, TMEM, tensor
+    // maps) on SMs the previous kernel on the stream leaves free, and wait
+    // here until it has finished; every global load or store comes after.
+    // (An L2 prefetch of the first stages issued before the wait made the
+    // per-call sweep 3.8% slower: it delays the first real load of every CTA
+    // that starts only after the previous kernel has drained.)
     griddep_launch_dependents();
-    if (threadIdx.x == 0 && cluster_id < num_tiles) {
-        int mt, nt;
-        tile_coords(cluster_id, p.m_tiles, p.n_tiles, p.group_m, mt, nt);
-        const int kg_pf = min(kg_end, kg_begin + ST);
-        for (int kg = kg_begin; kg < kg_pf; ++kg)
-            for (int at = 0; at < KA; ++at) {
-                const int k0 = (kg * KA + at) * (F8 ? 2 * kBK : kBK);  // in elements
-                if (A_MN) {
-                    tma_prefetch_l2_2d(&tmA, mt * kBM, k0);
-                    tma_prefetch_l2_2d(&tmA, mt * kBM + 64, k0);
-                } else {
-                    tma_prefetch_l2_2d(&tmA, k0, mt * kBM);
-                }
-                if (B_MN) {
-                    for (int c = 0; c < (BN + 63) / 64; ++c) tma_prefetch_l2_2d(&tmB, nt * BN + c * 64, k0);
-                } else {
-                    tma_prefetch_l2_2d(&tmB, k0, nt * BN);
-                }
-            }
-    }
     __syncwarp();
     griddep_wait();
 

@@ -177,14 +177,6 @@ __device__ __forceinline__ void bulk_wait_all() {
     asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// Prefetches a tensor box into L2 (no shared-memory destination, no barrier).
-__device__ __forceinline__ void tma_prefetch_l2_2d(const void *map, int32_t c0, int32_t c1) {
-    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                     reinterpret_cast<uint64_t>(map)),
-                 "r"(c0), "r"(c1)
-                 : "memory");
-}
-
 // Generic-proxy writes to global memory become visible to later async-proxy
 // (TMA) reads.
 __device__ __forceinline__ void fence_proxy_async_global() {
