@@ -578,9 +578,28 @@ def hot_path_rows(isam, dev, peaks):
                    flush=flush)
     byts = N * Hh * Ww * (Cin * 2 + Cout * 4) + 9 * Cin * 2 + Cin * Cout * 2
     gbs = byts / ms / 1e6
+    # The same layer sustained: a CUDA graph of calls on 8 operand sets in
+    # turn (1 GB per replay, so every call reads its input from HBM, and each
+    # call's output is written back while later calls run), per call.
+    sets = 8
+    xs = [synth.bf16_normal_torch(synth.stream_seed(synth.BASE_SEED, 4, 10 + i), N * Hh * Ww * Cin, dev)
+          for i in range(sets)]
+    ods = [torch.empty(N * Hh * Ww * Cout, dtype=torch.float32, device=dev) for _ in range(sets)]
+    run_sets = lambda: [isam.dwsep_conv(N, Hh, Ww, Cin, Cout, xs[i], dw, pw, ods[i]) for i in range(sets)]
+    run_sets()
+    isam.sync()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        run_sets()
+    ms_rot = timed("dwsep_32x56x56_128_256_rotating", graph.replay, reps=10, warmup=3) / sets
+    del graph
     out["dwsep_32x56x56_128_256"] = {"ms": round(ms, 4), "gbs": round(gbs, 1),
                                      "frac_hbm": round(gbs / peaks["hbm_gbs"], 4),
-                                     "tflops": round(2.0 * N * Hh * Ww * Cin * (9 + Cout) / ms / 1e9, 2)}
+                                     "tflops": round(2.0 * N * Hh * Ww * Cin * (9 + Cout) / ms / 1e9, 2),
+                                     "ms_rotating": round(ms_rot, 4),
+                                     "frac_hbm_rotating": round(byts / ms_rot / 1e6 / peaks["hbm_gbs"], 4),
+                                     "what": "ms: one call after an L2 flush (a 256 MB write); ms_rotating: per call "
+                                             "of a graph of 8 calls on 8 operand sets (1 GB per replay)"}
     # The same layer unfused: the depthwise factor to memory (bf16), then the
     # pointwise factor through isam_gemm (M = N*H*W, N = Cout, K = Cin).
     M = N * Hh * Ww
@@ -595,10 +614,22 @@ def hot_path_rows(isam, dev, peaks):
         isam.gemm(M, Cout, Cin, 0, 0, 1.0, yb, pw, 0.0, od)
     ms_u = timed("dwsep_unfused_32x56x56_128_256", unfused, reps=20, warmup=3, flush=flush)
     bytes_u = byts + 2 * M * Cin * 2  # the intermediate written and read back
+
+    def unfused_sets():
+        for i in range(sets):
+            isam.depthwise_conv3x3(N, Hh, Ww, Cin, xs[i], dw, yb)
+            isam.gemm(M, Cout, Cin, 0, 0, 1.0, yb, pw, 0.0, ods[i])
+    unfused_sets()
+    isam.sync()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        unfused_sets()
+    ms_urot = timed("dwsep_unfused_32x56x56_128_256_rotating", graph.replay, reps=10, warmup=3) / sets
+    del graph, xs, ods
     out["dwsep_unfused_32x56x56_128_256"] = {
         "ms": round(ms_u, 4), "depthwise_ms": round(ms_dw, 4), "pointwise_ms": round(ms_pw, 4),
         "gbs": round(bytes_u / ms_u / 1e6, 1), "frac_hbm": round(bytes_u / ms_u / 1e6 / peaks["hbm_gbs"], 4),
-        "layer_gbs": round(byts / ms_u / 1e6, 1),
+        "layer_gbs": round(byts / ms_u / 1e6, 1), "ms_rotating": round(ms_urot, 4),
         "what": "isam_depthwise_conv3x3 (bf16 intermediate in HBM) then isam_gemm; gbs counts the intermediate's "
                 "round trip, layer_gbs the fused layer's algorithmic bytes"}
     isam.sync()
