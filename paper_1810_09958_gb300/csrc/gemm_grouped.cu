@@ -9,10 +9,10 @@
 // units (Sections 3.3-3.4) applied across a set of matrix multiplications.
 //
 // Per CTA: warp 0 TMA producer, warp 1 single-thread tcgen05.mma issuer into a
-// double-buffered TMEM accumulator, warps 2-5 epilogue moving C through
-// swizzled shared memory with TMA (or plain stores when a row of C is not
-// 16-byte aligned).  Layout (NN/TN/NT/TT) and tile width are per problem; a
-// problem's tensor maps travel in the kernel parameters.
+// double-buffered TMEM accumulator, warps 2-5 epilogue storing C straight
+// from TMEM (16-byte stores, or single floats when a row of C is not 16-byte
+// aligned).  Layout (NN/TN/NT/TT) and tile width are per problem; a problem's
+// tensor maps travel in the kernel parameters.
 #include <algorithm>
 #include <cstdlib>
 #include <cstdio>
@@ -35,7 +35,6 @@ constexpr int kMaxGroup = 64;
 constexpr int kBNMax = 128;
 constexpr int kAStage = kBM * kBK * 2;      // 16 KB
 constexpr int kBStage = kBNMax * kBK * 2;   // 16 KB (either B layout at BN = 128)
-constexpr int kEpiBytes = 4 * 2 * 4096;     // per-warp 2 x 32x32 fp32 staging
 
 enum : uint32_t {
     SITE_G_EMPTY = 0x401,
@@ -52,7 +51,6 @@ struct GroupProblem {
     int a_mn, b_mn, bn;
     int panels;       // 128-row A panels per tile: 1, or 2 (256-row tiles for the heavy problems)
     int fp8;          // E4M3 operands (both K-major): 128-element K atoms
-    int tma_c;        // C rows 16-byte aligned: TMA epilogue
     int tile_start;   // first global tile index of this problem
     float alpha, beta;
     float *C;
@@ -65,7 +63,6 @@ struct GroupParams {
     GroupProblem prob[kMaxGroup];
     CUtensorMap tmA[kMaxGroup];
     CUtensorMap tmB[kMaxGroup];
-    CUtensorMap tmC[kMaxGroup];
 };
 
 // The problem that owns `tile`, searched forward from `i` (a CTA visits its
@@ -88,14 +85,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
     const int ST = p.stages;
     uint8_t *sA = smem;
     uint8_t *sB = smem + static_cast<size_t>(ST) * kAStage;
-    uint8_t *ebuf = sB + static_cast<size_t>(ST) * kBStage;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(ebuf + kEpiBytes);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + static_cast<size_t>(ST) * kBStage);
     uint64_t *full = bars;
     uint64_t *empty = bars + ST;
     uint64_t *tfull = empty + ST;
     uint64_t *tempty = tfull + 2;
-    uint64_t *cbar = tempty + 2;    // [4 warps][2]
-    uint64_t *done = cbar + 8;
+    uint64_t *done = tempty + 2;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(done + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -112,7 +107,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
             mbar_init(&tfull[i], 1);
             mbar_init(&tempty[i], 4);
         }
-        for (int i = 0; i < 8; ++i) mbar_init(&cbar[i], 1);
         mbar_init(done, 4);
         *abort_flag = 0;
         fence_mbar_init();
@@ -341,13 +335,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
         __syncwarp();
     } else {
         // ------------------------------------------------ epilogue (warps 2-5)
-        const int ew = warp - 2;
         const int q = warp & 3;
-        uint8_t *stg = ebuf + ew * 8192;
-        uint64_t *cb = cbar + ew * 2;
-        uint32_t cpar[2] = {0u, 0u};
-        bool cpend[2] = {false, false};
-        int gbuf = 0, acc = 0, pi = 0;
+        // Straight from TMEM to C: lane i holds row i of the warp's 32 rows,
+        // 32 consecutive columns per TMEM load, stored as 16-byte pieces (or
+        // single floats where C's rows are not 16-byte aligned).  No staging
+        // buffer: the 32 KB it took is a seventh ring stage, and the
+        // epilogue, which overlaps the next tile's main loop through the
+        // second accumulator, has time for the scattered stores.
+        int acc = 0, pi = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < p.total_tiles; tile += gridDim.x) {
             pi = find_problem(p, tile, pi);
@@ -355,114 +350,63 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
             const int local = tile - pr.tile_start;
             const int mt = local % pr.m_tiles, nt = local / pr.m_tiles;
             const int col0 = nt * pr.bn;
-            const bool load_c = pr.tma_c && pr.beta != 0.0f;
             const int nch = (pr.bn + 31) / 32;
-            bool ok = true;
-            for (int pn = 0; ok && pn < pr.panels; ++pn) {
-            const int row0 = (mt * pr.panels + pn) * kBM + q * 32;
-            if ((mt * pr.panels + pn) * kBM >= pr.M) {
-                // a second panel wholly below the matrix: nothing to store
-                continue;
-            }
-            if (load_c) {
-                if (lane == 0) {
-                    bulk_wait_read<0>();
-                    const int b = gbuf & 1;
-                    mbar_arrive_expect_tx(&cb[b], 4096);
-                    tma_load_2d(&p.tmC[pi], &cb[b], stg + b * 4096, col0, row0);
-                }
-                cpend[gbuf & 1] = true;
-                __syncwarp();
-            }
-            if (pn == 0) {
-                if (!warp_wait(&tfull[acc], acc_phase, w, SITE_G_TFULL)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-            }
-            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
-                                   static_cast<uint32_t>(acc * 2 * kBNMax + pn * kBNMax);
-            for (int j = 0; j < nch; ++j) {
-                const int b = gbuf & 1;
-                if (load_c && j + 1 < nch) {
-                    if (lane == 0) {
-                        bulk_wait_read<0>();
-                        mbar_arrive_expect_tx(&cb[b ^ 1], 4096);
-                        tma_load_2d(&p.tmC[pi], &cb[b ^ 1], stg + (b ^ 1) * 4096, col0 + (j + 1) * 32, row0);
-                    }
-                    cpend[b ^ 1] = true;
-                }
-                if (!load_c && lane == 0) bulk_wait_read<1>();
-                uint32_t r[32];
-                if (pr.bn - j * 32 >= 32) {
-                    tmem_ld32(tbase + j * 32, r);
-                } else {
-                    uint32_t h[16];
-                    tmem_ld16(tbase + j * 32, h);
+            const bool vec = (pr.N & 3) == 0;
+            if (!warp_wait(&tfull[acc], acc_phase, w, SITE_G_TFULL)) break;
+            tc_fence_after();
+            for (int pn = 0; pn < pr.panels; ++pn) {
+                const int grow = (mt * pr.panels + pn) * kBM + q * 32 + lane;
+                const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                       static_cast<uint32_t>(acc * 2 * kBNMax + pn * kBNMax);
+                for (int j = 0; j < nch; ++j) {
+                    uint32_t r[32];
+                    if (pr.bn - j * 32 >= 32) {
+                        tmem_ld32(tbase + j * 32, r);
+                    } else {
+                        uint32_t h[16];
+                        tmem_ld16(tbase + j * 32, h);
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        r[i] = h[i];
-                        r[16 + i] = 0u;
-                    }
-                }
-                tmem_ld_wait();
-                if (load_c) {
-                    if (!warp_wait(&cb[b], cpar[b], w, SITE_G_CLOAD)) {
-                        ok = false;
-                        break;
-                    }
-                    cpar[b] ^= 1u;
-                    cpend[b] = false;
-                }
-                __syncwarp();
-                uint8_t *sb = stg + b * 4096;
-#pragma unroll
-                for (int ch = 0; ch < 8; ++ch) {
-                    const int pos = ch ^ (lane & 7);
-                    float4 *slot = reinterpret_cast<float4 *>(sb + lane * 128 + pos * 16);
-                    float4 v = make_float4(pr.alpha * __uint_as_float(r[4 * ch]),
-                                           pr.alpha * __uint_as_float(r[4 * ch + 1]),
-                                           pr.alpha * __uint_as_float(r[4 * ch + 2]),
-                                           pr.alpha * __uint_as_float(r[4 * ch + 3]));
-                    if (load_c) {
-                        const float4 cv = *slot;
-                        v.x += pr.beta * cv.x;
-                        v.y += pr.beta * cv.y;
-                        v.z += pr.beta * cv.z;
-                        v.w += pr.beta * cv.w;
-                    }
-                    *slot = v;
-                }
-                const int cbase = col0 + j * 32;
-                if (pr.tma_c) {
-                    fence_proxy_async_smem();
-                    __syncwarp();
-                    if (lane == 0) {
-                        tma_store_2d(&p.tmC[pi], sb, cbase, row0);
-                        bulk_commit();
-                    }
-                } else {
-                    // Rows of C not 16-byte aligned: plain stores, one row per
-                    // iteration, 32 consecutive columns (coalesced).
-                    __syncwarp();
-                    const int col = cbase + lane;
-                    for (int rr = 0; rr < 32; ++rr) {
-                        const int grow = row0 + rr;
-                        if (grow >= pr.M) break;
-                        if (col < pr.N && lane < pr.bn - j * 32) {
-                            const int pos = (lane >> 2) ^ (rr & 7);
-                            float v = *reinterpret_cast<const float *>(sb + rr * 128 + pos * 16 + (lane & 3) * 4);
-                            if (pr.beta != 0.0f) v += pr.beta * pr.C[static_cast<size_t>(grow) * pr.N + col];
-                            pr.C[static_cast<size_t>(grow) * pr.N + col] = v;
+                        for (int i = 0; i < 16; ++i) {
+                            r[i] = h[i];
+                            r[16 + i] = 0u;
                         }
                     }
-                    __syncwarp();
+                    tmem_ld_wait();
+                    if (grow < pr.M) {
+                        float *crow = pr.C + static_cast<size_t>(grow) * pr.N;
+                        const int cbase = col0 + j * 32;
+                        const int cend = min(pr.N, col0 + pr.bn);  // columns of this tile inside C
+#pragma unroll
+                        for (int ch = 0; ch < 8; ++ch) {
+                            const int col = cbase + 4 * ch;
+                            if (col >= cend) break;
+                            float v[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) v[e] = pr.alpha * __uint_as_float(r[4 * ch + e]);
+                            if (vec && col + 3 < cend) {
+                                float4 *dst = reinterpret_cast<float4 *>(crow + col);
+                                if (pr.beta != 0.0f) {
+                                    const float4 cv = *dst;
+                                    v[0] += pr.beta * cv.x;
+                                    v[1] += pr.beta * cv.y;
+                                    v[2] += pr.beta * cv.z;
+                                    v[3] += pr.beta * cv.w;
+                                }
+                                *dst = make_float4(v[0], v[1], v[2], v[3]);
+                            } else {
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    if (col + e >= cend) break;
+                                    float x = v[e];
+                                    if (pr.beta != 0.0f) x += pr.beta * crow[col + e];
+                                    crow[col + e] = x;
+                                }
+                            }
+                        }
+                    }
+                    __syncwarp();  // joined again before the next aligned tcgen05.ld
                 }
-                ++gbuf;
             }
-            }
-            if (!ok) break;
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&tempty[acc]);
@@ -472,9 +416,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
                 acc_phase ^= 1u;
             }
         }
-        for (int b = 0; b < 2; ++b)
-            if (cpend[b] && lane == 0) drain_wait(&cb[b], cpar[b], p.timeout_ns);
-        if (lane == 0) bulk_wait_all<0>();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(done);
@@ -492,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_group_kernel(const __grid_co
 }
 
 size_t group_smem_bytes(int stages) {
-    return 1024 + static_cast<size_t>(stages) * (kAStage + kBStage) + kEpiBytes + (2 * stages + 13) * 8 + 16;
+    return 1024 + static_cast<size_t>(stages) * (kAStage + kBStage) + (2 * stages + 5) * 8 + 16;
 }
 
 std::mutex g_group_mu;
@@ -552,7 +493,6 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
         pr.m_tiles = (d.M + kBM * pr.panels - 1) / (kBM * pr.panels);
         pr.n_tiles = (d.N + pr.bn - 1) / pr.bn;
         pr.kb_total = atoms(order[s]);
-        pr.tma_c = (d.N % 4 == 0) ? 1 : 0;
         pr.tile_start = tiles;
         pr.alpha = d.alpha;
         pr.beta = d.beta;
@@ -578,9 +518,6 @@ int gemm_grouped_launch(int count, const GemmDesc *g, DeviceState &ds, cudaStrea
                                        static_cast<uint32_t>(pr.bn));
             if (rc) return rc;
         }
-        if (pr.tma_c &&
-            (rc = make_tmap_2d_f32(&p.tmC[s], d.C, d.N, d.M, static_cast<uint64_t>(d.N) * 4, 32, 32)))
-            return rc;
     }
     p.total_tiles = tiles;
     int st = 8;
