@@ -49,11 +49,11 @@ METRIC = "GEMM TFLOP/s (tall-skinny sweep) and GRU timesteps/s on 1 GB300; % of 
 WORKLOAD = ("tall-skinny GEMM sweep: (M,K) in {(1760,1760),(2560,2560),(4096,4096),(7680,2560)} "
             "x N in {16,32,64,128} x {NN,TN}; bf16 U[-1,1]; fp32 accumulate/output; beta=0")
 # dram__bytes_read.sum + dram__bytes_write.sum of one gemm_group_kernel launch
-# over the sweep (750135808 + 24974592 bytes), from an ncu capture of the kernel
-# with 256-row tiles for the heavy problems and per-tile register copies of the
-# problem fields; None whenever the kernel changes until the counters are
-# taken again.
-TRAFFIC_PER_STEP = 775110400
+# over the sweep (749995520 + 24220928 bytes), from an ncu capture of the kernel
+# with 256-row tiles for the heavy problems, per-tile register copies of the
+# problem fields and C stored straight from TMEM; None whenever the kernel
+# changes until the counters are taken again.
+TRAFFIC_PER_STEP = 774216448
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
